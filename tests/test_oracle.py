@@ -1,0 +1,366 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Every check here is independent of the oracle's own code: closed forms worked
+by hand (tests/golden), the geometric Kneedle definition evaluated in fp64,
+library routines that compute special cases (numpy sort, bincount, matmul),
+exact identities of App. A.3, and an exhaustive error sweep of the routing
+exponential against double-precision exp.
+"""
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_04401_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+# ------------------------------------------------------------------ EXP spec
+def test_exp_error_exhaustive():
+    """EXP within 2 ulp of exp() on every fp32 in [-104, 0] with a normal result."""
+    err, worst = oracle.exp_max_ulp(-104.0, 0.0)
+    assert err <= 2.0, (err, worst)
+
+
+def test_exp_special_values():
+    assert oracle.exp([0.0])[0] == np.float32(1.0)
+    assert oracle.exp([-np.inf])[0] == 0.0
+    assert oracle.exp([-104.5])[0] == 0.0
+    # n < -126 flushes to zero (documented): exp(-88) ~ 6e-39 is below 2^-126
+    assert oracle.exp([-88.0])[0] == 0.0
+    z = np.float32(-87.0)
+    assert abs(float(oracle.exp([z])[0]) - math.exp(float(z))) <= 2 ** -149 * 8 + math.exp(float(z)) * 2 ** -22
+
+
+# ------------------------------------------------------------ Algorithm 1
+def _golden_steps():
+    rows = []
+    with open(os.path.join(GOLDEN, "step_curves.txt")) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith("#"):
+                continue
+            N, m, K, hi, lo, e, k = line.split()
+            rows.append((int(N), int(m), int(K), float(hi), float(lo), int(e), int(k)))
+    return rows
+
+
+@pytest.mark.parametrize("N,m,K,hi,lo,e,k", _golden_steps())
+def test_step_curves(N, m, K, hi, lo, e, k):
+    lg = np.full((1, N), lo, np.float32)
+    lg[0, :m] = hi
+    r = oracle.route(lg, K=K, with_sorted=True)
+    assert r["elbow"][0] == e
+    assert r["k"][0] == k
+
+
+def test_step_curves_any_position():
+    """The step's members need not be the first experts: e = m wherever they sit."""
+    rng = np.random.default_rng(5)
+    for _ in range(50):
+        N = int(rng.choice([16, 64, 128]))
+        m = int(rng.integers(1, N - 1))
+        lg = np.zeros((1, N), np.float32)
+        members = rng.choice(N, size=m, replace=False)
+        lg[0, members] = 5.0
+        r = oracle.route(lg, K=8, with_sorted=True)
+        assert r["elbow"][0] == m
+        assert r["k"][0] == min(m + 1, 8)
+        # ties broken by ascending expert id (reading R3)
+        assert list(r["ids"][0][: min(m, 8)]) == sorted(members)[: min(m, 8)]
+
+
+def test_three_level_closed_form():
+    """Levels A > B > C with counts m1, m2, rest. With beta = p'_B:
+    D peaks at i = m1 (value 1 - beta - x'_{m1}) or at i = m1 + m2 (value
+    1 - x'_{m1+m2}); the first wins iff beta < m2 / (N - 1)."""
+    N = 64
+    cases = 0
+    for m1 in (1, 2, 4):
+        for m2 in (2, 5, 9):
+            for b in np.linspace(-3.0, 3.0, 13):
+                lg = np.full((1, N), -2.0, np.float32)
+                lg[0, :m1] = 6.0
+                lg[0, m1:m1 + m2] = b
+                # beta from the fp64 softmax (levels are exact ratios of exps)
+                a, bb, c = math.exp(6.0), math.exp(float(np.float32(b))), math.exp(-2.0)
+                beta = (bb - c) / (a - c)
+                thr = m2 / (N - 1)
+                if abs(beta - thr) < 1e-4:
+                    continue
+                want = m1 if beta < thr else m1 + m2
+                r = oracle.route(lg, K=64, with_sorted=True)
+                assert r["elbow"][0] == want, (m1, m2, b, beta, thr)
+                cases += 1
+    assert cases > 50
+
+
+def _kneedle_fp64(logits_row):
+    """Kneedle knee in fp64: points (x'_i, p'_i) of the descending curve, knee =
+    the point farthest below the straight line through the first and last
+    points (perpendicular distance via the 2-D cross product)."""
+    l = logits_row.astype(np.float64)
+    p = np.exp(l - l.max())
+    p /= p.sum()
+    order = sorted(range(len(p)), key=lambda j: (-p[j], j))
+    ps = p[order]
+    n = len(ps)
+    xs = np.arange(n) / (n - 1)
+    pn = (ps - ps[-1]) / (ps[0] - ps[-1])
+    (x0, y0), (x1, y1) = (xs[0], pn[0]), (xs[-1], pn[-1])
+    # signed distance, positive below the chord of a descending curve
+    dist = ((x1 - x0) * (y0 - pn) - (xs - x0) * (y0 - y1)) / math.hypot(x1 - x0, y1 - y0)
+    return dist, order, ps
+
+
+def test_bruteforce_small_n():
+    """Tiny N, random logits: the oracle's elbow is the fp64 Kneedle knee, and its
+    sorted order is the fp64 descending order, wherever fp32 cannot flip them."""
+    rng = np.random.default_rng(11)
+    checked = 0
+    for N in (4, 8, 16, 32):
+        lg = (rng.standard_normal((400, N)) * rng.uniform(0.3, 3.0, (400, 1))).astype(np.float32)
+        r = oracle.route(lg, K=N, with_sorted=True)
+        for t in range(lg.shape[0]):
+            dist, order, ps = _kneedle_fp64(lg[t])
+            top2 = np.sort(dist)[-2:]
+            if top2[1] - top2[0] > 1e-5:
+                assert r["elbow"][t] == int(np.argmax(dist))
+                checked += 1
+            gaps = -np.diff(ps)
+            if gaps.min() > 1e-6 * ps[0]:
+                assert list(r["ids"][t]) == order[:N]
+    assert checked > 1000
+
+
+def test_bruteforce_permutations():
+    """All orderings of one multiset of logits give the same elbow and, up to the
+    rounding of the position-ordered softmax sum, the same sorted curve; the ids
+    follow the permutation (the sort is a total order)."""
+    import itertools
+    base = np.array([3.0, 0.5, 1.5, 0.5, -1.0, 2.0], np.float32)
+    N = 8
+    ref = None
+    for perm in itertools.permutations(range(6)):
+        lg = np.full((1, N), -3.0, np.float32)
+        lg[0, list(perm)] = base
+        r = oracle.route(lg, K=N, with_sorted=True)
+        if ref is None:
+            ref = (r["sorted_p"][0].copy(), r["elbow"][0])
+        np.testing.assert_allclose(r["sorted_p"][0], ref[0], rtol=2.0 ** -21)
+        assert r["elbow"][0] == ref[1]
+        want = sorted(range(N), key=lambda j: (-float(lg[0, j]), j))
+        assert list(r["ids"][0]) == want
+
+
+# ------------------------------------------------------ selection and gates
+@pytest.mark.parametrize("N,K", [(64, 8), (128, 8), (64, 1), (16, 16), (128, 3)])
+def test_selection_invariants(N, K):
+    rng = np.random.default_rng(N * 100 + K)
+    lg = synth.boosted_logits(rng, 3000, N)
+    el = oracle.route(lg, K=K, with_sorted=True)
+    tk = oracle.route(lg, K=K, mode=oracle.MODE_TOPK)
+    k = el["k"]
+    assert np.all((1 <= k) & (k <= K))
+    assert np.all(tk["k"] == K)
+    # same sort in both modes: elbow-K is a prefix of top-K (Sec. 2.1)
+    assert np.array_equal(el["ids"], tk["ids"])
+    # capped count follows the elbow (Sec. 2.1, reading R2)
+    assert np.array_equal(k, np.minimum(el["elbow"] + 1, K))
+    # ids are the first K of the descending order; distinct
+    for t in range(0, lg.shape[0], 7):
+        assert len(set(el["ids"][t])) == K
+    # gates: the sorted probabilities for s < k, zero after; non-increasing
+    s = np.arange(K)[None, :]
+    sp = el["sorted_p"][:, :K]
+    assert np.array_equal(el["gates"], np.where(s < k[:, None], sp, 0).astype(np.float32))
+    assert np.array_equal(tk["gates"], sp)
+    assert np.all(np.diff(el["gates"], axis=1) <= 0)
+    # top-K against numpy's fp64 softmax + stable argsort where fp32 cannot reorder
+    l64 = lg.astype(np.float64)
+    p64 = np.exp(l64 - l64.max(1, keepdims=True))
+    p64 /= p64.sum(1, keepdims=True)
+    order = np.argsort(-p64, axis=1, kind="stable")[:, :K + 1]
+    top = np.take_along_axis(p64, order, 1)
+    clear = np.all(-np.diff(top, axis=1) > 1e-5 * top[:, :1], axis=1)
+    assert clear.mean() > 0.5
+    assert np.array_equal(el["ids"][clear], order[clear, :K])
+    np.testing.assert_allclose(tk["gates"], top[:, :K], rtol=3e-6, atol=1e-12)
+    # softmax sums to one within N * 2^-23 (each p_j carries <= 2.5 ulp)
+    assert np.all(np.abs(el["sorted_p"].astype(np.float64).sum(1) - 1.0) <= N * 2.0 ** -23)
+
+
+def test_renorm_gates():
+    rng = np.random.default_rng(3)
+    lg = synth.boosted_logits(rng, 2000, 64)
+    r = oracle.route(lg, K=8, renorm=1)
+    tot = r["gates"].astype(np.float64).sum(1)
+    assert np.all(np.abs(tot - 1.0) <= 8 * 2.0 ** -23)
+    base = oracle.route(lg, K=8)
+    assert np.array_equal(r["k"], base["k"]) and np.array_equal(r["ids"], base["ids"])
+    # k = 1 with renorm: the single gate is exactly 1
+    one = oracle.route(lg, K=1, renorm=1)
+    assert np.all(one["gates"][:, 0] == 1.0)
+
+
+def test_flat_and_degenerate():
+    N = 64
+    # all logits equal: R = 0, k = 1 (documented degenerate case)
+    r = oracle.route(np.full((3, N), 2.5, np.float32), K=8, with_sorted=True)
+    assert np.all(r["k"] == 1) and np.all(r["elbow"] == 0)
+    assert list(r["ids"][0]) == list(range(8))
+    # huge spread: tail probabilities underflow to exactly 0
+    lg = np.full((1, N), -500.0, np.float32)
+    lg[0, 7] = 0.0
+    r = oracle.route(lg, K=8, with_sorted=True)
+    assert r["sorted_p"][0, 0] == 1.0 and np.all(r["sorted_p"][0, 1:] == 0)
+    assert r["k"][0] == 2 and r["ids"][0, 0] == 7
+
+
+# ----------------------------------------------- load balance (App. A.3)
+def test_theorem1_and_corollaries():
+    """Theorem 1 and Corollaries 1-2 hold exactly on the empirical loads of any
+    batch, and q_elb - q_top = delta/(1-delta) (q_top - r) (the proof's identity)."""
+    for seed, N in ((1, 64), (2, 128)):
+        rng = np.random.default_rng(seed)
+        lg = synth.boosted_logits(rng, 4000, N)
+        r = oracle.route(lg, K=8)
+        lb = oracle.load_balance(r["k"], r["ids"], N)
+        d = lb["delta"]
+        assert 0 < d < 1
+        assert lb["l1"] <= lb["l1_bound"] + 1e-12
+        assert lb["max_change"] <= lb["l1_bound"] + 1e-12
+        assert lb["cv2_change"] <= lb["cv2_bound"] + 1e-12
+        R = lb["L_top"] - lb["L_elb"]
+        assert np.all(R >= -1e-15)
+        rr = R / (d * 8)
+        np.testing.assert_allclose(lb["q_elb"] - lb["q_top"], d / (1 - d) * (lb["q_top"] - rr), atol=1e-12)
+        np.testing.assert_allclose(lb["L_top"].sum(), 8.0)
+        np.testing.assert_allclose(lb["L_elb"].sum(), r["k"].mean())
+
+
+# --------------------------------------------------------------- dispatch
+def _check_dispatch(k, ids, N):
+    out = oracle.dispatch(k, ids, N)
+    T, K = ids.shape
+    s = np.arange(K)[None, :]
+    valid = s < k[:, None]
+    e_pairs = ids[valid]
+    t_pairs = np.repeat(np.arange(T), k)
+    # counts and offsets: exclusive scan of the histogram
+    cnt = np.bincount(e_pairs, minlength=N)
+    assert np.array_equal(out["offsets"], np.concatenate([[0], np.cumsum(cnt)]).astype(np.int32))
+    # stable counting sort of the pairs by expert = stable argsort
+    want = t_pairs[np.argsort(e_pairs, kind="stable")]
+    assert np.array_equal(out["perm"], want)
+    pp = out["pair_pos"]
+    assert np.all(pp[~valid] == -1)
+    assert np.array_equal(out["perm"][pp[valid]], t_pairs)
+    assert sorted(pp[valid].tolist()) == list(range(len(t_pairs)))
+    return out
+
+
+def test_dispatch_random():
+    rng = np.random.default_rng(9)
+    for N, K, T in ((64, 8, 5000), (128, 8, 3000), (64, 1, 1000), (8, 8, 300)):
+        ids = np.argsort(rng.random((T, N)), axis=1)[:, :K].astype(np.int32)
+        k = rng.integers(1, K + 1, size=T).astype(np.int32)
+        _check_dispatch(k, ids, N)
+
+
+def test_dispatch_edges():
+    N, K = 64, 8
+    # every token on expert 5 first
+    T = 1000
+    ids = np.tile(np.arange(K, dtype=np.int32), (T, 1))
+    ids[:, 0] = 5
+    ids[:, 5] = 0
+    out = _check_dispatch(np.ones(T, np.int32), ids, N)
+    assert out["offsets"][5] == 0 and out["offsets"][6] == T
+    # empty batch
+    out = _check_dispatch(np.zeros(0, np.int32), np.zeros((0, K), np.int32), N)
+    assert np.all(out["offsets"] == 0)
+    # k = 0 tokens are allowed by the dispatch (no pairs)
+    _check_dispatch(np.zeros(10, np.int32), np.tile(np.arange(K, dtype=np.int32), (10, 1)), N)
+    # invalid: duplicate expert inside a token
+    bad = np.tile(np.arange(K, dtype=np.int32), (2, 1))
+    bad[1, 3] = bad[1, 1]
+    with pytest.raises(ValueError):
+        oracle.dispatch(np.full(2, K, np.int32), bad, N)
+
+
+# ------------------------------------------------------------------ layer
+def _mlp64(xf, wgu, wd, e, I):
+    g = xf @ wgu[e, :I].T
+    u = xf @ wgu[e, I:].T
+    h = g / (1.0 + np.exp(-g)) * u
+    return h @ wd[e].T
+
+
+def _small_layer(seed, T=24, d=64, N=8, I=32):
+    rng = np.random.default_rng(seed)
+    wr, w_hat = synth.router_weights(rng, N, d)
+    x = synth.tokens(rng, T, w_hat)
+    wgu, wd = synth.expert_weights(seed, N, d, I)
+    f = lambda b: synth.bf16_bits_to_f32(b).astype(np.float64)
+    return x, wr, wgu, wd, f(x), f(wr), f(wgu), f(wd)
+
+
+def test_router_logits_vs_matmul():
+    x, wr, *_ , xf, wrf, _, _ = _small_layer(1)
+    lg = oracle.router_logits(x, wr)
+    want = (xf @ wrf.T).astype(np.float32)
+    np.testing.assert_allclose(lg, want, rtol=2 ** -23, atol=1e-30)
+
+
+def test_layer_single_expert_is_dense_swiglu():
+    """K = 1, renorm = 1: each token gets gate 1 on its top expert, so the layer is
+    the dense SwiGLU MLP of that expert (numpy fp64 matmul)."""
+    x, wr, wgu, wd, xf, wrf, wguf, wdf = _small_layer(2)
+    I = wgu.shape[1] // 2
+    out = oracle.layer_rows(x, wr, wgu, wd, K=1, renorm=1)
+    assert np.all(out["k"] == 1) and np.all(out["gates"][:, 0] == 1.0)
+    for t in range(x.shape[0]):
+        want = _mlp64(xf[t:t + 1], wguf, wdf, out["ids"][t, 0], I)[0]
+        np.testing.assert_allclose(out["y"][t], want, rtol=1e-10, atol=1e-12)
+
+
+def test_layer_combine_vs_matmul():
+    """General K: y_t = sum_{s<k_t} g_{t,s} MLP_{ids[t,s]}(x_t), with the residual."""
+    x, wr, wgu, wd, xf, wrf, wguf, wdf = _small_layer(3)
+    I = wgu.shape[1] // 2
+    res = synth.bf16_bits(np.random.default_rng(4).standard_normal(x.shape).astype(np.float32))
+    for mode in (oracle.MODE_ELBOW, oracle.MODE_TOPK):
+        out = oracle.layer_rows(x, wr, wgu, wd, K=4, mode=mode, residual_bits=res)
+        r = oracle.route(out["logits"], K=4, mode=mode)
+        assert np.array_equal(r["k"], out["k"]) and np.array_equal(r["ids"], out["ids"])
+        for t in range(x.shape[0]):
+            want = synth.bf16_bits_to_f32(res[t]).astype(np.float64).copy()
+            for s in range(out["k"][t]):
+                want += float(out["gates"][t, s]) * _mlp64(xf[t:t + 1], wguf, wdf, out["ids"][t, s], I)[0]
+            np.testing.assert_allclose(out["y"][t], want, rtol=1e-10, atol=1e-12)
+    # routed rows are independent: a subset of rows reproduces the same outputs
+    sub = oracle.layer_rows(x, wr, wgu, wd, rows=[5, 0, 17], K=4)
+    full = oracle.layer_rows(x, wr, wgu, wd, K=4)
+    assert np.array_equal(sub["y"], full["y"][[5, 0, 17]])
+
+
+def test_layer_storage_rounding_is_small():
+    """Rounding h and the expert outputs to bf16 (the kernels' storage precision)
+    moves the output by far less than the parity tolerance."""
+    x, wr, wgu, wd, *_ = _small_layer(6, T=16, d=128, N=8, I=64)
+    a = oracle.layer_rows(x, wr, wgu, wd, K=8)["y"]
+    b = oracle.layer_rows(x, wr, wgu, wd, K=8, round_h=True, round_y=True)["y"]
+    assert np.linalg.norm(a - b) / np.linalg.norm(a) < 5e-3
+
+
+def test_synthetic_tokens_have_elbows():
+    """The signal-noise generator (Sec. 2.2) gives a head of boosted experts: the
+    elbow sits at |S_t| for most tokens and mean k is well inside [1, K]."""
+    inp = synth.layer_inputs(T=256, d=256, N=64, I=64, seed=7, with_experts=False)
+    lg = oracle.router_logits(inp["x"], inp["w_router"])
+    r = oracle.route(lg, K=8)
+    assert 3.0 < r["k"].mean() < 8.0
