@@ -1,0 +1,193 @@
+/*
+ * elbow_moe.h - C ABI of the GB300 (sm_103a) elbow-routed MoE layer.
+ *
+ * The method is "Elbow-based MoE Routing" (arxiv 2608.04401): per token, the
+ * router's softmax probabilities are sorted in descending order, a
+ * Kneedle-style elbow e is found on the curve normalised to [0,1] (Alg. 1),
+ * and only k = min(e, K) experts are used instead of a fixed top-K
+ * (Sec. 2.1). This library runs that MoE layer forward on one GPU.
+ *
+ * Conventions for every entry point:
+ *   - All tensor pointers are DEVICE pointers owned by the caller; the library
+ *     allocates no memory and never synchronises the stream (except
+ *     moe_read_device_error, which says so).
+ *   - Tensors are dense, row-major, with the shapes given per argument.
+ *     bf16 tensors are passed as uint16_t bit patterns.
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream). Work is
+ *     enqueued on it and the call returns at once.
+ *   - Every call returns a moe_status and never aborts the process. Argument
+ *     errors are detected on the host before anything is enqueued.
+ *   - Supported shapes: N (experts) in {64, 128}; 1 <= K <= 8 and K <= N;
+ *     T >= 0 tokens (T = 0 is a no-op); for the layer, d_model a multiple of
+ *     256 and the SwiGLU intermediate I a multiple of 128, d, I <= 16384.
+ *   - Pointers must be 16-byte aligned.
+ *
+ * Routing arithmetic is fp32 and fully specified (see elbow_route), so that
+ * routing decisions are reproducible bit for bit by an independent
+ * implementation of the same specification.
+ */
+#ifndef ELBOW_MOE_H
+#define ELBOW_MOE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  MOE_OK = 0,
+  MOE_ERR_INVALID_ARG = 1,    /* null or misaligned pointer, negative size, bad params */
+  MOE_ERR_UNSUPPORTED = 2,    /* shape outside the supported set above */
+  MOE_ERR_WORKSPACE = 3,      /* workspace missing or smaller than the query says */
+  MOE_ERR_CUDA = 4,           /* a CUDA runtime/driver call failed */
+  MOE_ERR_DEVICE_TIMEOUT = 5  /* a kernel gave up a bounded wait (see moe_read_device_error) */
+} moe_status;
+
+typedef enum { MOE_ROUTE_ELBOW = 0, MOE_ROUTE_TOPK = 1 } moe_route_mode;
+
+/* Routing parameters. K: the cap (top-K of the base router, Sec. 2.1).
+ * eps: the epsilon of Alg. 1's normalisation (the paper leaves it unstated;
+ * default 1e-8). mode: ELBOW (k = min(e, K)) or TOPK (k = K, the fixed top-K
+ * baseline of Sec. 3 on the same kernels). renorm: 0 = gates are the selected
+ * experts' softmax probabilities (default); 1 = divided by their sum. */
+typedef struct {
+  int K;
+  float eps;
+  int mode;
+  int renorm;
+} moe_route_params;
+
+/* Human-readable name of a status code (static storage). */
+const char* moe_status_string(moe_status s);
+
+/*
+ * elbow_route - Alg. 1 and the capped selection of Sec. 2.1, per token.
+ *
+ *   logits    [T, N] fp32      router logits l(x)
+ *   k_out     [T]    int32     k = min(e + 1, K) (ELBOW) or K (TOPK), 1 <= k <= K
+ *   ids_out   [T, K] int32     expert ids of the K largest probabilities in
+ *                              descending order (ties: lower id first); all K
+ *                              are written, the first k are the selection
+ *   gates_out [T, K] fp32      p_(s) for s < k, 0 for s >= k (renorm: divided
+ *                              by the sum of the first k, left to right)
+ *
+ * fp32 specification (every operation rounded to nearest even, no
+ * contraction): m = max_j l_j; e_j = EXP(l_j - m) with EXP the library's
+ * Cody-Waite/Taylor exponential (zero below 2^-126); s = balanced tree sum
+ * (v_i += v_{i+h}, h = N/2 .. 1); p_j = e_j * (1/s); sort p descending;
+ * den = (p_max - p_min) + eps; p'_i = (p_(i) - p_min) * (1/den);
+ * x'_i = i/(N-1); D_i = (1 - p'_i) - x'_i (the deviation below the chord of
+ * the descending curve; Alg. 1 prints the sign reversed, which would give
+ * k = 1 always); e = smallest argmax_i D_i. Logits must be finite.
+ */
+moe_status elbow_route(const float* logits, int64_t T, int N, const moe_route_params* rp,
+                       int32_t* k_out, int32_t* ids_out, float* gates_out, void* stream);
+
+/*
+ * moe_dispatch - token-to-expert grouping of the selected (t, s < k_t) pairs,
+ * as the MoE block of App. A.4 sends each token to its selected experts.
+ *
+ *   k        [T]      int32  selected counts (0 <= k_t <= K)
+ *   ids      [T, K]   int32  expert ids (distinct within a token, < N)
+ *   offsets  [N + 1]  int32  exclusive prefix sum of the per-expert counts;
+ *                            offsets[N] = sum_t k_t
+ *   perm     [T * K]  int32  capacity T*K; perm[offsets[e] .. offsets[e+1])
+ *                            are the tokens routed to expert e, ascending
+ *                            (stable); entries from offsets[N] on are untouched
+ *   pair_pos [T, K]   int32  position in perm of pair (t, s), -1 for s >= k_t
+ *   ws       device workspace of at least moe_dispatch_workspace_size bytes
+ * Ids outside [0, N) are not checked on the device: they are undefined
+ * behaviour (elbow_route never produces them).
+ */
+size_t moe_dispatch_workspace_size(int64_t T, int N, int K);
+moe_status moe_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
+                        int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
+                        size_t ws_bytes, void* stream);
+
+/*
+ * moe_layer_forward - one MoE layer forward under elbow routing (Sec. 2,
+ * App. A.4): router logits l = W_r x (bf16 x bf16, fp32 accumulate), routing
+ * as elbow_route, dispatch as moe_dispatch, per-expert SwiGLU
+ *   h = silu(W_gate[e] x) * (W_up[e] x)   (bf16 tensor cores, fp32 accumulate,
+ *                                          h stored as bf16)
+ *   o = W_down[e] h                       (stored as bf16)
+ * and the combine y_t = sum_{s < k_t} g_{t,s} o_{t,s} (+ residual_t), summed
+ * in s order in fp32 and rounded to bf16.
+ *
+ *   x          [T, d]       bf16   tokens
+ *   w_router   [N, d]       bf16   router weight W_r
+ *   w_gate_up  [N, 2I, d]   bf16   rows [0, I) = W_gate[e], rows [I, 2I) = W_up[e]
+ *   w_down     [N, d, I]    bf16   W_down[e]
+ *   residual   [T, d]       bf16   optional (NULL = none); may alias y
+ *   y          [T, d]       bf16   output
+ *   logits_out [T, N] fp32, k_out [T], ids_out [T, K], gates_out [T, K],
+ *   offsets_out [N + 1]            optional copies of the intermediate
+ *                                  results (NULL = not written)
+ *   ws         device workspace of at least moe_layer_workspace_size bytes,
+ *              256-byte aligned; it also holds the device error word read by
+ *              moe_read_device_error.
+ * TOPK mode runs the same kernels with k = K.
+ */
+size_t moe_layer_workspace_size(int64_t T, int d, int N, int I, int K);
+moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const uint16_t* w_gate_up,
+                             const uint16_t* w_down, int64_t T, int d, int N, int I,
+                             const moe_route_params* rp, const uint16_t* residual, uint16_t* y,
+                             float* logits_out, int32_t* k_out, int32_t* ids_out, float* gates_out,
+                             int32_t* offsets_out, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * moe_read_device_error - SYNCHRONISES `stream`, then reads the error word
+ * that the layer's kernels leave in `ws` (they clear it at the start of each
+ * moe_layer_forward). Returns MOE_OK, or MOE_ERR_DEVICE_TIMEOUT if a kernel
+ * gave up a bounded wait on its pipeline barriers (its outputs are then
+ * invalid; the CUDA context stays usable).
+ */
+moe_status moe_read_device_error(const void* ws, void* stream);
+
+/* ---- step-level entry points (the layer's stages, for testing and reuse) ---- */
+
+/* Router logits l = W_r x: x [T, d] bf16, w_router [N, d] bf16 -> logits [T, N]
+ * fp32 (tensor cores, fp32 accumulation). d a multiple of 64. err_word: a
+ * device int32 that receives a nonzero code on a device timeout (may be NULL). */
+moe_status moe_router_logits(const uint16_t* x, const uint16_t* w_router, int64_t T, int d, int N,
+                             float* logits, int32_t* err_word, void* stream);
+
+/* Expert SwiGLU over dispatched rows: for each expert e and each row r in
+ * [offsets[e], offsets[e+1]): h[r] = silu(W_gate[e] xs[r]) * (W_up[e] xs[r]),
+ * with xs [P, d] bf16 the tokens already gathered in dispatch order (P = the
+ * row capacity, >= offsets[N]), h [P, I] bf16. `tile_off` [N + 1] int32 are
+ * the exclusive prefix sums of ceil(count_e / 128) (moe_dispatch's workspace
+ * holds them; see moe_dispatch_tile_offsets). */
+moe_status moe_expert_gate_up(const uint16_t* xs, const uint16_t* w_gate_up, const int32_t* offsets,
+                              const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* h,
+                              int32_t* err_word, void* stream);
+
+/* Expert down projection: o[r] = W_down[e] h[r] for rows of expert e;
+ * h [P, I] bf16 -> o [P, d] bf16. */
+moe_status moe_expert_down(const uint16_t* h, const uint16_t* w_down, const int32_t* offsets,
+                           const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* o,
+                           int32_t* err_word, void* stream);
+
+/* Device pointer, inside a moe_dispatch workspace, of the [N + 1] int32 tile
+ * offsets (exclusive prefix sums of ceil(count_e / 128)) that the last
+ * moe_dispatch on that workspace wrote. */
+const int32_t* moe_dispatch_tile_offsets(const void* ws, int64_t T, int N, int K);
+
+/* Gather rows: xs[r] = x[perm[r]] for r < offsets[N] (x [T, d] bf16,
+ * xs [P, d] bf16, P >= offsets[N]). */
+moe_status moe_gather_rows(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int64_t T,
+                           int64_t P, int d, int N, uint16_t* xs, void* stream);
+
+/* Combine: y_t = sum_{s < k_t} gates[t,s] * o[pair_pos[t,s]] (+ residual_t),
+ * fp32 in s order, rounded to bf16. o [P, d] bf16; residual may be NULL. */
+moe_status moe_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_pos,
+                       const float* gates, const uint16_t* residual, int64_t T, int d, int K,
+                       uint16_t* y, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ELBOW_MOE_H */

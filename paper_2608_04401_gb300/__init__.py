@@ -1,0 +1,266 @@
+"""GB300 (sm_103a) elbow-routed MoE layer: thin Python binding of the C ABI.
+
+Every function here marshals torch CUDA tensors into the C entry points of
+libelbow_moe.so (declared in include/elbow_moe.h) and allocates the outputs
+with torch; all arithmetic runs in the library's CUDA kernels. There is no
+fallback: if the library is missing or a CUDA device is absent, calls raise.
+
+Names follow the C ABI: elbow_route, moe_dispatch, moe_layer_forward, and the
+step-level entry points router_logits, gather_rows, expert_gate_up,
+expert_down, combine.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+__all__ = [
+    "MODE_ELBOW", "MODE_TOPK", "MoeError", "library", "build",
+    "elbow_route", "moe_dispatch", "dispatch_workspace_size", "layer_workspace_size",
+    "moe_layer_forward", "read_device_error", "router_logits", "gather_rows",
+    "expert_gate_up", "expert_down", "combine",
+]
+
+MODE_ELBOW = 0
+MODE_TOPK = 1
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB_PATH = os.path.join(_HERE, "_lib", "libelbow_moe.so")
+_lock = threading.Lock()
+_lib = None
+
+
+class MoeError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        msg = library().moe_status_string(status).decode() if _lib is not None else str(status)
+        super().__init__(f"{where}: {msg}")
+
+
+class RouteParams(ctypes.Structure):
+    _fields_ = [("K", ctypes.c_int), ("eps", ctypes.c_float), ("mode", ctypes.c_int),
+                ("renorm", ctypes.c_int)]
+
+
+def build(force: bool = False) -> str:
+    """Compile libelbow_moe.so in-tree (nvcc, sm_103a)."""
+    from . import buildlib
+    return buildlib.build(force=force)
+
+
+def library():
+    """Load libelbow_moe.so (raises if it has not been built)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(_LIB_PATH):
+            raise RuntimeError(f"{_LIB_PATH} is missing: run paper_2608_04401_gb300.build()")
+        lib = ctypes.CDLL(_LIB_PATH)
+        P, i64, i32, f32, sz = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_float,
+                                ctypes.c_size_t)
+        RP = ctypes.POINTER(RouteParams)
+        sig = {
+            "moe_status_string": ([i32], ctypes.c_char_p),
+            "elbow_route": ([P, i64, i32, RP, P, P, P, P], i32),
+            "moe_dispatch_workspace_size": ([i64, i32, i32], sz),
+            "moe_dispatch": ([P, P, i64, i32, i32, P, P, P, P, sz, P], i32),
+            "moe_dispatch_tile_offsets": ([P, i64, i32, i32], P),
+            "moe_layer_workspace_size": ([i64, i32, i32, i32, i32], sz),
+            "moe_layer_forward": ([P, P, P, P, i64, i32, i32, i32, RP, P, P, P, P, P, P, P, P, sz, P],
+                                  i32),
+            "moe_read_device_error": ([P, P], i32),
+            "moe_router_logits": ([P, P, i64, i32, i32, P, P, P], i32),
+            "moe_expert_gate_up": ([P, P, P, P, i64, i32, i32, i32, P, P, P], i32),
+            "moe_expert_down": ([P, P, P, P, i64, i32, i32, i32, P, P, P], i32),
+            "moe_gather_rows": ([P, P, P, i64, i64, i32, i32, P, P], i32),
+            "moe_combine": ([P, P, P, P, P, i64, i32, i32, P, P], i32),
+        }
+        for name, (args, res) in sig.items():
+            fn = getattr(lib, name)
+            fn.argtypes = args
+            fn.restype = res
+        _lib = lib
+        return lib
+
+
+def _torch():
+    import torch
+    return torch
+
+
+def _p(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    torch = _torch()
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _check(status: int, where: str):
+    if status != 0:
+        raise MoeError(status, where)
+
+
+def _cuda(t, dtype, name):
+    torch = _torch()
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t
+
+
+def _params(K, eps, mode, renorm):
+    return ctypes.byref(RouteParams(int(K), float(eps), int(mode), int(renorm)))
+
+
+def elbow_route(logits, K: int = 8, eps: float = 1e-8, mode: int = MODE_ELBOW, renorm: int = 0,
+                stream=None):
+    """Route fp32 logits [T, N]: returns (k [T] int32, ids [T, K] int32, gates [T, K] fp32)."""
+    torch = _torch()
+    lib = library()
+    _cuda(logits, torch.float32, "logits")
+    T, N = logits.shape
+    k = torch.empty(T, dtype=torch.int32, device=logits.device)
+    ids = torch.empty(T, K, dtype=torch.int32, device=logits.device)
+    gates = torch.empty(T, K, dtype=torch.float32, device=logits.device)
+    _check(lib.elbow_route(_p(logits), T, N, _params(K, eps, mode, renorm), _p(k), _p(ids),
+                           _p(gates), _stream(stream)), "elbow_route")
+    return k, ids, gates
+
+
+def dispatch_workspace_size(T: int, N: int, K: int) -> int:
+    return int(library().moe_dispatch_workspace_size(T, N, K))
+
+
+def moe_dispatch(k, ids, N: int, ws=None, stream=None):
+    """Stable token-to-expert dispatch: returns (offsets [N+1], perm [T*K], pair_pos [T, K],
+    ws). perm is valid up to offsets[N]; ws holds the m-tile offsets."""
+    torch = _torch()
+    lib = library()
+    _cuda(k, torch.int32, "k")
+    _cuda(ids, torch.int32, "ids")
+    T, K = ids.shape
+    dev = ids.device
+    need = dispatch_workspace_size(T, N, K)
+    if ws is None:
+        ws = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
+    offsets = torch.empty(N + 1, dtype=torch.int32, device=dev)
+    perm = torch.empty(max(1, T * K), dtype=torch.int32, device=dev)
+    pair_pos = torch.empty(T, K, dtype=torch.int32, device=dev)
+    _check(lib.moe_dispatch(_p(k), _p(ids), T, N, K, _p(offsets), _p(perm), _p(pair_pos), _p(ws),
+                            ws.numel(), _stream(stream)), "moe_dispatch")
+    return offsets, perm, pair_pos, ws
+
+
+def dispatch_tile_offsets(ws, T: int, N: int, K: int):
+    """The [N+1] m-tile offsets a moe_dispatch left in its workspace (a view)."""
+    torch = _torch()
+    ptr = library().moe_dispatch_tile_offsets(_p(ws), T, N, K)
+    off = ptr - ws.data_ptr()
+    return ws[off: off + 4 * (N + 1)].view(torch.int32)
+
+
+def layer_workspace_size(T: int, d: int, N: int, I: int, K: int) -> int:
+    return int(library().moe_layer_workspace_size(T, d, N, I, K))
+
+
+def moe_layer_forward(x, w_router, w_gate_up, w_down, K: int = 8, eps: float = 1e-8,
+                      mode: int = MODE_ELBOW, renorm: int = 0, residual=None, y=None, ws=None,
+                      return_intermediates: bool = False, stream=None):
+    """One MoE layer forward. x [T, d], w_router [N, d], w_gate_up [N, 2I, d],
+    w_down [N, d, I] (bf16 CUDA tensors). Returns y [T, d] bf16, or
+    (y, dict(logits, k, ids, gates, offsets)) with return_intermediates."""
+    torch = _torch()
+    lib = library()
+    bf = torch.bfloat16
+    for t, n in ((x, "x"), (w_router, "w_router"), (w_gate_up, "w_gate_up"), (w_down, "w_down")):
+        _cuda(t, bf, n)
+    if residual is not None:
+        _cuda(residual, bf, "residual")
+    T, d = x.shape
+    N = w_router.shape[0]
+    I = w_gate_up.shape[1] // 2
+    dev = x.device
+    if y is None:
+        y = torch.empty(T, d, dtype=bf, device=dev)
+    need = layer_workspace_size(T, d, N, I, K)
+    if ws is None:
+        ws = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
+    inter = None
+    if return_intermediates:
+        inter = dict(logits=torch.empty(T, N, dtype=torch.float32, device=dev),
+                     k=torch.empty(T, dtype=torch.int32, device=dev),
+                     ids=torch.empty(T, K, dtype=torch.int32, device=dev),
+                     gates=torch.empty(T, K, dtype=torch.float32, device=dev),
+                     offsets=torch.empty(N + 1, dtype=torch.int32, device=dev))
+    g = (lambda n: _p(inter[n])) if inter else (lambda n: None)
+    _check(lib.moe_layer_forward(_p(x), _p(w_router), _p(w_gate_up), _p(w_down), T, d, N, I,
+                                 _params(K, eps, mode, renorm), _p(residual), _p(y), g("logits"),
+                                 g("k"), g("ids"), g("gates"), g("offsets"), _p(ws), ws.numel(),
+                                 _stream(stream)), "moe_layer_forward")
+    return (y, inter) if return_intermediates else y
+
+
+def read_device_error(ws, stream=None):
+    """Synchronise the stream and raise MoeError if a layer kernel timed out."""
+    _check(library().moe_read_device_error(_p(ws), _stream(stream)), "device")
+
+
+def router_logits(x, w_router, err=None, stream=None):
+    torch = _torch()
+    _cuda(x, torch.bfloat16, "x")
+    _cuda(w_router, torch.bfloat16, "w_router")
+    T, d = x.shape
+    N = w_router.shape[0]
+    out = torch.empty(T, N, dtype=torch.float32, device=x.device)
+    _check(library().moe_router_logits(_p(x), _p(w_router), T, d, N, _p(out), _p(err),
+                                       _stream(stream)), "moe_router_logits")
+    return out
+
+
+def gather_rows(x, perm, offsets, P: int, stream=None):
+    torch = _torch()
+    T, d = x.shape
+    N = offsets.numel() - 1
+    xs = torch.empty(max(P, 1), d, dtype=x.dtype, device=x.device)
+    _check(library().moe_gather_rows(_p(x), _p(perm), _p(offsets), T, P, d, N, _p(xs),
+                                     _stream(stream)), "moe_gather_rows")
+    return xs
+
+
+def expert_gate_up(xs, w_gate_up, offsets, tile_off, err=None, stream=None):
+    torch = _torch()
+    P, d = xs.shape
+    N, I2, _ = w_gate_up.shape
+    h = torch.empty(P, I2 // 2, dtype=torch.bfloat16, device=xs.device)
+    _check(library().moe_expert_gate_up(_p(xs), _p(w_gate_up), _p(offsets), _p(tile_off), P, d, N,
+                                        I2 // 2, _p(h), _p(err), _stream(stream)),
+           "moe_expert_gate_up")
+    return h
+
+
+def expert_down(h, w_down, offsets, tile_off, err=None, stream=None):
+    torch = _torch()
+    P, I = h.shape
+    N, d, _ = w_down.shape
+    o = torch.empty(P, d, dtype=torch.bfloat16, device=h.device)
+    _check(library().moe_expert_down(_p(h), _p(w_down), _p(offsets), _p(tile_off), P, d, N, I,
+                                     _p(o), _p(err), _stream(stream)), "moe_expert_down")
+    return o
+
+
+def combine(o, k, pair_pos, gates, residual=None, stream=None):
+    torch = _torch()
+    T, K = pair_pos.shape
+    d = o.shape[1]
+    y = torch.empty(T, d, dtype=torch.bfloat16, device=o.device)
+    _check(library().moe_combine(_p(o), _p(k), _p(pair_pos), _p(gates), _p(residual), T, d, K,
+                                 _p(y), _stream(stream)), "moe_combine")
+    return y

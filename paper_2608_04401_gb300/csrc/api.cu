@@ -1,0 +1,300 @@
+// C ABI of the elbow-routed MoE layer: argument validation, the workspace
+// layout, and the launch sequence of the layer forward. No allocation, no
+// stream synchronisation (moe_read_device_error excepted, as documented).
+#include <cstring>
+
+#include "common.cuh"
+
+namespace moe {
+cudaError_t launch_elbow_route(const float* logits, int64_t T, int N, int K, float eps,
+                               int topk_mode, int renorm, int32_t* k_out, int32_t* ids_out,
+                               float* gates_out, cudaStream_t stream);
+size_t dispatch_ws_bytes(int64_t T, int N);
+int32_t* dispatch_tile_off(void* ws, int64_t T, int N);
+cudaError_t launch_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
+                            int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
+                            int32_t* offsets_copy, cudaStream_t stream);
+cudaError_t launch_gather(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int N,
+                          int64_t P, int d, uint16_t* xs, int num_sms, cudaStream_t stream);
+cudaError_t launch_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_pos,
+                           const float* gates, const uint16_t* residual, int64_t T, int d, int K,
+                           uint16_t* y, int num_sms, cudaStream_t stream);
+cudaError_t launch_router_gemm(const uint16_t* x, const uint16_t* wr, int64_t T, int d, int N,
+                               float* logits, int32_t* err, int num_sms, cudaStream_t stream);
+cudaError_t launch_gateup_gemm(const uint16_t* xs, const uint16_t* wgu, const int32_t* offsets,
+                               const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* h,
+                               int32_t* err, int num_sms, cudaStream_t stream);
+cudaError_t launch_down_gemm(const uint16_t* h, const uint16_t* wd, const int32_t* offsets,
+                             const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* o,
+                             int32_t* err, int num_sms, cudaStream_t stream);
+}  // namespace moe
+
+namespace {
+
+constexpr int64_t kMaxTokens = int64_t(1) << 28;  // keeps T * K * 8 row counts in int32
+constexpr int kMaxDim = 16384;
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t up256(size_t b) { return (b + 255) & ~static_cast<size_t>(255); }
+
+int sm_count() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+    return 148;
+  return n;
+}
+
+moe_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MOE_OK : MOE_ERR_CUDA; }
+
+moe_status check_route_params(const moe_route_params* rp, int N) {
+  if (!rp) return MOE_ERR_INVALID_ARG;
+  if (rp->mode != MOE_ROUTE_ELBOW && rp->mode != MOE_ROUTE_TOPK) return MOE_ERR_INVALID_ARG;
+  if (rp->renorm != 0 && rp->renorm != 1) return MOE_ERR_INVALID_ARG;
+  if (!(rp->eps >= 0.0f) || rp->eps > 1.0f) return MOE_ERR_INVALID_ARG;
+  if (rp->K < 1 || rp->K > 8 || rp->K > N) return MOE_ERR_UNSUPPORTED;
+  return MOE_OK;
+}
+
+bool supported_n(int N) { return N == 64 || N == 128; }
+
+// Layer workspace layout (every region 256-byte aligned):
+//   header (error word) | logits [T,N] f32 | k [T] | ids [T,K] | gates [T,K]
+//   | offsets [N+1] | dispatch scratch | perm [T*K] | pair_pos [T*K]
+//   | xs [T*K, d] bf16 | h [T*K, I] bf16 | o [T*K, d] bf16
+struct LayerWs {
+  int32_t* err;
+  float* logits;
+  int32_t* k;
+  int32_t* ids;
+  float* gates;
+  int32_t* offsets;
+  void* disp;
+  int32_t* perm;
+  int32_t* pair_pos;
+  uint16_t* xs;
+  uint16_t* h;
+  uint16_t* o;
+  size_t bytes;
+};
+
+LayerWs layer_ws(void* base, int64_t T, int d, int N, int I, int K) {
+  LayerWs w{};
+  char* p = static_cast<char*>(base);
+  size_t off = 0;
+  auto take = [&](size_t b) {
+    char* q = p ? p + off : nullptr;
+    off += up256(b);
+    return q;
+  };
+  const size_t P = static_cast<size_t>(T) * K;
+  w.err = reinterpret_cast<int32_t*>(take(256));
+  w.logits = reinterpret_cast<float*>(take(sizeof(float) * T * N));
+  w.k = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * T));
+  w.ids = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * P));
+  w.gates = reinterpret_cast<float*>(take(sizeof(float) * P));
+  w.offsets = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * (N + 1)));
+  w.disp = take(moe::dispatch_ws_bytes(T, N));
+  w.perm = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * (P > 0 ? P : 1)));
+  w.pair_pos = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * (P > 0 ? P : 1)));
+  w.xs = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * P * d));
+  w.h = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * P * I));
+  w.o = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * P * d));
+  w.bytes = off;
+  return w;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* moe_status_string(moe_status s) {
+  switch (s) {
+    case MOE_OK: return "MOE_OK";
+    case MOE_ERR_INVALID_ARG: return "MOE_ERR_INVALID_ARG: null/misaligned pointer or bad parameter";
+    case MOE_ERR_UNSUPPORTED: return "MOE_ERR_UNSUPPORTED: shape outside the supported set";
+    case MOE_ERR_WORKSPACE: return "MOE_ERR_WORKSPACE: workspace missing or too small";
+    case MOE_ERR_CUDA: return "MOE_ERR_CUDA: a CUDA call failed";
+    case MOE_ERR_DEVICE_TIMEOUT: return "MOE_ERR_DEVICE_TIMEOUT: a kernel gave up a bounded wait";
+  }
+  return "unknown moe_status";
+}
+
+moe_status elbow_route(const float* logits, int64_t T, int N, const moe_route_params* rp,
+                       int32_t* k_out, int32_t* ids_out, float* gates_out, void* stream) {
+  if (T < 0 || T > kMaxTokens) return MOE_ERR_INVALID_ARG;
+  if (!supported_n(N)) return MOE_ERR_UNSUPPORTED;
+  moe_status st = check_route_params(rp, N);
+  if (st != MOE_OK) return st;
+  if (T == 0) return MOE_OK;
+  if (!logits || !k_out || !ids_out || !gates_out) return MOE_ERR_INVALID_ARG;
+  if (!aligned16(logits) || !aligned16(ids_out) || !aligned16(gates_out) ||
+      (reinterpret_cast<uintptr_t>(k_out) & 3u))
+    return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_elbow_route(logits, T, N, rp->K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
+                                             rp->renorm, k_out, ids_out, gates_out,
+                                             static_cast<cudaStream_t>(stream)));
+}
+
+size_t moe_dispatch_workspace_size(int64_t T, int N, int K) {
+  (void)K;
+  if (T < 0 || !supported_n(N)) return 0;
+  return moe::dispatch_ws_bytes(T, N);
+}
+
+const int32_t* moe_dispatch_tile_offsets(const void* ws, int64_t T, int N, int K) {
+  (void)K;
+  if (!ws || T < 0 || !supported_n(N)) return nullptr;
+  return moe::dispatch_tile_off(const_cast<void*>(ws), T, N);
+}
+
+moe_status moe_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
+                        int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
+                        size_t ws_bytes, void* stream) {
+  if (T < 0 || T > kMaxTokens) return MOE_ERR_INVALID_ARG;
+  if (!supported_n(N) || K < 1 || K > 8 || K > N) return MOE_ERR_UNSUPPORTED;
+  if (!offsets || !ws) return MOE_ERR_INVALID_ARG;
+  if (T > 0 && (!k || !ids || !perm || !pair_pos)) return MOE_ERR_INVALID_ARG;
+  if (ws_bytes < moe::dispatch_ws_bytes(T, N)) return MOE_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u)) return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_dispatch(k, ids, T, N, K, offsets, perm, pair_pos, ws, nullptr,
+                                          static_cast<cudaStream_t>(stream)));
+}
+
+size_t moe_layer_workspace_size(int64_t T, int d, int N, int I, int K) {
+  if (T < 0 || d <= 0 || I <= 0 || K < 1 || !supported_n(N)) return 0;
+  return layer_ws(nullptr, T, d, N, I, K).bytes;
+}
+
+moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const uint16_t* w_gate_up,
+                             const uint16_t* w_down, int64_t T, int d, int N, int I,
+                             const moe_route_params* rp, const uint16_t* residual, uint16_t* y,
+                             float* logits_out, int32_t* k_out, int32_t* ids_out, float* gates_out,
+                             int32_t* offsets_out, void* ws, size_t ws_bytes, void* stream) {
+  if (T < 0 || T > kMaxTokens) return MOE_ERR_INVALID_ARG;
+  if (!supported_n(N)) return MOE_ERR_UNSUPPORTED;
+  if (d <= 0 || d > kMaxDim || d % 256 != 0 || I <= 0 || I > kMaxDim || I % 128 != 0)
+    return MOE_ERR_UNSUPPORTED;
+  moe_status st = check_route_params(rp, N);
+  if (st != MOE_OK) return st;
+  const int K = rp->K;
+  if (!ws) return MOE_ERR_WORKSPACE;
+  if (reinterpret_cast<uintptr_t>(ws) & 255u) return MOE_ERR_INVALID_ARG;
+  LayerWs w = layer_ws(ws, T, d, N, I, K);
+  if (ws_bytes < w.bytes) return MOE_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // clear the device error word first, so that a no-op call reads clean
+  if (cudaMemsetAsync(w.err, 0, sizeof(int32_t), s) != cudaSuccess) return MOE_ERR_CUDA;
+  if (T == 0) return MOE_OK;
+  const void* need[] = {x, w_router, w_gate_up, w_down, y};
+  for (const void* p : need)
+    if (!p || !aligned16(p)) return MOE_ERR_INVALID_ARG;
+  if (residual && !aligned16(residual)) return MOE_ERR_INVALID_ARG;
+  if ((logits_out && !aligned16(logits_out)) || (ids_out && !aligned16(ids_out)) ||
+      (gates_out && !aligned16(gates_out)) ||
+      (k_out && (reinterpret_cast<uintptr_t>(k_out) & 3u)) ||
+      (offsets_out && (reinterpret_cast<uintptr_t>(offsets_out) & 3u)))
+    return MOE_ERR_INVALID_ARG;
+
+  float* logits = logits_out ? logits_out : w.logits;
+  int32_t* kk = k_out ? k_out : w.k;
+  int32_t* ids = ids_out ? ids_out : w.ids;
+  float* gates = gates_out ? gates_out : w.gates;
+  const int64_t P = T * K;
+  const int nsm = sm_count();
+
+  cudaError_t e;
+  e = moe::launch_router_gemm(x, w_router, T, d, N, logits, w.err, nsm, s);
+  if (e != cudaSuccess) return MOE_ERR_CUDA;
+  e = moe::launch_elbow_route(logits, T, N, K, rp->eps, rp->mode == MOE_ROUTE_TOPK, rp->renorm, kk,
+                              ids, gates, s);
+  if (e != cudaSuccess) return MOE_ERR_CUDA;
+  e = moe::launch_dispatch(kk, ids, T, N, K, w.offsets, w.perm, w.pair_pos, w.disp, offsets_out, s);
+  if (e != cudaSuccess) return MOE_ERR_CUDA;
+  const int32_t* tile_off = moe::dispatch_tile_off(w.disp, T, N);
+  e = moe::launch_gather(x, w.perm, w.offsets, N, P, d, w.xs, nsm, s);
+  if (e != cudaSuccess) return MOE_ERR_CUDA;
+  e = moe::launch_gateup_gemm(w.xs, w_gate_up, w.offsets, tile_off, P, d, N, I, w.h, w.err, nsm, s);
+  if (e != cudaSuccess) return MOE_ERR_CUDA;
+  e = moe::launch_down_gemm(w.h, w_down, w.offsets, tile_off, P, d, N, I, w.o, w.err, nsm, s);
+  if (e != cudaSuccess) return MOE_ERR_CUDA;
+  e = moe::launch_combine(w.o, kk, w.pair_pos, gates, residual, T, d, K, y, nsm, s);
+  if (e != cudaSuccess) return MOE_ERR_CUDA;
+  return MOE_OK;
+}
+
+moe_status moe_read_device_error(const void* ws, void* stream) {
+  if (!ws) return MOE_ERR_INVALID_ARG;
+  int32_t v = 0;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(s) != cudaSuccess) return MOE_ERR_CUDA;
+  if (cudaMemcpy(&v, ws, sizeof v, cudaMemcpyDeviceToHost) != cudaSuccess) return MOE_ERR_CUDA;
+  return v == 0 ? MOE_OK : MOE_ERR_DEVICE_TIMEOUT;
+}
+
+moe_status moe_router_logits(const uint16_t* x, const uint16_t* w_router, int64_t T, int d, int N,
+                             float* logits, int32_t* err_word, void* stream) {
+  if (T < 0 || T > kMaxTokens) return MOE_ERR_INVALID_ARG;
+  if (!supported_n(N) || d <= 0 || d > kMaxDim || d % 64 != 0) return MOE_ERR_UNSUPPORTED;
+  if (T == 0) return MOE_OK;
+  if (!x || !w_router || !logits || !aligned16(x) || !aligned16(w_router) || !aligned16(logits))
+    return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_router_gemm(x, w_router, T, d, N, logits, err_word, sm_count(),
+                                             static_cast<cudaStream_t>(stream)));
+}
+
+moe_status moe_expert_gate_up(const uint16_t* xs, const uint16_t* w_gate_up, const int32_t* offsets,
+                              const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* h,
+                              int32_t* err_word, void* stream) {
+  if (P < 0 || P > kMaxTokens * 8) return MOE_ERR_INVALID_ARG;
+  if (!supported_n(N) || d <= 0 || d > kMaxDim || d % 64 != 0 || I <= 0 || I > kMaxDim ||
+      I % 128 != 0)
+    return MOE_ERR_UNSUPPORTED;
+  if (P == 0) return MOE_OK;
+  if (!xs || !w_gate_up || !offsets || !tile_off || !h || !aligned16(xs) || !aligned16(w_gate_up) ||
+      !aligned16(h))
+    return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_gateup_gemm(xs, w_gate_up, offsets, tile_off, P, d, N, I, h,
+                                             err_word, sm_count(), static_cast<cudaStream_t>(stream)));
+}
+
+moe_status moe_expert_down(const uint16_t* h, const uint16_t* w_down, const int32_t* offsets,
+                           const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* o,
+                           int32_t* err_word, void* stream) {
+  if (P < 0 || P > kMaxTokens * 8) return MOE_ERR_INVALID_ARG;
+  if (!supported_n(N) || d <= 0 || d > kMaxDim || d % 256 != 0 || I <= 0 || I > kMaxDim ||
+      I % 64 != 0)
+    return MOE_ERR_UNSUPPORTED;
+  if (P == 0) return MOE_OK;
+  if (!h || !w_down || !offsets || !tile_off || !o || !aligned16(h) || !aligned16(w_down) ||
+      !aligned16(o))
+    return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_down_gemm(h, w_down, offsets, tile_off, P, d, N, I, o, err_word,
+                                           sm_count(), static_cast<cudaStream_t>(stream)));
+}
+
+moe_status moe_gather_rows(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int64_t T,
+                           int64_t P, int d, int N, uint16_t* xs, void* stream) {
+  (void)T;
+  if (P < 0 || d <= 0 || d % 8 != 0) return MOE_ERR_INVALID_ARG;
+  if (!supported_n(N)) return MOE_ERR_UNSUPPORTED;
+  if (P == 0) return MOE_OK;
+  if (!x || !perm || !offsets || !xs || !aligned16(x) || !aligned16(xs)) return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_gather(x, perm, offsets, N, P, d, xs, sm_count(),
+                                        static_cast<cudaStream_t>(stream)));
+}
+
+moe_status moe_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_pos,
+                       const float* gates, const uint16_t* residual, int64_t T, int d, int K,
+                       uint16_t* y, void* stream) {
+  if (T < 0 || d <= 0 || d % 8 != 0 || K < 1 || K > 8) return MOE_ERR_INVALID_ARG;
+  if (T == 0) return MOE_OK;
+  if (!o || !k || !pair_pos || !gates || !y || !aligned16(o) || !aligned16(y) ||
+      (residual && !aligned16(residual)))
+    return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_combine(o, k, pair_pos, gates, residual, T, d, K, y, sm_count(),
+                                         static_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

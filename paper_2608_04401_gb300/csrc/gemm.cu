@@ -1,0 +1,455 @@
+// Persistent tcgen05 GEMMs with TMA-fed shared-memory pipelines and TMEM
+// accumulators, for the three contractions of the layer:
+//
+//   kRouter : logits[T, N]  = x[T, d] . W_r[N, d]^T              (fp32 out)
+//   kGateUp : h[P, I]       = silu(xs W_gate[e]^T) * (xs W_up[e]^T), per expert
+//             e over its dispatched rows [offsets[e], offsets[e+1])   (bf16 out)
+//   kDown   : o[P, d]       = h W_down[e]^T, per expert            (bf16 out)
+//
+// Both operands are K-major bf16 tiles of 64 columns (128 bytes) moved by TMA
+// with 128-byte swizzle; the MMA is tcgen05.mma.cta_group::1.kind::f16 with
+// M = 128 and N = BN (64/128 for the router, 256 for the experts), fp32
+// accumulation in TMEM. For kGateUp the 256-row B tile is the 128 gate rows
+// and the matching 128 up rows of the expert, so one accumulator holds both
+// halves of the SwiGLU and the epilogue fuses silu(g) * u.
+//
+// Warp roles (192 threads, one CTA per SM):
+//   warp 0     : TMA producer (one elected lane)
+//   warp 1     : TMEM allocator + MMA issuer (one elected lane)
+//   warps 2..5 : epilogue; warp w reads TMEM lanes [32 (w % 4), +32)
+// Two TMEM accumulators (2 x BN columns) let the epilogue of tile i overlap
+// the main loop of tile i + 1. Tiles are scheduled statically
+// (tile = blockIdx.x + i * gridDim.x); for the grouped modes a tile index maps
+// to (expert, n-block, m-block) through the device-side m-tile prefix sums, so
+// the ragged expert sizes never travel to the host. Consecutive tiles share
+// an expert's weight block (m-block fastest), which keeps it in L2.
+//
+// Every barrier wait is bounded (kWaitLimitNs); a timed-out CTA raises a flag
+// that stops its other roles, drains what it has in flight, frees its TMEM and
+// writes an error code into the caller's error word.
+#include "common.cuh"
+
+namespace moe {
+namespace gemm {
+
+constexpr int BM = 128;
+constexpr int BK = 64;
+constexpr int kThreads = 192;
+enum Mode { kRouter = 0, kGateUp = 1, kDown = 2 };
+
+template <int BN>
+struct Cfg {
+  static constexpr int kABytes = BM * BK * 2;
+  static constexpr int kBBytes = BN * BK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kStages = (192 * 1024) / kStageBytes;
+  static constexpr int kTmemCols = (2 * BN <= 64) ? 64 : (2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512));
+  static constexpr int kBarOff = kStages * kStageBytes;
+  // barriers: full[S], empty[S], tfull[2], tempty[2], drain
+  static constexpr int kNumBars = 2 * kStages + 5;
+  static constexpr int kMiscOff = kBarOff + kNumBars * 8;
+  static constexpr int kTableOff = kMiscOff + 16;
+  static constexpr int kMaxGroups = 128;
+  static constexpr int kSmemBytes = kTableOff + 2 * (kMaxGroups + 1) * 4 + 1024;  // + align slack
+};
+
+struct Args {
+  const int32_t* offsets;   // [G + 1] row offsets per group (grouped modes)
+  const int32_t* tile_off;  // [G + 1] prefix sums of ceil(rows_g / 128)
+  int groups;               // G
+  int64_t m_rows;           // router: T
+  int n_tiles;              // n-blocks per group
+  int k_blocks;             // K / 64
+  int b_rows;               // rows of B per group (2I for gate/up, d for down)
+  int b_half;               // gate/up: I (row offset of the up half)
+  void* out;
+  int64_t ldo;              // output row stride, elements
+  int32_t* err;             // device error word (may be null)
+};
+
+struct Tile {
+  int g, nb, row0, rows;
+};
+
+template <int MODE>
+MOE_DEV Tile decode(int tile, const Args& a, const int* s_off, const int* s_toff) {
+  Tile t;
+  if (MODE == kRouter) {
+    t.g = 0;
+    t.nb = 0;
+    t.row0 = tile * BM;
+    t.rows = static_cast<int>(min_of<int64_t>(BM, a.m_rows - t.row0));
+    return t;
+  }
+  int lo = 0, hi = a.groups;  // s_toff[lo] * n_tiles <= tile < s_toff[hi] * n_tiles
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (s_toff[mid] * a.n_tiles <= tile) lo = mid; else hi = mid;
+  }
+  const int mt = s_toff[lo + 1] - s_toff[lo];
+  const int local = tile - s_toff[lo] * a.n_tiles;
+  const int mb = local % mt;
+  t.g = lo;
+  t.nb = local / mt;
+  t.row0 = s_off[lo] + mb * BM;
+  t.rows = min(BM, s_off[lo + 1] - t.row0);
+  return t;
+}
+
+MOE_DEV float silu(float g) { return g / (1.0f + __expf(-g)); }
+
+template <int MODE, int BN>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                const Args args) {
+  using C = Cfg<BN>;
+  constexpr int S = C::kStages;
+  constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t bar0 = sbase + C::kBarOff;
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };
+  auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * S + a); };
+  auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * S + 2 + a); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * S + 4);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::kMiscOff);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::kMiscOff + 4);
+  int* s_off = reinterpret_cast<int*>(smem + C::kTableOff);
+  int* s_toff = s_off + (C::kMaxGroups + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull_bar(a), 1);
+      mbar_init(tempty_bar(a), 4);
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (MODE != kRouter) {
+    for (int i = threadIdx.x; i <= args.groups; i += kThreads) {
+      s_off[i] = args.offsets[i];
+      s_toff[i] = args.tile_off[i];
+    }
+  }
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&tmA);
+    prefetch_tensormap(&tmB);
+  }
+  if (warp == 1) {
+    __syncwarp();
+    tmem_alloc<C::kTmemCols>(smem_u32(tmem_slot));
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int total = (MODE == kRouter) ? static_cast<int>((args.m_rows + BM - 1) / BM)
+                                      : s_toff[args.groups] * args.n_tiles;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int issued = 0;
+      for (int tile = blockIdx.x; tile < total && !*abort_flag; tile += gridDim.x) {
+        const Tile t = decode<MODE>(tile, args, s_off, s_toff);
+        for (int kb = 0; kb < args.k_blocks; ++kb) {
+          if (!mbar_wait_bounded(empty_bar(stage), phase ^ 1u, abort_flag)) break;
+          const uint32_t a_dst = sbase + stage * C::kStageBytes;
+          const uint32_t b_dst = a_dst + C::kABytes;
+          mbar_arrive_expect_tx(full_bar(stage), C::kStageBytes);
+          tma_load_2d(a_dst, &tmA, full_bar(stage), kb * BK, t.row0);
+          if (MODE == kGateUp) {
+            const int brow = t.g * args.b_rows + t.nb * 128;
+            tma_load_2d(b_dst, &tmB, full_bar(stage), kb * BK, brow);
+            tma_load_2d(b_dst + 128 * BK * 2, &tmB, full_bar(stage), kb * BK, brow + args.b_half);
+          } else {
+            tma_load_2d(b_dst, &tmB, full_bar(stage), kb * BK, t.g * args.b_rows + t.nb * BN);
+          }
+          ++issued;
+          if (++stage == S) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (*abort_flag) {
+        // let the copies this thread started land before the CTA exits
+        int st = stage;
+        uint32_t ph = phase;
+        const int n = issued < S ? issued : S;
+        for (int i = 0; i < n; ++i) {
+          if (--st < 0) { st = S - 1; ph ^= 1u; }
+          const uint64_t t0 = global_timer_ns();
+          while (!mbar_try_wait(full_bar(st), ph) && global_timer_ns() - t0 < 100000000ull) {
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ----------------------------------------------------------------- MMA
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int local = 0;
+      bool issued_any = false;
+      for (int tile = blockIdx.x; tile < total && !*abort_flag; tile += gridDim.x, ++local) {
+        const int acc = local & 1;
+        const uint32_t acc_phase = (local >> 1) & 1;
+        if (!mbar_wait_bounded(tempty_bar(acc), acc_phase ^ 1u, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        bool ok = true;
+        for (int kb = 0; kb < args.k_blocks; ++kb) {
+          if (!mbar_wait_bounded(full_bar(stage), phase, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t a_addr = sbase + stage * C::kStageBytes;
+          const uint64_t adesc = smem_desc_sw128(a_addr);
+          const uint64_t bdesc = smem_desc_sw128(a_addr + C::kABytes);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            // advance 16 bf16 (32 bytes) along K inside the swizzled rows
+            umma_bf16(d_tmem, adesc + 2 * k, bdesc + 2 * k, kIdesc, (kb | k) != 0 ? 1u : 0u);
+          }
+          issued_any = true;
+          umma_commit(empty_bar(stage));
+          if (++stage == S) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit(tfull_bar(acc));
+      }
+      if (*abort_flag && issued_any) {
+        // wait for the MMAs in flight before TMEM is released
+        umma_commit(drain_bar);
+        const uint64_t t0 = global_timer_ns();
+        while (!mbar_try_wait(drain_bar, 0) && global_timer_ns() - t0 < 100000000ull) {
+        }
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int q = warp & 3;
+    const int r = q * 32 + lane;
+    int local = 0;
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++local) {
+      const Tile t = decode<MODE>(tile, args, s_off, s_toff);
+      const int acc = local & 1;
+      const uint32_t acc_phase = (local >> 1) & 1;
+      const bool ok = mbar_wait_bounded(tfull_bar(acc), acc_phase, abort_flag);
+      // all lanes agree (and reconverge) before the warp-collective TMEM loads
+      if (!__all_sync(0xffffffffu, ok)) break;
+      tc_fence_after();
+      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN;
+      const bool valid = r < t.rows;
+      const int64_t grow = static_cast<int64_t>(t.row0) + r;
+      if (MODE == kRouter) {
+        float* out = static_cast<float*>(args.out) + grow * args.ldo;
+#pragma unroll
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t v[32];
+          tmem_ld_32x32b_x32(taddr + c, v);
+          tmem_ld_wait();
+          if (valid) {
+            float4* o4 = reinterpret_cast<float4*>(out + c);
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+              o4[u] = make_float4(__uint_as_float(v[4 * u]), __uint_as_float(v[4 * u + 1]),
+                                  __uint_as_float(v[4 * u + 2]), __uint_as_float(v[4 * u + 3]));
+          }
+        }
+      } else if (MODE == kGateUp) {
+        __nv_bfloat16* out = static_cast<__nv_bfloat16*>(args.out) + grow * args.ldo + t.nb * 128;
+#pragma unroll 1
+        for (int c = 0; c < 128; c += 32) {
+          uint32_t gv[32], uv[32];
+          tmem_ld_32x32b_x32(taddr + c, gv);
+          tmem_ld_32x32b_x32(taddr + 128 + c, uv);
+          tmem_ld_wait();
+          if (valid) {
+            uint4* o4 = reinterpret_cast<uint4*>(out + c);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              uint32_t w[4];
+#pragma unroll
+              for (int z = 0; z < 4; ++z) {
+                const int i0 = 8 * u + 2 * z;
+                w[z] = pack_bf16x2(silu(__uint_as_float(gv[i0])) * __uint_as_float(uv[i0]),
+                                   silu(__uint_as_float(gv[i0 + 1])) * __uint_as_float(uv[i0 + 1]));
+              }
+              o4[u] = make_uint4(w[0], w[1], w[2], w[3]);
+            }
+          }
+        }
+      } else {
+        __nv_bfloat16* out = static_cast<__nv_bfloat16*>(args.out) + grow * args.ldo + t.nb * BN;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t v[32];
+          tmem_ld_32x32b_x32(taddr + c, v);
+          tmem_ld_wait();
+          if (valid) {
+            uint4* o4 = reinterpret_cast<uint4*>(out + c);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              uint32_t w[4];
+#pragma unroll
+              for (int z = 0; z < 4; ++z) {
+                const int i0 = 8 * u + 2 * z;
+                w[z] = pack_bf16x2(__uint_as_float(v[i0]), __uint_as_float(v[i0 + 1]));
+              }
+              o4[u] = make_uint4(w[0], w[1], w[2], w[3]);
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty_bar(acc));
+    }
+  }
+
+  __syncthreads();
+  if (threadIdx.x == 0 && *abort_flag && args.err) atomicExch(args.err, kDevErrTimeout);
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc<C::kTmemCols>(tmem_base);
+  }
+}
+
+// ---------------------------------------------------------------- host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 tensor [outer, inner] (row-major), box [box_outer, 64], 128B swizzle.
+static bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
+                     uint32_t box_outer) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int MODE, int BN>
+static cudaError_t launch_mode(const CUtensorMap& a, const CUtensorMap& b, const Args& args,
+                               int grid, cudaStream_t stream) {
+  using C = Cfg<BN>;
+  static int attr_dev = -1;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (attr_dev != dev) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<MODE, BN>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr_dev = dev;
+  }
+  gemm_kernel<MODE, BN><<<grid, kThreads, C::kSmemBytes, stream>>>(a, b, args);
+  return cudaGetLastError();
+}
+
+}  // namespace gemm
+
+// logits[T, N] = x[T, d] W_r[N, d]^T
+cudaError_t launch_router_gemm(const uint16_t* x, const uint16_t* wr, int64_t T, int d, int N,
+                               float* logits, int32_t* err, int num_sms, cudaStream_t stream) {
+  using namespace gemm;
+  if (T == 0) return cudaSuccess;
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, x, d, T, BM) || !make_map(&mb, wr, d, N, N)) return cudaErrorInvalidValue;
+  Args a{};
+  a.groups = 1;
+  a.m_rows = T;
+  a.n_tiles = 1;
+  a.k_blocks = d / BK;
+  a.out = logits;
+  a.ldo = N;
+  a.err = err;
+  const int64_t tiles = (T + BM - 1) / BM;
+  const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
+  if (N == 64) return launch_mode<kRouter, 64>(ma, mb, a, grid, stream);
+  return launch_mode<kRouter, 128>(ma, mb, a, grid, stream);
+}
+
+// h[P, I] = silu(xs W_g^T) * (xs W_u^T) per expert
+cudaError_t launch_gateup_gemm(const uint16_t* xs, const uint16_t* wgu, const int32_t* offsets,
+                               const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* h,
+                               int32_t* err, int num_sms, cudaStream_t stream) {
+  using namespace gemm;
+  if (P == 0) return cudaSuccess;
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, xs, d, P, BM) ||
+      !make_map(&mb, wgu, d, static_cast<uint64_t>(N) * 2 * I, 128))
+    return cudaErrorInvalidValue;
+  Args a{};
+  a.offsets = offsets;
+  a.tile_off = tile_off;
+  a.groups = N;
+  a.n_tiles = I / 128;
+  a.k_blocks = d / BK;
+  a.b_rows = 2 * I;
+  a.b_half = I;
+  a.out = h;
+  a.ldo = I;
+  a.err = err;
+  return launch_mode<kGateUp, 256>(ma, mb, a, num_sms, stream);
+}
+
+// o[P, d] = h W_d[e]^T per expert
+cudaError_t launch_down_gemm(const uint16_t* h, const uint16_t* wd, const int32_t* offsets,
+                             const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* o,
+                             int32_t* err, int num_sms, cudaStream_t stream) {
+  using namespace gemm;
+  if (P == 0) return cudaSuccess;
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, h, I, P, BM) || !make_map(&mb, wd, I, static_cast<uint64_t>(N) * d, 256))
+    return cudaErrorInvalidValue;
+  Args a{};
+  a.offsets = offsets;
+  a.tile_off = tile_off;
+  a.groups = N;
+  a.n_tiles = d / 256;
+  a.k_blocks = I / BK;
+  a.b_rows = d;
+  a.out = o;
+  a.ldo = d;
+  a.err = err;
+  return launch_mode<kDown, 256>(ma, mb, a, num_sms, stream);
+}
+
+}  // namespace moe

@@ -1,0 +1,89 @@
+"""The C-ABI library builds, loads and exports every entry point that
+include/elbow_moe.h declares; host-side argument validation returns the
+documented status codes. No kernel is launched here (no GPU needed)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2608_04401_gb300 as moe
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "elbow_moe.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    moe.build()
+    return moe.library()
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    names = re.findall(r"^\s*(?:const\s+)?[A-Za-z_][A-Za-z0-9_]*\s*\*?\s+\*?([a-z_][a-z0-9_]*)\s*\(",
+                       src, flags=re.M)
+    return sorted(set(names))
+
+
+def test_header_declares_the_boundary():
+    names = _declared()
+    for n in ("elbow_route", "moe_dispatch", "moe_layer_forward", "moe_layer_workspace_size",
+              "moe_status_string", "moe_read_device_error"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for n in _declared():
+        assert hasattr(lib, n), n
+
+
+def test_status_strings(lib):
+    for s in range(6):
+        assert lib.moe_status_string(s).startswith(b"MOE_")
+
+
+def _rp(K=8, eps=1e-8, mode=0, renorm=0):
+    return ctypes.byref(moe.RouteParams(K, eps, mode, renorm))
+
+
+def test_route_validation(lib):
+    fake = ctypes.c_void_p(256)
+    # unsupported N, K
+    assert lib.elbow_route(fake, 10, 65, _rp(), fake, fake, fake, None) == 2
+    assert lib.elbow_route(fake, 10, 64, _rp(K=9), fake, fake, fake, None) == 2
+    assert lib.elbow_route(fake, 10, 64, _rp(K=0), fake, fake, fake, None) == 2
+    # bad params / pointers
+    assert lib.elbow_route(fake, 10, 64, _rp(mode=3), fake, fake, fake, None) == 1
+    assert lib.elbow_route(fake, 10, 64, _rp(eps=-1.0), fake, fake, fake, None) == 1
+    assert lib.elbow_route(None, 10, 64, _rp(), fake, fake, fake, None) == 1
+    assert lib.elbow_route(ctypes.c_void_p(258), 10, 64, _rp(), fake, fake, fake, None) == 1
+    assert lib.elbow_route(fake, -1, 64, _rp(), fake, fake, fake, None) == 1
+    assert lib.elbow_route(fake, 10, 64, None, fake, fake, fake, None) == 1
+    # T = 0 is a no-op that launches nothing
+    assert lib.elbow_route(None, 0, 64, _rp(), None, None, None, None) == 0
+
+
+def test_dispatch_validation(lib):
+    fake = ctypes.c_void_p(256)
+    need = lib.moe_dispatch_workspace_size(1000, 64, 8)
+    assert need > 0
+    assert lib.moe_dispatch(fake, fake, 1000, 64, 8, fake, fake, fake, fake, need - 1, None) == 3
+    assert lib.moe_dispatch(fake, fake, 1000, 96, 8, fake, fake, fake, fake, need, None) == 2
+    assert lib.moe_dispatch(fake, fake, 1000, 64, 8, None, fake, fake, fake, need, None) == 1
+
+
+def test_layer_validation(lib):
+    fake = ctypes.c_void_p(256)
+    ws = lib.moe_layer_workspace_size(64, 2048, 64, 1024, 8)
+    assert ws > 64 * 8 * (2048 * 2 * 2 + 1024 * 2)
+    args = lambda T=64, d=2048, N=64, I=1024, rp=None, wsb=ws: (
+        fake, fake, fake, fake, T, d, N, I, rp or _rp(), None, fake, None, None, None, None, None,
+        fake, wsb, None)
+    assert lib.moe_layer_forward(*args(d=2000)) == 2
+    assert lib.moe_layer_forward(*args(I=1000)) == 2
+    assert lib.moe_layer_forward(*args(N=32)) == 2
+    assert lib.moe_layer_forward(*args(wsb=ws - 1)) == 3
+    assert lib.moe_layer_forward(*args(rp=_rp(renorm=2))) == 1
+    assert lib.moe_layer_workspace_size(64, 2048, 63, 1024, 8) == 0

@@ -1,0 +1,139 @@
+"""GPU parity of routing (elbow_route) and dispatch (moe_dispatch) against the
+CPU oracle: bit-exact k, ids, gates, offsets, perm and pair_pos on the same
+seeded fp32 logits, including the full 1,048,576-token routing stress."""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_04401_gb300 import synth
+
+from gpu_util import to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def moe():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2608_04401_gb300 as m
+    m.build()
+    m.library()
+    return m
+
+
+def _route_both(moe, lg, K=8, mode=0, renorm=0, eps=1e-8):
+    k, ids, gates = moe.elbow_route(to_dev(lg), K=K, eps=eps, mode=mode, renorm=renorm)
+    ref = oracle.route(lg, K=K, eps=eps, mode=mode, renorm=renorm)
+    return (k.cpu().numpy(), ids.cpu().numpy(), gates.cpu().numpy()), ref
+
+
+def _assert_route_equal(got, ref):
+    k, ids, gates = got
+    bad = np.nonzero(k != ref["k"])[0]
+    assert bad.size == 0, f"k differs at {bad[:10]} (of {bad.size})"
+    assert np.array_equal(ids, ref["ids"])
+    assert np.array_equal(gates.view(np.uint32), ref["gates"].view(np.uint32))
+
+
+@pytest.mark.parametrize("N", [64, 128])
+@pytest.mark.parametrize("T", [1, 127, 129, 5000])
+def test_route_bitexact_sizes(moe, N, T):
+    rng = np.random.default_rng(T * 7 + N)
+    lg = synth.boosted_logits(rng, T, N)
+    _assert_route_equal(*_route_both(moe, lg))
+
+
+@pytest.mark.parametrize("K,mode,renorm", [(8, 1, 0), (8, 0, 1), (1, 0, 0), (3, 0, 0), (5, 1, 1)])
+def test_route_bitexact_params(moe, K, mode, renorm):
+    rng = np.random.default_rng(K * 10 + mode + 3 * renorm)
+    for N in (64, 128):
+        lg = synth.boosted_logits(rng, 3001, N)
+        _assert_route_equal(*_route_both(moe, lg, K=K, mode=mode, renorm=renorm))
+
+
+def test_route_edge_cases(moe):
+    N = 64
+    rows = []
+    rows.append(np.zeros(N))                      # uniform: k = 1
+    rows.append(np.full(N, 3.25))                 # uniform, nonzero
+    for m in (1, 2, 5, 7, 8, 20, 62, 63):          # step curves
+        r = np.zeros(N); r[:m] = 6.0; rows.append(r)
+    r = np.zeros(N); r[[3, 9, 40]] = 4.0; rows.append(r)   # ties among the head
+    r = np.full(N, -500.0); r[11] = 0.0; rows.append(r)    # tail underflows to 0
+    r = np.arange(N, dtype=np.float64) * 0.01; rows.append(r)  # nearly linear curve
+    r = np.zeros(N); r[::2] = 1e-7; rows.append(r)   # distinct logits, equal probabilities
+    r = np.linspace(-60, 30, N); rows.append(r)      # wide range
+    rng = np.random.default_rng(0)
+    q = np.round(rng.standard_normal((200, N)) * 2) / 2   # many exact ties
+    lg = np.concatenate([np.array(rows), q]).astype(np.float32)
+    for K in (8, 2):
+        for mode in (0, 1):
+            _assert_route_equal(*_route_both(moe, lg, K=K, mode=mode))
+    lg128 = np.concatenate([lg, lg], axis=1)
+    _assert_route_equal(*_route_both(moe, lg128))
+    # eps = 0 on a non-degenerate batch
+    _assert_route_equal(*_route_both(moe, q.astype(np.float32), eps=0.0))
+
+
+def test_route_full_stress(moe):
+    """The 1,048,576 x 64 routing stress, compared token by token."""
+    w = synth.WORKLOADS["route_t1m"]
+    rng = np.random.Generator(np.random.PCG64(w["seed"]))
+    lg = synth.boosted_logits(rng, w["T"], w["N"])
+    got, ref = _route_both(moe, lg, K=w["K"])
+    _assert_route_equal(got, ref)
+    assert 1.0 < ref["k"].mean() < 8.0
+
+
+def _dispatch_both(moe, k, ids, N):
+    import torch
+    off, perm, pp, ws = moe.moe_dispatch(to_dev(k), to_dev(ids), N)
+    torch.cuda.synchronize()
+    ref = oracle.dispatch(k, ids, N)
+    off = off.cpu().numpy()
+    assert np.array_equal(off, ref["offsets"])
+    P = int(off[-1])
+    assert np.array_equal(perm.cpu().numpy()[:P], ref["perm"])
+    assert np.array_equal(pp.cpu().numpy(), ref["pair_pos"])
+    # m-tile prefix sums left in the workspace
+    T, K = ids.shape
+    toff = moe.dispatch_tile_offsets(ws, T, N, K).cpu().numpy()
+    cnt = np.diff(ref["offsets"])
+    assert np.array_equal(toff, np.concatenate([[0], np.cumsum((cnt + 127) // 128)]))
+    return ref
+
+
+@pytest.mark.parametrize("N", [64, 128])
+@pytest.mark.parametrize("T", [1, 33, 2047, 2048, 2049, 20000])
+def test_dispatch_bitexact(moe, N, T):
+    rng = np.random.default_rng(T + N)
+    r = oracle.route(synth.boosted_logits(rng, T, N), K=8)
+    _dispatch_both(moe, r["k"], r["ids"], N)
+
+
+def test_dispatch_edges(moe):
+    N, K = 64, 8
+    T = 5000
+    ids = np.tile(np.arange(K, dtype=np.int32), (T, 1))
+    _dispatch_both(moe, np.ones(T, np.int32), ids, N)             # all on expert 0
+    _dispatch_both(moe, np.full(T, K, np.int32), ids, N)           # fixed top-8
+    _dispatch_both(moe, np.zeros(T, np.int32), ids, N)             # no pairs
+    ids2 = ids.copy(); ids2[:, 0] = 63; ids2[:, 7] = 0
+    _dispatch_both(moe, np.full(T, 3, np.int32), ids2, N)          # last expert
+    ids3 = np.tile(np.arange(120, 128, dtype=np.int32), (T, 1))
+    _dispatch_both(moe, np.full(T, K, np.int32), ids3, 128)
+    # T = 0
+    import torch
+    off, perm, pp, ws = moe.moe_dispatch(torch.zeros(0, dtype=torch.int32, device="cuda"),
+                                         torch.zeros(0, K, dtype=torch.int32, device="cuda"), N)
+    assert np.all(off.cpu().numpy() == 0)
+
+
+def test_dispatch_full_stress(moe):
+    w = synth.WORKLOADS["route_t1m"]
+    rng = np.random.Generator(np.random.PCG64(w["seed"] + 1))
+    lg = synth.boosted_logits(rng, w["T"], w["N"])
+    r = oracle.route(lg, K=8)
+    _dispatch_both(moe, r["k"], r["ids"], w["N"])
