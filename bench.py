@@ -1,0 +1,458 @@
+"""Benchmark of the elbow-routed MoE layer on GB300.
+
+One step = one MoE layer forward (router GEMM, elbow routing, dispatch,
+gather, grouped SwiGLU gate/up GEMM, grouped down GEMM, combine) over the
+16,384-token OLMoE-shaped prefill batch (d = 2048, 64 experts, I = 1024,
+K = 8), inputs resident in HBM. `value` = tokens/s in elbow mode; the same
+kernels in fixed top-8 mode are reported beside it. Per-kernel CUDA-event
+times give the roofline of the dominant kernel (the gate/up GEMM, against the
+measured dense bf16 peak) and of the routing/dispatch kernels on the
+1,048,576-token routing stress (against the measured HBM copy bandwidth).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Multi-GPU (torchrun): every rank runs its own batch (weak scaling, no
+data-path collective); timing is max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "MoE-layer tokens/s elbow vs fixed top-8; route GB/s & GEMM tensor-pipe % of peak"
+WORKLOAD = "layer_t16k"
+ROUTE_WORKLOAD = "route_t1m"
+# steps per launch sequence of moe_layer_forward (router GEMM, route, dispatch
+# count/scan/scatter, gather, gate/up GEMM, down GEMM, combine)
+KERNELS_PER_STEP = 9
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--tokens", type=int, default=0,
+                    help="override the batch size T of the layer workload (profiling runs)")
+    ap.add_argument("--quick", action="store_true",
+                    help="time only the layer forward (no breakdown, stress, e2e, CPU baseline)")
+    ap.add_argument("--route-only", action="store_true",
+                    help="time only routing and dispatch on the 1,048,576-token stress")
+    return ap.parse_args()
+
+
+def dist_setup(n):
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if os.environ.get("BENCH_BACKEND", "nccl") == "nccl" else "gloo"
+        dist.init_process_group(backend)
+        pg = dist
+    return rank, world, local, pg
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return dict(hbm=float(j["hbm_gbs"]), bf16=float(j["bf16_tflops"]),
+                    bf16_sus=float(j.get("bf16_tflops_sustained", j["bf16_tflops"])),
+                    source="measured")
+    return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, source="fallback")
+
+
+def ncu_traffic(key):
+    """DRAM bytes per launch from the committed ncu capture, or None when the
+    kernel's sources changed since the counters were taken."""
+    import hashlib
+    p = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        j = json.load(f).get(key)
+    if not j:
+        return None
+    h = hashlib.sha256()
+    for src in j["sources"]:
+        with open(os.path.join(ROOT, src), "rb") as f:
+            h.update(f.read())
+    if h.hexdigest() != j["source_sha256"]:
+        return None
+    return int(j["dram_read_bytes"]) + int(j["dram_write_bytes"])
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        self.out = ""
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out = ""
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in (self.out or "").splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def bf16_dev(bits, dev):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
+
+
+def time_steps(fn, steps, stream, pg):
+    """Barrier + sync on both sides; CUDA events on the launching stream."""
+    import torch
+    if pg is not None:
+        pg.barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        fn()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    if pg is not None:
+        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        ms = float(t.item())
+    return ms / steps
+
+
+def run_ours(args, rank, world, local, pg):
+    import torch
+
+    import paper_2608_04401_gb300 as moe
+    from paper_2608_04401_gb300 import synth
+
+    moe.build()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream()
+    pk = peaks()
+    if args.route_only:
+        return {"metric": METRIC, "route_stress": route_stress(moe, args, stream, dev, pk),
+                "quick": True}
+    w = synth.WORKLOADS[WORKLOAD]
+    T, d, N, I, K = w["T"], w["d"], w["N"], w["I"], w["K"]
+    if args.tokens > 0:
+        T = args.tokens
+    inp = synth.layer_inputs(T=T, d=d, N=N, I=I, seed=w["seed"] + 7919 * rank)
+    x = bf16_dev(inp["x"], dev)
+    wr = bf16_dev(inp["w_router"], dev)
+    wgu = bf16_dev(inp["w_gate_up"], dev)
+    wd = bf16_dev(inp["w_down"], dev)
+    ws = torch.empty(moe.layer_workspace_size(T, d, N, I, K), dtype=torch.uint8, device=dev)
+    y = torch.empty(T, d, dtype=torch.bfloat16, device=dev)
+
+    def step(mode):
+        return lambda: moe.moe_layer_forward(x, wr, wgu, wd, K=K, mode=mode, y=y, ws=ws)
+
+    for mode in (moe.MODE_ELBOW, moe.MODE_TOPK):
+        for _ in range(max(3, args.warmup)):
+            step(mode)()
+    moe.read_device_error(ws)
+
+    with ClockSampler(local) as clk:
+        ms_elbow = time_steps(step(moe.MODE_ELBOW), args.steps, stream, pg)
+        ms_topk = time_steps(step(moe.MODE_TOPK), args.steps, stream, pg)
+    moe.read_device_error(ws)
+    clocks = clk.summary()
+    if args.quick:
+        return {"metric": METRIC, "value": world * T / (ms_elbow * 1e-3), "unit": "tokens/s",
+                "n_gpus": world, "steps": args.steps, "ms_per_step": ms_elbow,
+                "topk_ms_per_step": ms_topk, "config": {"workload": f"{WORKLOAD} T={T}"},
+                "quick": True, "clocks": clocks}
+
+    # routing statistics of this batch
+    _, it = moe.moe_layer_forward(x, wr, wgu, wd, K=K, y=y, ws=ws, return_intermediates=True)
+    kk = it["k"].cpu().numpy()
+    sum_k = int(kk.sum())
+    load = np.diff(it["offsets"].cpu().numpy())
+
+    # per-kernel breakdown (same kernels through the step-level entry points)
+    kern = kernel_breakdown(moe, x, wr, wgu, wd, T, d, N, I, K, args, stream, dev)
+    flops_gu = 4.0 * d * I * sum_k
+    flops_dn = 2.0 * d * I * sum_k
+    gu_ms = kern["gate_up"]["ms"]
+    dn_ms = kern["down"]["ms"]
+    gu_tf = flops_gu / (gu_ms * 1e-3) / 1e12
+    dn_tf = flops_dn / (dn_ms * 1e-3) / 1e12
+    kern["gate_up"].update(tflops=gu_tf, frac=gu_tf / pk["bf16_sus"])
+    kern["down"].update(tflops=dn_tf, frac=dn_tf / pk["bf16_sus"])
+
+    route = route_stress(moe, args, stream, dev, pk)
+
+    # end to end through the public API with host buffers
+    xh = torch.empty(T, d, dtype=torch.bfloat16, pin_memory=True)
+    xh.copy_(x.cpu())
+    yh = torch.empty(T, d, dtype=torch.bfloat16, pin_memory=True)
+    xd = torch.empty_like(x)
+
+    def e2e_step():
+        xd.copy_(xh, non_blocking=True)
+        moe.moe_layer_forward(xd, wr, wgu, wd, K=K, y=y, ws=ws)
+        yh.copy_(y, non_blocking=True)
+
+    for _ in range(3):
+        e2e_step()
+    ms_e2e = time_steps(e2e_step, max(20, args.steps // 4), stream, pg)
+
+    tok_s = world * T / (ms_elbow * 1e-3)
+    out = {
+        "metric": METRIC,
+        "value": tok_s,
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": max(3, args.warmup),
+        "ms_per_step": ms_elbow,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded signal-noise tokens and N(0,0.02) experts; OLMoE shapes)",
+        "config": {
+            "workload": f"{WORKLOAD}: one MoE layer, T={T} tokens, d_model={d}, N={N} experts, "
+                        f"SwiGLU I={I}, K={K}, elbow routing",
+            "tokens_per_gpu": T,
+            "l2": "inputs larger than L2: 805 MB of expert weights and 64 MB of tokens per step",
+            "parallelism": f"replicas x{world} (independent batches, no collective)",
+        },
+        "topk": {"value": world * T / (ms_topk * 1e-3), "unit": "tokens/s", "ms_per_step": ms_topk,
+                 "elbow_speedup": ms_topk / ms_elbow},
+        "routing": {"mean_k": sum_k / T, "k_hist": np.bincount(kk, minlength=K + 1)[1:].tolist(),
+                    "expert_load_min": int(load.min()), "expert_load_max": int(load.max())},
+        "roofline": {"kernel": "grouped gate/up GEMM + SwiGLU (tcgen05)", "bound": "tensor",
+                     "achieved": gu_tf, "peak": pk["bf16_sus"], "unit": "TFLOP/s",
+                     "frac": gu_tf / pk["bf16_sus"], "traffic": ncu_traffic("gemm_gate_up_layer_t16k"),
+                     "traffic_unit": "bytes per launch (ncu dram read + write)",
+                     "algorithmic_bytes": 2 * sum_k * d + 2 * N * 2 * I * d + 2 * sum_k * I,
+                     "peak_source": f"{pk['source']} bf16 dense, sustained",
+                     "frac_of_burst": gu_tf / pk["bf16"]},
+        "kernels": kern,
+        "route_stress": route,
+        "e2e": {"value": world * T / (ms_e2e * 1e-3), "unit": "tokens/s", "ms_per_step": ms_e2e,
+                "h2d_bytes_per_step": T * d * 2, "d2h_bytes_per_step": T * d * 2},
+        "gpu_launches": KERNELS_PER_STEP * args.steps * 2,
+        "clocks": clocks,
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(inp, K)
+    return out
+
+
+def kernel_breakdown(moe, x, wr, wgu, wd, T, d, N, I, K, args, stream, dev):
+    """Average duration of each kernel of the layer, CUDA events between the
+    step-level calls on one stream, over `steps` back-to-back steps."""
+    import torch
+    names = ["router_gemm", "route", "dispatch", "gather", "gate_up", "down", "combine"]
+    acc = {n: 0.0 for n in names}
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    P = T * K
+    steps = max(10, args.steps // 4)
+    dws = torch.empty(moe.dispatch_workspace_size(T, N, K), dtype=torch.uint8, device=dev)
+    for it in range(steps + 3):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)]
+        ev[0].record(stream)
+        lg = moe.router_logits(x, wr, err=err)
+        ev[1].record(stream)
+        k, ids, gates = moe.elbow_route(lg, K=K)
+        ev[2].record(stream)
+        off, perm, pp, _ = moe.moe_dispatch(k, ids, N, ws=dws)
+        ev[3].record(stream)
+        xs = moe.gather_rows(x, perm, off, P)
+        ev[4].record(stream)
+        toff = moe.dispatch_tile_offsets(dws, T, N, K)
+        h = moe.expert_gate_up(xs, wgu, off, toff, err=err)
+        ev[5].record(stream)
+        o = moe.expert_down(h, wd, off, toff, err=err)
+        ev[6].record(stream)
+        moe.combine(o, k, pp, gates)
+        ev[7].record(stream)
+        torch.cuda.synchronize()
+        if it >= 3:
+            for i, n in enumerate(names):
+                acc[n] += ev[i].elapsed_time(ev[i + 1])
+    assert int(err.item()) == 0, "device timeout in a GEMM"
+    tot = sum(acc.values())
+    return {n: {"ms": acc[n] / steps, "share": acc[n] / tot} for n in names}
+
+
+def route_stress(moe, args, stream, dev, pk):
+    """elbow_route and moe_dispatch on the 1,048,576 x 64 fp32-logit stress."""
+    import torch
+    from paper_2608_04401_gb300 import synth
+    w = synth.WORKLOADS[ROUTE_WORKLOAD]
+    T, N, K = w["T"], w["N"], w["K"]
+    rng = np.random.Generator(np.random.PCG64(w["seed"]))
+    lg = torch.from_numpy(synth.boosted_logits(rng, T, N)).to(dev)
+    k = torch.empty(T, dtype=torch.int32, device=dev)
+    ids = torch.empty(T, K, dtype=torch.int32, device=dev)
+    gates = torch.empty(T, K, dtype=torch.float32, device=dev)
+    lib = moe.library()
+    rp = moe._params(K, 1e-8, 0, 0)
+    s = moe._stream()
+    P = moe._p
+
+    def route():
+        lib.elbow_route(P(lg), T, N, rp, P(k), P(ids), P(gates), s)
+
+    dws = torch.empty(moe.dispatch_workspace_size(T, N, K), dtype=torch.uint8, device=dev)
+    off = torch.empty(N + 1, dtype=torch.int32, device=dev)
+    perm = torch.empty(T * K, dtype=torch.int32, device=dev)
+    pp = torch.empty(T, K, dtype=torch.int32, device=dev)
+
+    def disp():
+        lib.moe_dispatch(P(k), P(ids), T, N, K, P(off), P(perm), P(pp), P(dws), dws.numel(), s)
+
+    for _ in range(3):
+        route()
+        disp()
+    n = max(20, args.steps // 4)
+    ms_r = time_steps(route, n, stream, None)
+    ms_d = time_steps(disp, n, stream, None)
+    sum_k = int(k.sum().item())
+    # algorithmic bytes: route reads N fp32 logits, writes k + K ids + K gates
+    br = T * (4 * N + 4 + 8 * K)
+    # dispatch reads k and the K ids, writes one perm entry per pair and K pair positions
+    bd = T * (4 + 4 * K) + 4 * sum_k + 4 * T * K
+    gr = br / (ms_r * 1e-3) / 1e9
+    gd = bd / (ms_d * 1e-3) / 1e9
+    return {"workload": f"{ROUTE_WORKLOAD}: T={T} x N={N} fp32 logits, K={K}",
+            "route": {"ms": ms_r, "GBps": gr, "frac": gr / pk["hbm"], "bytes": br,
+                      "tokens_per_s": T / (ms_r * 1e-3)},
+            "dispatch": {"ms": ms_d, "GBps": gd, "frac": gd / pk["hbm"], "bytes": bd},
+            "peak_GBps": pk["hbm"], "peak_source": pk["source"] + " HBM copy",
+            "mean_k": sum_k / T}
+
+
+def cpu_baseline(inp, K, budget_s=12.0):
+    """The CPU oracle, as it stands, on a bounded sample of the same workload."""
+    import oracle
+    T = inp["x"].shape[0]
+    rows = np.arange(8, dtype=np.int64)
+    t0 = time.perf_counter()
+    oracle.layer_rows(inp["x"], inp["w_router"], inp["w_gate_up"], inp["w_down"], rows=rows, K=K)
+    dt = time.perf_counter() - t0
+    n = int(min(T, max(8, 8 * budget_s / max(dt, 1e-3))))
+    rows = np.linspace(0, T - 1, n).astype(np.int64)
+    t0 = time.perf_counter()
+    oracle.layer_rows(inp["x"], inp["w_router"], inp["w_gate_up"], inp["w_down"], rows=rows, K=K)
+    dt = time.perf_counter() - t0
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    return {"value": n / dt, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"{n} of the {T} tokens of the same layer (fp64 C oracle, OpenMP), {dt:.1f} s"}
+
+
+def run_reference(args, rank, world):
+    """The oracle, as it stands, timed on the host cores (rank 0 only)."""
+    if rank != 0:
+        return None
+    import oracle
+    from paper_2608_04401_gb300 import synth
+    oracle.build()
+    w = synth.WORKLOADS[WORKLOAD]
+    T, K = w["T"], w["K"]
+    inp = synth.layer_inputs(T=T, d=w["d"], N=w["N"], I=w["I"], seed=w["seed"])
+    sample = 16
+    rng = np.random.default_rng(0)
+
+    def step():
+        rows = np.sort(rng.choice(T, sample, replace=False)).astype(np.int64)
+        oracle.layer_rows(inp["x"], inp["w_router"], inp["w_gate_up"], inp["w_down"], rows=rows,
+                          K=K)
+
+    for _ in range(max(1, min(args.warmup, 3))):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps if args.steps <= 50 else 50):
+        step()
+    n = args.steps if args.steps <= 50 else 50
+    dt = (time.perf_counter() - t0) / n
+    val = sample / dt
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    return {
+        "impl": "reference", "metric": METRIC, "value": val, "unit": "tokens/s", "n_gpus": world,
+        "steps": n, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": f"{WORKLOAD}: one MoE layer, T={T}, d_model={w['d']}, "
+                               f"N={w['N']}, I={w['I']}, K={K}, elbow routing; each step routes "
+                               f"and computes a {sample}-token sample"},
+        "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": f"{sample} random tokens of the {T}-token layer per step"},
+        "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    args = parse()
+    rank, world, local, pg = dist_setup(args.gpus)
+    if args.impl == "reference":
+        out = run_reference(args, rank, world)
+    else:
+        out = run_ours(args, rank, world, local, pg)
+    if rank == 0 and out is not None:
+        print(json.dumps(out))
+    if pg is not None:
+        pg.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
