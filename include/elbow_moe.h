@@ -107,6 +107,29 @@ moe_status moe_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, 
                         size_t ws_bytes, void* stream);
 
 /*
+ * moe_dispatch_noalloc - moe_dispatch for callers that cannot allocate device
+ * memory when they dispatch: for example a serving runtime that sizes all of
+ * its device memory up front and allows no allocation on the request path
+ * (an allocation can stall on the device or fragment its pool), or a plug-in
+ * whose host framework passes it only input and output buffers. The paper has
+ * no counterpart; this is a packaging variant of the same dispatch kernels.
+ *
+ * Arguments and results are those of moe_dispatch, without the workspace. The
+ * scratch (per-chunk counts and bases, 2 * 512 * 128 int32 plus the tile
+ * offsets, about 513 KB) is a fixed array inside the library, which every GPU
+ * that loads the library keeps until the process exits. Limits: T <= 1,048,576
+ * tokens (larger T returns MOE_ERR_UNSUPPORTED), N in {64, 128}, K <= 8.
+ * No cudaMalloc, cudaFree or other allocating call is made.
+ * The first call on each device looks up the array's device address (with
+ * that device current) and caches it; make that first call before any stream
+ * capture. All calls share the one array and each call rewrites every part of
+ * it that it reads, so no clearing is needed; calls whose kernels overlap on
+ * the GPU (different streams, or different host threads) race on the array.
+ */
+moe_status moe_dispatch_noalloc(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
+                                int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* stream);
+
+/*
  * moe_layer_forward - one MoE layer forward under elbow routing (Sec. 2,
  * App. A.4): router logits l = W_r x (bf16 x bf16, fp32 accumulate), routing
  * as elbow_route, dispatch as moe_dispatch, per-expert SwiGLU

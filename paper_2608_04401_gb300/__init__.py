@@ -17,7 +17,7 @@ import threading
 
 __all__ = [
     "MODE_ELBOW", "MODE_TOPK", "MoeError", "library", "build",
-    "elbow_route", "moe_dispatch", "dispatch_workspace_size", "layer_workspace_size",
+    "elbow_route", "moe_dispatch", "moe_dispatch_noalloc", "dispatch_workspace_size", "layer_workspace_size",
     "moe_layer_forward", "read_device_error", "router_logits", "gather_rows",
     "expert_gate_up", "expert_down", "combine",
 ]
@@ -67,6 +67,7 @@ def library():
             "moe_dispatch_workspace_size": ([i64, i32, i32], sz),
             "moe_dispatch": ([P, P, i64, i32, i32, P, P, P, P, sz, P], i32),
             "moe_dispatch_tile_offsets": ([P, i64, i32, i32], P),
+            "moe_dispatch_noalloc": ([P, P, i64, i32, i32, P, P, P, P], i32),
             "moe_layer_workspace_size": ([i64, i32, i32, i32, i32], sz),
             "moe_layer_forward": ([P, P, P, P, i64, i32, i32, i32, RP, P, P, P, P, P, P, P, P, sz, P],
                                   i32),
@@ -157,6 +158,26 @@ def moe_dispatch(k, ids, N: int, ws=None, stream=None):
     _check(lib.moe_dispatch(_p(k), _p(ids), T, N, K, _p(offsets), _p(perm), _p(pair_pos), _p(ws),
                             ws.numel(), _stream(stream)), "moe_dispatch")
     return offsets, perm, pair_pos, ws
+
+
+def moe_dispatch_noalloc(k, ids, N: int, offsets=None, perm=None, pair_pos=None, stream=None):
+    """moe_dispatch without a workspace (the library's fixed scratch array is used).
+    Output buffers may be passed in; returns (offsets, perm, pair_pos)."""
+    torch = _torch()
+    lib = library()
+    _cuda(k, torch.int32, "k")
+    _cuda(ids, torch.int32, "ids")
+    T, K = ids.shape
+    dev = ids.device
+    if offsets is None:
+        offsets = torch.empty(N + 1, dtype=torch.int32, device=dev)
+    if perm is None:
+        perm = torch.empty(max(1, T * K), dtype=torch.int32, device=dev)
+    if pair_pos is None:
+        pair_pos = torch.empty(T, K, dtype=torch.int32, device=dev)
+    _check(lib.moe_dispatch_noalloc(_p(k), _p(ids), T, N, K, _p(offsets), _p(perm), _p(pair_pos),
+                                    _stream(stream)), "moe_dispatch_noalloc")
+    return offsets, perm, pair_pos
 
 
 def dispatch_tile_offsets(ws, T: int, N: int, K: int):

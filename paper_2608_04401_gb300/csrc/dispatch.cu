@@ -9,6 +9,8 @@
 //   scatter : each chunk walks its tokens in order, 32 per warp; a pair's
 //             position = chunk base + earlier warps of this round (ballots in
 //             smem) + earlier lanes of this warp (popc of the ballot).
+#include <mutex>
+
 #include "common.cuh"
 
 namespace moe {
@@ -276,3 +278,81 @@ cudaError_t launch_combine(const uint16_t* o, const int32_t* k, const int32_t* p
 }
 
 }  // namespace moe
+
+// ---------------------------------------------------------------------------
+// Dispatch without a caller-provided workspace.
+//
+// Some callers cannot allocate device memory at the point where they dispatch:
+// a serving runtime that plans every byte of device memory up front and forbids
+// allocation on its request path (an allocation can block on the device or
+// fragment a pre-sized pool), or a plug-in whose host framework hands it only
+// the input and output buffers. For them the dispatch's scratch (per-chunk
+// expert counts and bases, and the m-tile offsets) lives in one file-scope
+// device array of fixed size instead of a workspace. Every GPU that loads this
+// library holds the array until the process exits.
+namespace moe {
+namespace disp {
+constexpr int64_t kNoAllocMaxTokens = int64_t(1) << 20;  // 1,048,576 tokens
+constexpr int kNoAllocMaxExperts = 128;
+constexpr int64_t kNoAllocChunks = (kNoAllocMaxTokens + kChunk - 1) / kChunk;
+constexpr int64_t kNoAllocInts = 2 * kNoAllocChunks * kNoAllocMaxExperts + 256;  // ~513 KB
+}  // namespace disp
+}  // namespace moe
+
+static __device__ __align__(256) int32_t g_noalloc_dispatch_scratch[moe::disp::kNoAllocInts];
+
+namespace {
+constexpr int kNoAllocMaxDevices = 64;
+std::mutex g_noalloc_mu;
+int32_t* g_noalloc_ptr[kNoAllocMaxDevices] = {};
+
+// Device address of the scratch array on the current device. The host-side
+// symbol is only a stand-in, so the address is looked up once per device (with
+// that device current) and cached.
+cudaError_t noalloc_scratch(int32_t** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kNoAllocMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_dispatch_scratch);
+    if (e != cudaSuccess) return e;
+    g_noalloc_ptr[dev] = static_cast<int32_t*>(p);
+  }
+  *out = g_noalloc_ptr[dev];
+  return cudaSuccess;
+}
+}  // namespace
+
+extern "C" moe_status moe_dispatch_noalloc(const int32_t* k, const int32_t* ids, int64_t T, int N,
+                                           int K, int32_t* offsets, int32_t* perm,
+                                           int32_t* pair_pos, void* stream) {
+  using namespace moe::disp;
+  if (T < 0) return MOE_ERR_INVALID_ARG;
+  if (T > kNoAllocMaxTokens) return MOE_ERR_UNSUPPORTED;
+  if ((N != 64 && N != 128) || K < 1 || K > 8 || K > N) return MOE_ERR_UNSUPPORTED;
+  if (!offsets) return MOE_ERR_INVALID_ARG;
+  if (T > 0 && (!k || !ids || !perm || !pair_pos)) return MOE_ERR_INVALID_ARG;
+  int32_t* scratch = nullptr;
+  if (noalloc_scratch(&scratch) != cudaSuccess) return MOE_ERR_CUDA;
+  // Layout: per-chunk counts [chunks][N] | per-chunk bases [chunks][N] | tile offsets
+  // [N+1]. The counts and bases of every chunk in use and all N+1 tile offsets are
+  // rewritten by each call, so nothing has to be cleared first.
+  int32_t* blk_cnt = scratch;
+  int32_t* blk_base = scratch + kNoAllocChunks * kNoAllocMaxExperts;
+  int32_t* tile_off = scratch + 2 * kNoAllocChunks * kNoAllocMaxExperts;
+  const int nblk = static_cast<int>((T + kChunk - 1) / kChunk);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (N == 64) {
+    if (nblk > 0) count_kernel<64><<<nblk, kThreads, 0, s>>>(k, ids, T, K, blk_cnt);
+    scan_kernel<64><<<1, 1024, 0, s>>>(blk_cnt, nblk, blk_base, offsets, tile_off, nullptr);
+    if (nblk > 0) scatter_kernel<64><<<nblk, kThreads, 0, s>>>(k, ids, T, K, blk_base, perm, pair_pos);
+  } else {
+    if (nblk > 0) count_kernel<128><<<nblk, kThreads, 0, s>>>(k, ids, T, K, blk_cnt);
+    scan_kernel<128><<<1, 1024, 0, s>>>(blk_cnt, nblk, blk_base, offsets, tile_off, nullptr);
+    if (nblk > 0) scatter_kernel<128><<<nblk, kThreads, 0, s>>>(k, ids, T, K, blk_base, perm, pair_pos);
+  }
+  return cudaGetLastError() == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
+}
