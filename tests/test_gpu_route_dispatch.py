@@ -77,6 +77,34 @@ def test_route_edge_cases(moe):
     _assert_route_equal(*_route_both(moe, q.astype(np.float32), eps=0.0))
 
 
+@pytest.mark.parametrize("N", [64, 128])
+def test_route_near_ties_and_flat_curves(moe, N):
+    """Curves that defeat shortcuts: values a few ulps apart in the top ranks,
+    exact ties around rank 31, flat and linear curves, wide heads of 24-40
+    boosted experts, and tails that underflow."""
+    rng = np.random.default_rng(N + 99)
+    T = 4096
+    lg = rng.standard_normal((T, N)).astype(np.float32)
+    # 1) near ties: a base value plus perturbations of a few ulps
+    lg[0:512] = (2.0 + rng.integers(-3, 4, (512, N)) * np.float32(2.0 ** -22)).astype(np.float32)
+    # 2) exact ties everywhere in the top 40 ranks
+    lg[512:1024] = np.round(rng.uniform(-1, 1, (512, N)) * 4) / 4
+    # 3) flat / linear curves, permuted
+    for t in range(1024, 1536):
+        lg[t] = rng.permutation(np.linspace(0, rng.uniform(0.1, 4.0), N))
+    # 4) wide heads
+    for t in range(1536, 2048):
+        hsz = rng.integers(24, 41)
+        lg[t] = rng.standard_normal(N) * 0.3
+        lg[t, rng.choice(N, hsz, replace=False)] += rng.uniform(0.5, 1.0, hsz)
+    # 5) spikes over a -60..-200 tail (partial underflow of the exponent)
+    lg[2048:2560] = rng.uniform(-200, -60, (512, N))
+    lg[2048:2560, 0] = 0.0
+    lg = lg.astype(np.float32)
+    for K, mode in ((8, 0), (8, 1), (4, 0), (1, 0)):
+        _assert_route_equal(*_route_both(moe, lg, K=K, mode=mode))
+
+
 def test_route_full_stress(moe):
     """The 1,048,576 x 64 routing stress, compared token by token."""
     w = synth.WORKLOADS["route_t1m"]
