@@ -115,10 +115,11 @@ moe_status moe_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, 
  * no counterpart; this is a packaging variant of the same dispatch kernels.
  *
  * Arguments and results are those of moe_dispatch, without the workspace. The
- * scratch (per-chunk counts and bases, 2 * 512 * 128 int32 plus the tile
- * offsets, about 513 KB) is a fixed array inside the library, which every GPU
- * that loads the library keeps until the process exits. Limits: T <= 1,048,576
- * tokens (larger T returns MOE_ERR_UNSUPPORTED), N in {64, 128}, K <= 8.
+ * scratch (per-chunk expert counts, 128 experts x 2048 chunks of 128 tokens,
+ * plus totals and tile offsets: about 1 MB) is a fixed array inside the
+ * library, which every GPU that loads the library keeps until the process
+ * exits. Limits: T <= 262,144 tokens (larger T returns MOE_ERR_UNSUPPORTED),
+ * N in {64, 128}, K <= 8.
  * No cudaMalloc, cudaFree or other allocating call is made.
  * The first call on each device looks up the array's device address (with
  * that device current) and caches it; make that first call before any stream
@@ -176,6 +177,23 @@ moe_status moe_read_device_error(const void* ws, void* stream);
  * device int32 that receives a nonzero code on a device timeout (may be NULL). */
 moe_status moe_router_logits(const uint16_t* x, const uint16_t* w_router, int64_t T, int d, int N,
                              float* logits, int32_t* err_word, void* stream);
+
+/* Router GEMM with the elbow routing fused into its epilogue (the layer's
+ * first stage): the same logits as moe_router_logits, routed exactly as
+ * elbow_route routes them. logits_out [T, N] may be NULL (the logits then stay
+ * on chip). chunk_counts [N][ceil(T/128)] int32 (may be NULL): the number of
+ * selected pairs of each expert in each chunk of 128 tokens. */
+moe_status moe_router_route(const uint16_t* x, const uint16_t* w_router, int64_t T, int d, int N,
+                            const moe_route_params* rp, float* logits_out, int32_t* k_out,
+                            int32_t* ids_out, float* gates_out, int32_t* chunk_counts,
+                            int32_t* err_word, void* stream);
+
+/* moe_expert_gate_up with the rows gathered from x [T, d] by perm (row r of
+ * expert e is token perm[r]), without a gathered copy of x. */
+moe_status moe_expert_gate_up_gathered(const uint16_t* x, int64_t T, const int32_t* perm,
+                                       const uint16_t* w_gate_up, const int32_t* offsets,
+                                       const int32_t* tile_off, int64_t P, int d, int N, int I,
+                                       uint16_t* h, int32_t* err_word, void* stream);
 
 /* Expert SwiGLU over dispatched rows: for each expert e and each row r in
  * [offsets[e], offsets[e+1]): h[r] = silu(W_gate[e] xs[r]) * (W_up[e] xs[r]),

@@ -77,6 +77,8 @@ def library():
             "moe_expert_down": ([P, P, P, P, i64, i32, i32, i32, P, P, P], i32),
             "moe_gather_rows": ([P, P, P, i64, i64, i32, i32, P, P], i32),
             "moe_combine": ([P, P, P, P, P, i64, i32, i32, P, P], i32),
+            "moe_router_route": ([P, P, i64, i32, i32, RP, P, P, P, P, P, P, P], i32),
+            "moe_expert_gate_up_gathered": ([P, i64, P, P, P, P, i64, i32, i32, i32, P, P, P], i32),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -244,6 +246,40 @@ def router_logits(x, w_router, err=None, stream=None):
     _check(library().moe_router_logits(_p(x), _p(w_router), T, d, N, _p(out), _p(err),
                                        _stream(stream)), "moe_router_logits")
     return out
+
+
+def router_route(x, w_router, K: int = 8, eps: float = 1e-8, mode: int = MODE_ELBOW,
+                 renorm: int = 0, with_logits: bool = True, with_counts: bool = True, err=None,
+                 stream=None):
+    """Router GEMM with the elbow routing in its epilogue. Returns
+    (k, ids, gates, logits or None, chunk_counts [N, ceil(T/128)] or None)."""
+    torch = _torch()
+    _cuda(x, torch.bfloat16, "x")
+    _cuda(w_router, torch.bfloat16, "w_router")
+    T, d = x.shape
+    N = w_router.shape[0]
+    dev = x.device
+    k = torch.empty(T, dtype=torch.int32, device=dev)
+    ids = torch.empty(T, K, dtype=torch.int32, device=dev)
+    gates = torch.empty(T, K, dtype=torch.float32, device=dev)
+    lg = torch.empty(T, N, dtype=torch.float32, device=dev) if with_logits else None
+    cc = (torch.zeros(N, (T + 127) // 128, dtype=torch.int32, device=dev)
+          if with_counts else None)
+    _check(library().moe_router_route(_p(x), _p(w_router), T, d, N, _params(K, eps, mode, renorm),
+                                      _p(lg), _p(k), _p(ids), _p(gates), _p(cc), _p(err),
+                                      _stream(stream)), "moe_router_route")
+    return k, ids, gates, lg, cc
+
+
+def expert_gate_up_gathered(x, perm, w_gate_up, offsets, tile_off, P: int, err=None, stream=None):
+    torch = _torch()
+    T, d = x.shape
+    N, I2, _ = w_gate_up.shape
+    h = torch.empty(max(P, 1), I2 // 2, dtype=torch.bfloat16, device=x.device)
+    _check(library().moe_expert_gate_up_gathered(_p(x), T, _p(perm), _p(w_gate_up), _p(offsets),
+                                                 _p(tile_off), P, d, N, I2 // 2, _p(h), _p(err),
+                                                 _stream(stream)), "moe_expert_gate_up_gathered")
+    return h
 
 
 def gather_rows(x, perm, offsets, P: int, stream=None):

@@ -28,7 +28,7 @@ def nvcc() -> str:
 
 
 def _deps():
-    files = [os.path.join(CSRC, s) for s in SOURCES] + [os.path.join(CSRC, "common.cuh"),
+    files = [os.path.join(CSRC, s) for s in SOURCES] + [os.path.join(CSRC, "common.cuh"), os.path.join(CSRC, "route_impl.cuh"),
                                                         os.path.join(ROOT, "include", "elbow_moe.h"),
                                                         os.path.abspath(__file__)]
     return max(os.path.getmtime(f) for f in files)

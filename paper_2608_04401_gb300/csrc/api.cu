@@ -8,12 +8,13 @@
 namespace moe {
 cudaError_t launch_elbow_route(const float* logits, int64_t T, int N, int K, float eps,
                                int topk_mode, int renorm, int32_t* k_out, int32_t* ids_out,
-                               float* gates_out, cudaStream_t stream);
+                               float* gates_out, int32_t* blk_cnt, cudaStream_t stream);
 size_t dispatch_ws_bytes(int64_t T, int N);
 int32_t* dispatch_tile_off(void* ws, int64_t T, int N);
+int32_t* dispatch_counts(void* ws);
 cudaError_t launch_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
                             int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
-                            int32_t* offsets_copy, cudaStream_t stream);
+                            int32_t* offsets_copy, bool counts_ready, cudaStream_t stream);
 cudaError_t launch_gather(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int N,
                           int64_t P, int d, uint16_t* xs, int num_sms, cudaStream_t stream);
 cudaError_t launch_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_pos,
@@ -27,6 +28,14 @@ cudaError_t launch_gateup_gemm(const uint16_t* xs, const uint16_t* wgu, const in
 cudaError_t launch_down_gemm(const uint16_t* h, const uint16_t* wd, const int32_t* offsets,
                              const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* o,
                              int32_t* err, int num_sms, cudaStream_t stream);
+cudaError_t launch_router_route(const uint16_t* x, const uint16_t* wr, int64_t T, int d, int N,
+                                int K, float eps, int topk_mode, int renorm, float* logits_out,
+                                int32_t* k_out, int32_t* ids_out, float* gates_out,
+                                int32_t* blk_cnt, int32_t* err, int num_sms, cudaStream_t stream);
+cudaError_t launch_gateup_gather_gemm(const uint16_t* x, int64_t T, const int32_t* perm,
+                                      const uint16_t* wgu, const int32_t* offsets,
+                                      const int32_t* tile_off, int64_t P, int d, int N, int I,
+                                      uint16_t* h, int32_t* err, int num_sms, cudaStream_t stream);
 }  // namespace moe
 
 namespace {
@@ -60,12 +69,11 @@ moe_status check_route_params(const moe_route_params* rp, int N) {
 bool supported_n(int N) { return N == 64 || N == 128; }
 
 // Layer workspace layout (every region 256-byte aligned):
-//   header (error word) | logits [T,N] f32 | k [T] | ids [T,K] | gates [T,K]
-//   | offsets [N+1] | dispatch scratch | perm [T*K] | pair_pos [T*K]
-//   | xs [T*K, d] bf16 | h [T*K, I] bf16 | o [T*K, d] bf16
+//   header (error word) | k [T] | ids [T,K] | gates [T,K] | offsets [N+1]
+//   | dispatch scratch | perm [T*K] | pair_pos [T*K] | h [T*K, I] bf16
+//   | o [T*K, d] bf16
 struct LayerWs {
   int32_t* err;
-  float* logits;
   int32_t* k;
   int32_t* ids;
   float* gates;
@@ -73,7 +81,6 @@ struct LayerWs {
   void* disp;
   int32_t* perm;
   int32_t* pair_pos;
-  uint16_t* xs;
   uint16_t* h;
   uint16_t* o;
   size_t bytes;
@@ -90,7 +97,6 @@ LayerWs layer_ws(void* base, int64_t T, int d, int N, int I, int K) {
   };
   const size_t P = static_cast<size_t>(T) * K;
   w.err = reinterpret_cast<int32_t*>(take(256));
-  w.logits = reinterpret_cast<float*>(take(sizeof(float) * T * N));
   w.k = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * T));
   w.ids = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * P));
   w.gates = reinterpret_cast<float*>(take(sizeof(float) * P));
@@ -98,7 +104,6 @@ LayerWs layer_ws(void* base, int64_t T, int d, int N, int I, int K) {
   w.disp = take(moe::dispatch_ws_bytes(T, N));
   w.perm = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * (P > 0 ? P : 1)));
   w.pair_pos = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * (P > 0 ? P : 1)));
-  w.xs = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * P * d));
   w.h = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * P * I));
   w.o = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * P * d));
   w.bytes = off;
@@ -133,7 +138,7 @@ moe_status elbow_route(const float* logits, int64_t T, int N, const moe_route_pa
       (reinterpret_cast<uintptr_t>(k_out) & 3u))
     return MOE_ERR_INVALID_ARG;
   return cuda_status(moe::launch_elbow_route(logits, T, N, rp->K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
-                                             rp->renorm, k_out, ids_out, gates_out,
+                                             rp->renorm, k_out, ids_out, gates_out, nullptr,
                                              static_cast<cudaStream_t>(stream)));
 }
 
@@ -158,8 +163,9 @@ moe_status moe_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, 
   if (T > 0 && (!k || !ids || !perm || !pair_pos)) return MOE_ERR_INVALID_ARG;
   if (ws_bytes < moe::dispatch_ws_bytes(T, N)) return MOE_ERR_WORKSPACE;
   if ((reinterpret_cast<uintptr_t>(ws) & 255u)) return MOE_ERR_INVALID_ARG;
+  if (T > 0 && !aligned16(ids)) return MOE_ERR_INVALID_ARG;
   return cuda_status(moe::launch_dispatch(k, ids, T, N, K, offsets, perm, pair_pos, ws, nullptr,
-                                          static_cast<cudaStream_t>(stream)));
+                                          false, static_cast<cudaStream_t>(stream)));
 }
 
 size_t moe_layer_workspace_size(int64_t T, int d, int N, int I, int K) {
@@ -197,7 +203,6 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
       (offsets_out && (reinterpret_cast<uintptr_t>(offsets_out) & 3u)))
     return MOE_ERR_INVALID_ARG;
 
-  float* logits = logits_out ? logits_out : w.logits;
   int32_t* kk = k_out ? k_out : w.k;
   int32_t* ids = ids_out ? ids_out : w.ids;
   float* gates = gates_out ? gates_out : w.gates;
@@ -205,17 +210,19 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   const int nsm = sm_count();
 
   cudaError_t e;
-  e = moe::launch_router_gemm(x, w_router, T, d, N, logits, w.err, nsm, s);
+  // router GEMM with the elbow routing in its epilogue; it also leaves the
+  // per-chunk expert counts of the dispatch
+  e = moe::launch_router_route(x, w_router, T, d, N, K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
+                               rp->renorm, logits_out, kk, ids, gates, moe::dispatch_counts(w.disp),
+                               w.err, nsm, s);
   if (e != cudaSuccess) return MOE_ERR_CUDA;
-  e = moe::launch_elbow_route(logits, T, N, K, rp->eps, rp->mode == MOE_ROUTE_TOPK, rp->renorm, kk,
-                              ids, gates, s);
-  if (e != cudaSuccess) return MOE_ERR_CUDA;
-  e = moe::launch_dispatch(kk, ids, T, N, K, w.offsets, w.perm, w.pair_pos, w.disp, offsets_out, s);
+  e = moe::launch_dispatch(kk, ids, T, N, K, w.offsets, w.perm, w.pair_pos, w.disp, offsets_out,
+                           true, s);
   if (e != cudaSuccess) return MOE_ERR_CUDA;
   const int32_t* tile_off = moe::dispatch_tile_off(w.disp, T, N);
-  e = moe::launch_gather(x, w.perm, w.offsets, N, P, d, w.xs, nsm, s);
-  if (e != cudaSuccess) return MOE_ERR_CUDA;
-  e = moe::launch_gateup_gemm(w.xs, w_gate_up, w.offsets, tile_off, P, d, N, I, w.h, w.err, nsm, s);
+  // gate/up GEMM gathers its token rows itself (no dispatched copy of x)
+  e = moe::launch_gateup_gather_gemm(x, T, w.perm, w_gate_up, w.offsets, tile_off, P, d, N, I, w.h,
+                                     w.err, nsm, s);
   if (e != cudaSuccess) return MOE_ERR_CUDA;
   e = moe::launch_down_gemm(w.h, w_down, w.offsets, tile_off, P, d, N, I, w.o, w.err, nsm, s);
   if (e != cudaSuccess) return MOE_ERR_CUDA;
@@ -283,6 +290,42 @@ moe_status moe_gather_rows(const uint16_t* x, const int32_t* perm, const int32_t
   if (!x || !perm || !offsets || !xs || !aligned16(x) || !aligned16(xs)) return MOE_ERR_INVALID_ARG;
   return cuda_status(moe::launch_gather(x, perm, offsets, N, P, d, xs, sm_count(),
                                         static_cast<cudaStream_t>(stream)));
+}
+
+moe_status moe_router_route(const uint16_t* x, const uint16_t* w_router, int64_t T, int d, int N,
+                            const moe_route_params* rp, float* logits_out, int32_t* k_out,
+                            int32_t* ids_out, float* gates_out, int32_t* chunk_counts,
+                            int32_t* err_word, void* stream) {
+  if (T < 0 || T > kMaxTokens) return MOE_ERR_INVALID_ARG;
+  if (!supported_n(N) || d <= 0 || d > kMaxDim || d % 64 != 0) return MOE_ERR_UNSUPPORTED;
+  moe_status st = check_route_params(rp, N);
+  if (st != MOE_OK) return st;
+  if (T == 0) return MOE_OK;
+  if (!x || !w_router || !k_out || !ids_out || !gates_out || !aligned16(x) || !aligned16(w_router) ||
+      !aligned16(ids_out) || !aligned16(gates_out) || (logits_out && !aligned16(logits_out)) ||
+      (reinterpret_cast<uintptr_t>(k_out) & 3u))
+    return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_router_route(x, w_router, T, d, N, rp->K, rp->eps,
+                                              rp->mode == MOE_ROUTE_TOPK, rp->renorm, logits_out,
+                                              k_out, ids_out, gates_out, chunk_counts, err_word,
+                                              sm_count(), static_cast<cudaStream_t>(stream)));
+}
+
+moe_status moe_expert_gate_up_gathered(const uint16_t* x, int64_t T, const int32_t* perm,
+                                       const uint16_t* w_gate_up, const int32_t* offsets,
+                                       const int32_t* tile_off, int64_t P, int d, int N, int I,
+                                       uint16_t* h, int32_t* err_word, void* stream) {
+  if (T < 0 || P < 0 || P > kMaxTokens * 8) return MOE_ERR_INVALID_ARG;
+  if (!supported_n(N) || d <= 0 || d > kMaxDim || d % 64 != 0 || I <= 0 || I > kMaxDim ||
+      I % 128 != 0)
+    return MOE_ERR_UNSUPPORTED;
+  if (P == 0 || T == 0) return MOE_OK;
+  if (!x || !perm || !w_gate_up || !offsets || !tile_off || !h || !aligned16(x) ||
+      !aligned16(w_gate_up) || !aligned16(h))
+    return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_gateup_gather_gemm(x, T, perm, w_gate_up, offsets, tile_off, P, d, N,
+                                                    I, h, err_word, sm_count(),
+                                                    static_cast<cudaStream_t>(stream)));
 }
 
 moe_status moe_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_pos,

@@ -1,14 +1,17 @@
 // Token-to-expert dispatch of the selected (t, s < k_t) pairs, stable in t,
 // plus the row gather and the gate-weighted combine.
 //
-// Dispatch is a deterministic three-pass counting sort over token chunks:
-//   count   : per chunk (kChunk tokens), per-expert pair counts (smem atomics:
-//             the counts do not depend on their order)
-//   scan    : per expert, exclusive prefix over chunks; per-expert totals ->
-//             offsets [N+1]; m-tile prefix ceil(count_e / 128) -> tile_off
-//   scatter : each chunk walks its tokens in order, 32 per warp; a pair's
-//             position = chunk base + earlier warps of this round (ballots in
-//             smem) + earlier lanes of this warp (popc of the ballot).
+// Dispatch is a deterministic counting sort over chunks of 128 tokens:
+//   count   : per chunk, per-expert pair counts (warp ballots), stored
+//             expert-major: cnt[e][chunk]. The elbow router can write these
+//             itself, in which case this pass is skipped.
+//   scan    : one block per expert: exclusive prefix over the chunks, in
+//             place, and the expert's total.
+//   scatter : each chunk recomputes the expert offsets from the totals, then
+//             places its pairs: position = offsets[e] + chunk base + earlier
+//             warps of the chunk (ballots in smem) + earlier lanes of the warp
+//             (popc of the ballot). Chunk 0 also writes offsets [N+1] and the
+//             m-tile prefix sums ceil(count_e / 128) [N+1].
 #include <mutex>
 
 #include "common.cuh"
@@ -16,131 +19,193 @@
 namespace moe {
 namespace disp {
 
-constexpr int kThreads = 256;
-constexpr int kWarps = kThreads / 32;
-constexpr int kChunk = 2048;  // tokens per chunk (block)
+constexpr int kChunk = 128;  // tokens per chunk = threads per block
+constexpr int kWarps = kChunk / 32;
+constexpr int kScanThreads = 256;
 
-template <int N>
-__global__ void __launch_bounds__(kThreads) count_kernel(const int32_t* __restrict__ k,
-                                                         const int32_t* __restrict__ ids, int64_t T,
-                                                         int K, int32_t* __restrict__ blk_cnt) {
-  __shared__ int cnt[N];
-  for (int i = threadIdx.x; i < N; i += kThreads) cnt[i] = 0;
-  __syncthreads();
-  const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kChunk;
-  const int64_t t1 = min_of<int64_t>(T, t0 + kChunk);
-  for (int64_t t = t0 + threadIdx.x; t < t1; t += kThreads) {
-    const int kt = min(k[t], K);
-    for (int s = 0; s < kt; ++s) atomicAdd(&cnt[ids[t * K + s]], 1);
+// Expert-membership bit masks of one token's selection (experts 0..63, 64..127).
+MOE_DEV void load_selection(const int32_t* __restrict__ k, const int32_t* __restrict__ ids,
+                            int64_t t, bool valid, int K, int& kt, int (&my)[8], uint64_t& m0,
+                            uint64_t& m1) {
+  kt = valid ? min(k[t], K) : 0;
+  if (valid && K == 8) {
+    const int4 a = reinterpret_cast<const int4*>(ids + t * 8)[0];
+    const int4 b = reinterpret_cast<const int4*>(ids + t * 8)[1];
+    my[0] = a.x; my[1] = a.y; my[2] = a.z; my[3] = a.w;
+    my[4] = b.x; my[5] = b.y; my[6] = b.z; my[7] = b.w;
+  } else {
+#pragma unroll
+    for (int s = 0; s < 8; ++s) my[s] = (s < kt) ? ids[t * K + s] : 0;
   }
-  __syncthreads();
-  for (int i = threadIdx.x; i < N; i += kThreads) blk_cnt[static_cast<int64_t>(blockIdx.x) * N + i] = cnt[i];
-}
-
-// One block of 1024 threads: thread (g, e) owns expert e over the g-th slice
-// of the chunks.
-template <int N>
-__global__ void __launch_bounds__(1024) scan_kernel(const int32_t* __restrict__ blk_cnt, int nblk,
-                                                    int32_t* __restrict__ blk_base,
-                                                    int32_t* __restrict__ offsets,
-                                                    int32_t* __restrict__ tile_off,
-                                                    int32_t* __restrict__ offsets_copy) {
-  constexpr int G = 1024 / N;
-  __shared__ int part[G][N];
-  __shared__ int exp_off[N + 1];
-  const int e = threadIdx.x % N, g = threadIdx.x / N;
-  const int per = (nblk + G - 1) / G;
-  const int b0 = g * per, b1 = min(nblk, b0 + per);
-  int sum = 0;
-  for (int b = b0; b < b1; ++b) sum += blk_cnt[static_cast<int64_t>(b) * N + e];
-  part[g][e] = sum;
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    // totals per expert, then the exclusive scan over experts
-    int run = 0, trun = 0;
-    for (int x = 0; x < N; ++x) {
-      int tot = 0;
-      for (int y = 0; y < G; ++y) tot += part[y][x];
-      exp_off[x] = run;
-      offsets[x] = run;
-      tile_off[x] = trun;
-      if (offsets_copy) offsets_copy[x] = run;
-      run += tot;
-      trun += (tot + 127) / 128;
+  m0 = 0;
+  m1 = 0;
+#pragma unroll
+  for (int s = 0; s < 8; ++s) {
+    if (s < kt) {
+      if (my[s] < 64) m0 |= 1ull << my[s];
+      else m1 |= 1ull << (my[s] - 64);
     }
-    exp_off[N] = run;
-    offsets[N] = run;
-    tile_off[N] = trun;
-    if (offsets_copy) offsets_copy[N] = run;
-  }
-  __syncthreads();
-  int base = exp_off[e];
-  for (int y = 0; y < g; ++y) base += part[y][e];
-  for (int b = b0; b < b1; ++b) {
-    blk_base[static_cast<int64_t>(b) * N + e] = base;
-    base += blk_cnt[static_cast<int64_t>(b) * N + e];
   }
 }
 
 template <int N>
-__global__ void __launch_bounds__(kThreads) scatter_kernel(const int32_t* __restrict__ k,
-                                                           const int32_t* __restrict__ ids,
-                                                           int64_t T, int K,
-                                                           const int32_t* __restrict__ blk_base,
-                                                           int32_t* __restrict__ perm,
-                                                           int32_t* __restrict__ pair_pos) {
-  __shared__ int run[N];
+MOE_DEV bool has_expert(int e, uint64_t m0, uint64_t m1) {
+  return ((e < 64 ? (m0 >> e) : (m1 >> (e - 64))) & 1ull) != 0;
+}
+
+template <int N>
+__global__ void __launch_bounds__(kChunk) count_kernel(const int32_t* __restrict__ k,
+                                                       const int32_t* __restrict__ ids, int64_t T,
+                                                       int K, int nblk, int32_t* __restrict__ cnt) {
+  __shared__ int wcnt[kWarps][N];
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int64_t t = static_cast<int64_t>(blockIdx.x) * kChunk + threadIdx.x;
+  int kt, my[8];
+  uint64_t m0, m1;
+  load_selection(k, ids, t, t < T, K, kt, my, m0, m1);
+#pragma unroll
+  for (int e = 0; e < N; ++e) {
+    const int c = __popc(__ballot_sync(0xffffffffu, has_expert<N>(e, m0, m1)));
+    if (lane == (e & 31)) wcnt[warp][e] = c;
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < N; e += kChunk) {
+    int c = 0;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) c += wcnt[w][e];
+    cnt[static_cast<int64_t>(e) * nblk + blockIdx.x] = c;
+  }
+}
+
+// Block e: exclusive prefix sum of cnt[e][0 .. nblk) in place; total -> totals[e].
+// Thread i owns the contiguous range [i * per, (i + 1) * per): it sums it with
+// independent loads, the block scans the per-thread sums once, and each thread
+// rewrites its range with the running prefix.
+__global__ void __launch_bounds__(kScanThreads) scan_kernel(int32_t* __restrict__ cnt, int nblk,
+                                                            int32_t* __restrict__ totals) {
+  __shared__ int warp_sum[kScanThreads / 32];
+  int32_t* col = cnt + static_cast<int64_t>(blockIdx.x) * nblk;
+  const int lane = threadIdx.x % 32, warp = threadIdx.x / 32;
+  const int per = (nblk + kScanThreads - 1) / kScanThreads;
+  const int b0 = threadIdx.x * per;
+  const int b1 = min(nblk, b0 + per);
+  int sum = 0;
+#pragma unroll 8
+  for (int b = b0; b < b1; ++b) sum += col[b];
+  int x = sum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_sum[warp] = x;
+  __syncthreads();
+  int run = x - sum;
+  int total = 0;
+#pragma unroll
+  for (int w = 0; w < kScanThreads / 32; ++w) {
+    if (w < warp) run += warp_sum[w];
+    total += warp_sum[w];
+  }
+  for (int b = b0; b < b1; ++b) {
+    const int v = col[b];
+    col[b] = run;
+    run += v;
+  }
+  if (threadIdx.x == 0) totals[blockIdx.x] = total;
+}
+
+// Exclusive scan of N <= 128 values held by threads 0..N-1 of a 128-thread
+// block; every thread gets the scan of its own index (0 beyond N) and the total.
+template <int N>
+MOE_DEV int block_exclusive_scan_small(int v, int* warp_tmp, int& total) {
+  const int lane = threadIdx.x % 32, warp = threadIdx.x / 32;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) warp_tmp[warp] = x;
+  __syncthreads();
+  int before = 0;
+  total = 0;
+#pragma unroll
+  for (int w = 0; w < kWarps; ++w) {
+    if (w < warp) before += warp_tmp[w];
+    total += warp_tmp[w];
+  }
+  __syncthreads();
+  return before + x - v;
+}
+
+template <int N>
+__global__ void __launch_bounds__(kChunk) scatter_kernel(
+    const int32_t* __restrict__ k, const int32_t* __restrict__ ids, int64_t T, int K, int nblk,
+    const int32_t* __restrict__ base, const int32_t* __restrict__ totals,
+    int32_t* __restrict__ perm, int32_t* __restrict__ pair_pos, int32_t* __restrict__ offsets,
+    int32_t* __restrict__ tile_off, int32_t* __restrict__ offsets_copy) {
+  __shared__ int exp_off[N];
   __shared__ uint32_t bal[kWarps][N];
   __shared__ int wbase[kWarps][N];
+  __shared__ int warp_tmp[kWarps];
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  for (int i = threadIdx.x; i < N; i += kThreads) run[i] = blk_base[static_cast<int64_t>(blockIdx.x) * N + i];
-  const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kChunk;
-  const int64_t t1 = min_of<int64_t>(T, t0 + kChunk);
-  const uint32_t lt_mask = (1u << lane) - 1u;
-  for (int64_t r0 = t0; r0 < t1; r0 += kThreads) {
-    const int64_t t = r0 + threadIdx.x;
-    const bool valid = t < t1;
-    const int kt = valid ? min(k[t], K) : 0;
-    int my[8];
-    uint64_t m0 = 0, m1 = 0;
+  const int tid = threadIdx.x;
+
+  // expert offsets from the totals (every chunk recomputes them)
+  const int tot = tid < N ? totals[tid] : 0;
+  int total_pairs;
+  const int off = block_exclusive_scan_small<N>(tot, warp_tmp, total_pairs);
+  if (tid < N) exp_off[tid] = off;
+  if (blockIdx.x == 0) {
+    int total_tiles;
+    const int toff = block_exclusive_scan_small<N>(tid < N ? (tot + 127) / 128 : 0, warp_tmp,
+                                                   total_tiles);
+    if (tid < N) {
+      offsets[tid] = off;
+      tile_off[tid] = toff;
+      if (offsets_copy) offsets_copy[tid] = off;
+    }
+    if (tid == 0) {
+      offsets[N] = total_pairs;
+      tile_off[N] = total_tiles;
+      if (offsets_copy) offsets_copy[N] = total_pairs;
+    }
+  }
+
+  const int64_t t = static_cast<int64_t>(blockIdx.x) * kChunk + tid;
+  const bool valid = t < T;
+  int kt, my[8];
+  uint64_t m0, m1;
+  load_selection(k, ids, t, valid, K, kt, my, m0, m1);
+#pragma unroll
+  for (int e = 0; e < N; ++e) {
+    const uint32_t b = __ballot_sync(0xffffffffu, has_expert<N>(e, m0, m1));
+    if (lane == (e & 31)) bal[warp][e] = b;
+  }
+  __syncthreads();
+  for (int e = tid; e < N; e += kChunk) {
+    int acc = exp_off[e] + base[static_cast<int64_t>(e) * nblk + blockIdx.x];
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+      wbase[w][e] = acc;
+      acc += __popc(bal[w][e]);
+    }
+  }
+  __syncthreads();
+  if (valid) {
+    const uint32_t lt_mask = (1u << lane) - 1u;
 #pragma unroll
     for (int s = 0; s < 8; ++s) {
-      my[s] = (s < kt) ? ids[t * K + s] : -1;
-      if (s < kt) {
-        if (my[s] < 64) m0 |= 1ull << my[s];
-        else m1 |= 1ull << (my[s] - 64);
-      }
-    }
-    __syncthreads();  // previous round's readers of bal/wbase are done
-#pragma unroll
-    for (int e = 0; e < N; ++e) {
-      const bool has = ((e < 64 ? (m0 >> e) : (m1 >> (e - 64))) & 1ull) != 0;
-      const uint32_t b = __ballot_sync(0xffffffffu, has);
-      if (lane == (e & 31)) bal[warp][e] = b;
-    }
-    __syncthreads();
-    for (int e = threadIdx.x; e < N; e += kThreads) {
-      int acc = run[e];
-#pragma unroll
-      for (int w = 0; w < kWarps; ++w) {
-        wbase[w][e] = acc;
-        acc += __popc(bal[w][e]);
-      }
-      run[e] = acc;
-    }
-    __syncthreads();
-    if (valid) {
-#pragma unroll
-      for (int s = 0; s < 8; ++s) {
-        if (s < K) {
-          if (s < kt) {
-            const int e = my[s];
-            const int pos = wbase[warp][e] + __popc(bal[warp][e] & lt_mask);
-            perm[pos] = static_cast<int32_t>(t);
-            pair_pos[t * K + s] = pos;
-          } else {
-            pair_pos[t * K + s] = -1;
-          }
+      if (s < K) {
+        if (s < kt) {
+          const int e = my[s];
+          const int pos = wbase[warp][e] + __popc(bal[warp][e] & lt_mask);
+          // positions stay below T*K when the counts match the ids
+          if (pos >= 0 && static_cast<int64_t>(pos) < T * K) perm[pos] = static_cast<int32_t>(t);
+          pair_pos[t * K + s] = pos;
+        } else {
+          pair_pos[t * K + s] = -1;
         }
       }
     }
@@ -176,7 +241,7 @@ __global__ void __launch_bounds__(256) combine_kernel(const uint4* __restrict__ 
     float g[8];
 #pragma unroll
     for (int s = 0; s < 8; ++s) {
-      pos[s] = (s < kt) ? pair_pos[t * K + s] : 0;
+      pos[s] = (s < kt) ? min(max(pair_pos[t * K + s], 0), static_cast<int>(T * K - 1)) : 0;
       g[s] = (s < kt) ? gates[t * K + s] : 0.0f;
     }
     for (int c = threadIdx.x; c < d8; c += blockDim.x) {
@@ -216,41 +281,64 @@ __global__ void __launch_bounds__(256) combine_kernel(const uint4* __restrict__ 
 
 }  // namespace disp
 
+static int num_chunks(int64_t T) { return static_cast<int>((T + disp::kChunk - 1) / disp::kChunk); }
+
+// Workspace layout: cnt/base [N][nchunks] int32 | totals [N] | tile_off [N+1]
 size_t dispatch_ws_bytes(int64_t T, int N) {
-  const int64_t nblk = (T + disp::kChunk - 1) / disp::kChunk;
-  const size_t a = static_cast<size_t>(nblk > 0 ? nblk : 1) * N * sizeof(int32_t);
   auto up = [](size_t b) { return (b + 255) & ~static_cast<size_t>(255); };
-  return up(a) * 2 + up((N + 1) * sizeof(int32_t));
+  const size_t nblk = static_cast<size_t>(num_chunks(T) > 0 ? num_chunks(T) : 1);
+  return up(nblk * N * sizeof(int32_t)) + up(N * sizeof(int32_t)) + up((N + 1) * sizeof(int32_t));
 }
 
-// Workspace layout: blk_cnt [nblk][N] | blk_base [nblk][N] | tile_off [N+1]
+int32_t* dispatch_counts(void* ws) { return static_cast<int32_t*>(ws); }
+
+static int32_t* dispatch_totals(void* ws, int64_t T, int N) {
+  auto up = [](size_t b) { return (b + 255) & ~static_cast<size_t>(255); };
+  const size_t nblk = static_cast<size_t>(num_chunks(T) > 0 ? num_chunks(T) : 1);
+  return reinterpret_cast<int32_t*>(static_cast<char*>(ws) + up(nblk * N * sizeof(int32_t)));
+}
+
 int32_t* dispatch_tile_off(void* ws, int64_t T, int N) {
-  const int64_t nblk = (T + disp::kChunk - 1) / disp::kChunk;
-  const size_t a = static_cast<size_t>(nblk > 0 ? nblk : 1) * N * sizeof(int32_t);
-  const size_t up = (a + 255) & ~static_cast<size_t>(255);
-  return reinterpret_cast<int32_t*>(static_cast<char*>(ws) + 2 * up);
+  auto up = [](size_t b) { return (b + 255) & ~static_cast<size_t>(255); };
+  return reinterpret_cast<int32_t*>(reinterpret_cast<char*>(dispatch_totals(ws, T, N)) +
+                                    up(N * sizeof(int32_t)));
+}
+
+// counts_ready: the elbow router already wrote the per-chunk counts into
+// dispatch_counts(ws).
+static cudaError_t run_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
+                                int32_t* offsets, int32_t* perm, int32_t* pair_pos, int32_t* cnt,
+                                int32_t* totals, int32_t* tile_off, int32_t* offsets_copy,
+                                bool counts_ready, cudaStream_t stream) {
+  const int nblk = num_chunks(T);
+  if (nblk > 0 && !counts_ready) {
+    if (N == 64) disp::count_kernel<64><<<nblk, disp::kChunk, 0, stream>>>(k, ids, T, K, nblk, cnt);
+    else disp::count_kernel<128><<<nblk, disp::kChunk, 0, stream>>>(k, ids, T, K, nblk, cnt);
+  }
+  if (nblk > 0) {
+    disp::scan_kernel<<<N, disp::kScanThreads, 0, stream>>>(cnt, nblk, totals);
+  } else {
+    cudaError_t e = cudaMemsetAsync(totals, 0, N * sizeof(int32_t), stream);
+    if (e != cudaSuccess) return e;
+  }
+  const int grid = nblk > 0 ? nblk : 1;
+  if (N == 64)
+    disp::scatter_kernel<64><<<grid, disp::kChunk, 0, stream>>>(k, ids, T, K, nblk, cnt, totals, perm,
+                                                                pair_pos, offsets, tile_off,
+                                                                offsets_copy);
+  else
+    disp::scatter_kernel<128><<<grid, disp::kChunk, 0, stream>>>(k, ids, T, K, nblk, cnt, totals,
+                                                                 perm, pair_pos, offsets, tile_off,
+                                                                 offsets_copy);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
                             int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
-                            int32_t* offsets_copy, cudaStream_t stream) {
-  const int64_t nblk64 = (T + disp::kChunk - 1) / disp::kChunk;
-  const int nblk = static_cast<int>(nblk64);
-  const size_t a = static_cast<size_t>(nblk > 0 ? nblk : 1) * N * sizeof(int32_t);
-  const size_t up = (a + 255) & ~static_cast<size_t>(255);
-  int32_t* blk_cnt = static_cast<int32_t*>(ws);
-  int32_t* blk_base = reinterpret_cast<int32_t*>(static_cast<char*>(ws) + up);
-  int32_t* tile_off = dispatch_tile_off(ws, T, N);
-  if (N == 64) {
-    if (nblk > 0) disp::count_kernel<64><<<nblk, disp::kThreads, 0, stream>>>(k, ids, T, K, blk_cnt);
-    disp::scan_kernel<64><<<1, 1024, 0, stream>>>(blk_cnt, nblk, blk_base, offsets, tile_off, offsets_copy);
-    if (nblk > 0) disp::scatter_kernel<64><<<nblk, disp::kThreads, 0, stream>>>(k, ids, T, K, blk_base, perm, pair_pos);
-  } else {
-    if (nblk > 0) disp::count_kernel<128><<<nblk, disp::kThreads, 0, stream>>>(k, ids, T, K, blk_cnt);
-    disp::scan_kernel<128><<<1, 1024, 0, stream>>>(blk_cnt, nblk, blk_base, offsets, tile_off, offsets_copy);
-    if (nblk > 0) disp::scatter_kernel<128><<<nblk, disp::kThreads, 0, stream>>>(k, ids, T, K, blk_base, perm, pair_pos);
-  }
-  return cudaGetLastError();
+                            int32_t* offsets_copy, bool counts_ready, cudaStream_t stream) {
+  return run_dispatch(k, ids, T, N, K, offsets, perm, pair_pos, dispatch_counts(ws),
+                      dispatch_totals(ws, T, N), dispatch_tile_off(ws, T, N), offsets_copy,
+                      counts_ready, stream);
 }
 
 cudaError_t launch_gather(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int N,
@@ -292,10 +380,11 @@ cudaError_t launch_combine(const uint16_t* o, const int32_t* k, const int32_t* p
 // library holds the array until the process exits.
 namespace moe {
 namespace disp {
-constexpr int64_t kNoAllocMaxTokens = int64_t(1) << 20;  // 1,048,576 tokens
+constexpr int64_t kNoAllocMaxTokens = int64_t(1) << 18;  // 262,144 tokens
 constexpr int kNoAllocMaxExperts = 128;
 constexpr int64_t kNoAllocChunks = (kNoAllocMaxTokens + kChunk - 1) / kChunk;
-constexpr int64_t kNoAllocInts = 2 * kNoAllocChunks * kNoAllocMaxExperts + 256;  // ~513 KB
+// counts [experts][chunks], totals [experts], tile offsets [experts + 1]: ~1 MB
+constexpr int64_t kNoAllocInts = kNoAllocChunks * kNoAllocMaxExperts + 2 * kNoAllocMaxExperts + 64;
 }  // namespace disp
 }  // namespace moe
 
@@ -335,24 +424,17 @@ extern "C" moe_status moe_dispatch_noalloc(const int32_t* k, const int32_t* ids,
   if ((N != 64 && N != 128) || K < 1 || K > 8 || K > N) return MOE_ERR_UNSUPPORTED;
   if (!offsets) return MOE_ERR_INVALID_ARG;
   if (T > 0 && (!k || !ids || !perm || !pair_pos)) return MOE_ERR_INVALID_ARG;
+  if (T > 0 && (reinterpret_cast<uintptr_t>(ids) & 15u)) return MOE_ERR_INVALID_ARG;
   int32_t* scratch = nullptr;
   if (noalloc_scratch(&scratch) != cudaSuccess) return MOE_ERR_CUDA;
-  // Layout: per-chunk counts [chunks][N] | per-chunk bases [chunks][N] | tile offsets
-  // [N+1]. The counts and bases of every chunk in use and all N+1 tile offsets are
-  // rewritten by each call, so nothing has to be cleared first.
-  int32_t* blk_cnt = scratch;
-  int32_t* blk_base = scratch + kNoAllocChunks * kNoAllocMaxExperts;
-  int32_t* tile_off = scratch + 2 * kNoAllocChunks * kNoAllocMaxExperts;
-  const int nblk = static_cast<int>((T + kChunk - 1) / kChunk);
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (N == 64) {
-    if (nblk > 0) count_kernel<64><<<nblk, kThreads, 0, s>>>(k, ids, T, K, blk_cnt);
-    scan_kernel<64><<<1, 1024, 0, s>>>(blk_cnt, nblk, blk_base, offsets, tile_off, nullptr);
-    if (nblk > 0) scatter_kernel<64><<<nblk, kThreads, 0, s>>>(k, ids, T, K, blk_base, perm, pair_pos);
-  } else {
-    if (nblk > 0) count_kernel<128><<<nblk, kThreads, 0, s>>>(k, ids, T, K, blk_cnt);
-    scan_kernel<128><<<1, 1024, 0, s>>>(blk_cnt, nblk, blk_base, offsets, tile_off, nullptr);
-    if (nblk > 0) scatter_kernel<128><<<nblk, kThreads, 0, s>>>(k, ids, T, K, blk_base, perm, pair_pos);
-  }
+  // Layout: per-chunk counts [N][chunks] | totals [N] | tile offsets [N+1]. The
+  // counts of every chunk in use, the totals and all N+1 tile offsets are
+  // rewritten by each call before they are read, so nothing has to be cleared.
+  int32_t* cnt = scratch;
+  int32_t* totals = scratch + kNoAllocChunks * kNoAllocMaxExperts;
+  int32_t* tile_off = totals + kNoAllocMaxExperts;
+  if (moe::run_dispatch(k, ids, T, N, K, offsets, perm, pair_pos, cnt, totals, tile_off, nullptr,
+                        false, static_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return MOE_ERR_CUDA;
   return cudaGetLastError() == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
 }

@@ -1,10 +1,17 @@
 // Persistent tcgen05 GEMMs with TMA-fed shared-memory pipelines and TMEM
 // accumulators, for the three contractions of the layer:
 //
-//   kRouter : logits[T, N]  = x[T, d] . W_r[N, d]^T              (fp32 out)
-//   kGateUp : h[P, I]       = silu(xs W_gate[e]^T) * (xs W_up[e]^T), per expert
-//             e over its dispatched rows [offsets[e], offsets[e+1])   (bf16 out)
-//   kDown   : o[P, d]       = h W_down[e]^T, per expert            (bf16 out)
+//   kRouter       : logits[T, N] = x[T, d] . W_r[N, d]^T             (fp32 out)
+//   kRouterFused  : the same, with the elbow routing of each token run in the
+//                   epilogue (one epilogue thread per token row, the logits
+//                   staged in shared memory), plus the dispatch's per-chunk
+//                   expert counts; the logits need not leave the chip
+//   kGateUp       : h[P, I] = silu(xs W_gate[e]^T) * (xs W_up[e]^T), per expert
+//                   e over its dispatched rows [offsets[e], offsets[e+1]) (bf16)
+//   kGateUpGather : the same, with the A rows gathered from x[T, d] by the
+//                   dispatch permutation (cp.async into the swizzled layout),
+//                   so the dispatched copy of x is never materialised
+//   kDown         : o[P, d] = h W_down[e]^T, per expert                 (bf16 out)
 //
 // Both operands are K-major bf16 tiles of 64 columns (128 bytes) moved by TMA
 // with 128-byte swizzle; the MMA is tcgen05.mma.cta_group::1.kind::f16 with
@@ -14,7 +21,7 @@
 // halves of the SwiGLU and the epilogue fuses silu(g) * u.
 //
 // Warp roles (192 threads, one CTA per SM):
-//   warp 0     : TMA producer (one elected lane)
+//   warp 0     : TMA producer (one elected lane; all 32 lanes for gathers)
 //   warp 1     : TMEM allocator + MMA issuer (one elected lane)
 //   warps 2..5 : epilogue; warp w reads TMEM lanes [32 (w % 4), +32)
 // Two TMEM accumulators (2 x BN columns) let the epilogue of tile i overlap
@@ -28,21 +35,45 @@
 // that stops its other roles, drains what it has in flight, frees its TMEM and
 // writes an error code into the caller's error word.
 #include "common.cuh"
+#include "route_impl.cuh"
 
 namespace moe {
 namespace gemm {
 
 constexpr int BM = 128;
 constexpr int BK = 64;
-constexpr int kThreads = 192;
-enum Mode { kRouter = 0, kGateUp = 1, kDown = 2 };
+// Warps: kProdWarps producers, one MMA warp, four epilogue warps.
+template <int MODE>
+struct Roles {
+  static constexpr int kProdWarps = MODE == 3 ? 4 : 1;  // gathered A rows: four copy warps
+  static constexpr int kMmaWarp = kProdWarps;
+  static constexpr int kEpiWarp0 = kProdWarps + 1;
+  static constexpr int kThreads = 32 * (kProdWarps + 5);
+};
+enum Mode { kRouter = 0, kGateUp = 1, kDown = 2, kGateUpGather = 3, kRouterFused = 4 };
 
-template <int BN>
+template <int MODE>
+__host__ __device__ constexpr bool is_router() { return MODE == kRouter || MODE == kRouterFused; }
+template <int MODE>
+__host__ __device__ constexpr bool is_gateup() { return MODE == kGateUp || MODE == kGateUpGather; }
+
+// Routing constants for the fused router epilogue (x'_i for i < N, and the
+// fast-path bound), in the layout route_token expects.
+struct RouteX {
+  float x[128];
+  float bound;
+};
+
+template <int MODE, int BN>
 struct Cfg {
   static constexpr int kABytes = BM * BK * 2;
   static constexpr int kBBytes = BN * BK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kStages = (192 * 1024) / kStageBytes;
+  // fused routing: logit rows [128][BN + 4] fp32, 8 x 128 key slots, histogram
+  static constexpr int kRouteTileBytes = 128 * (BN + 4) * 4;
+  static constexpr int kRouteBytes =
+      MODE == kRouterFused ? kRouteTileBytes + 8 * 128 * 8 + BN * 4 : 0;
+  static constexpr int kStages = (208 * 1024 - kRouteBytes) / kStageBytes;
   static constexpr int kTmemCols = (2 * BN <= 64) ? 64 : (2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512));
   static constexpr int kBarOff = kStages * kStageBytes;
   // barriers: full[S], empty[S], tfull[2], tempty[2], drain
@@ -50,7 +81,9 @@ struct Cfg {
   static constexpr int kMiscOff = kBarOff + kNumBars * 8;
   static constexpr int kTableOff = kMiscOff + 16;
   static constexpr int kMaxGroups = 128;
-  static constexpr int kSmemBytes = kTableOff + 2 * (kMaxGroups + 1) * 4 + 1024;  // + align slack
+  static constexpr int kRouteOff = (kTableOff + 2 * (kMaxGroups + 1) * 4 + 15) & ~15;
+  static constexpr int kSmemBytes = kRouteOff + kRouteBytes + 1024;  // + align slack
+  static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 };
 
 struct Args {
@@ -65,6 +98,17 @@ struct Args {
   void* out;
   int64_t ldo;              // output row stride, elements
   int32_t* err;             // device error word (may be null)
+  const int32_t* perm;      // kGateUpGather: token of each dispatched row
+  const void* a_src;        // kGateUpGather: x [m_rows, lda] bf16
+  int64_t lda;
+  // kRouterFused
+  RouteX rx;
+  int K, topk_mode, renorm, nblk;
+  float eps;
+  int32_t* k_out;
+  int32_t* ids_out;
+  float* gates_out;
+  int32_t* blk_cnt;         // [N][nblk] per-128-token-chunk expert counts (may be null)
 };
 
 struct Tile {
@@ -74,7 +118,7 @@ struct Tile {
 template <int MODE>
 MOE_DEV Tile decode(int tile, const Args& a, const int* s_off, const int* s_toff) {
   Tile t;
-  if (MODE == kRouter) {
+  if (is_router<MODE>()) {
     t.g = 0;
     t.nb = 0;
     t.row0 = tile * BM;
@@ -98,11 +142,44 @@ MOE_DEV Tile decode(int tile, const Args& a, const int* s_off, const int* s_toff
 
 MOE_DEV float silu(float g) { return g / (1.0f + __expf(-g)); }
 
+MOE_DEV void cp_async_16(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+MOE_DEV void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+// Arrive on `bar` once all prior cp.async of this thread have completed (the
+// barrier's expected count includes this arrival).
+MOE_DEV void cp_async_arrive_noinc(uint32_t bar) {
+  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
+}
+template <int N>
+MOE_DEV void cp_async_wait_group() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Named barrier among the four epilogue warps.
+MOE_DEV void epilogue_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+// Named barrier among the four epilogue warps that also ANDs a predicate.
+MOE_DEV bool epilogue_all(bool v) {
+  int r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.s32 p, %1, 0;\n\t"
+      "bar.red.and.pred q, 1, 128, p;\n\t"
+      "selp.s32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(v ? 1 : 0)
+      : "memory");
+  return r != 0;
+}
+
 template <int MODE, int BN>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                const Args args) {
-  using C = Cfg<BN>;
+                const __grid_constant__ Args args) {
+  using C = Cfg<MODE, BN>;
+  using R = Roles<MODE>;
+  constexpr int kThreads = R::kThreads;
   constexpr int S = C::kStages;
   constexpr uint32_t kIdesc = idesc_bf16_f32(BM, BN);
 
@@ -124,7 +201,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      mbar_init(full_bar(s), 1);
+      // gathered mode: the expect-tx arrival for B plus one arrival per
+      // producer lane for its A copies
+      mbar_init(full_bar(s), MODE == kGateUpGather ? 1 + 32 * R::kProdWarps : 1);
       mbar_init(empty_bar(s), 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -135,7 +214,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (MODE != kRouter) {
+  if (!is_router<MODE>()) {  // grouped schedule tables (router modes have none)
     for (int i = threadIdx.x; i <= args.groups; i += kThreads) {
       s_off[i] = args.offsets[i];
       s_toff[i] = args.tile_off[i];
@@ -145,7 +224,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     prefetch_tensormap(&tmA);
     prefetch_tensormap(&tmB);
   }
-  if (warp == 1) {
+  if (warp == R::kMmaWarp) {
     __syncwarp();
     tmem_alloc<C::kTmemCols>(smem_u32(tmem_slot));
     tmem_relinquish();
@@ -155,10 +234,65 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  const int total = (MODE == kRouter) ? static_cast<int>((args.m_rows + BM - 1) / BM)
-                                      : s_toff[args.groups] * args.n_tiles;
+  const int total = is_router<MODE>() ? static_cast<int>((args.m_rows + BM - 1) / BM)
+                                       : s_toff[args.groups] * args.n_tiles;
 
-  if (warp == 0) {
+  if (MODE == kGateUpGather && warp < R::kProdWarps) {
+    // --------------------------------------- producers, gathered A rows
+    // A: cp.async, 16 bytes per lane, written straight into the 128B-swizzled
+    // K-major layout (chunk c of row r at r * 128 + ((c ^ (r & 7)) << 4)).
+    // Producer warp w owns rows 32w .. 32w+31; its copy i covers rows
+    // 32w + 4i .. +3 (lane l: row 32w + 4i + (l >> 3), chunk l & 7), four full
+    // 128-byte lines per copy. Each lane then arms an arrival on the stage's
+    // full barrier that fires when its copies have landed
+    // (cp.async.mbarrier.arrive.noinc); the MMA thread fences the async proxy
+    // after its wait. Lane 0 of warp 0 also brings B by TMA.
+    const __nv_bfloat16* xg = static_cast<const __nv_bfloat16*>(args.a_src);
+    const int chunk = lane & 7;
+    int stage = 0;
+    uint32_t phase = 0;
+    int issued = 0;
+    for (int tile = blockIdx.x; tile < total && !*abort_flag; tile += gridDim.x) {
+      const Tile t = decode<MODE>(tile, args, s_off, s_toff);
+      int64_t roff[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int r = 32 * warp + 4 * i + (lane >> 3);
+        int tok = args.perm[t.row0 + (r < t.rows ? r : 0)];
+        tok = min(max(tok, 0), static_cast<int>(args.m_rows - 1));
+        roff[i] = static_cast<int64_t>(tok) * args.lda + chunk * 8;
+      }
+      bool ok_tile = true;
+      for (int kb = 0; kb < args.k_blocks; ++kb) {
+        int ok = 1;
+        if (lane == 0) ok = mbar_wait_bounded(empty_bar(stage), phase ^ 1u, abort_flag) ? 1 : 0;
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) { ok_tile = false; break; }
+        const uint32_t a_dst = sbase + stage * C::kStageBytes;
+        const uint32_t b_dst = a_dst + C::kABytes;
+        if (warp == 0 && lane == 0) {
+          mbar_arrive_expect_tx(full_bar(stage), C::kBBytes);
+          const int brow = t.g * args.b_rows + t.nb * 128;
+          tma_load_2d(b_dst, &tmB, full_bar(stage), kb * BK, brow);
+          tma_load_2d(b_dst + 128 * BK * 2, &tmB, full_bar(stage), kb * BK, brow + args.b_half);
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int r = 32 * warp + 4 * i + (lane >> 3);
+          const uint32_t dst = a_dst + r * 128 + ((chunk ^ (r & 7)) << 4);
+          cp_async_16(dst, xg + roff[i] + kb * BK);
+        }
+        cp_async_arrive_noinc(full_bar(stage));
+        ++issued;
+        if (++stage == S) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      if (!ok_tile) break;
+    }
+    cp_async_wait_group<0>();  // nothing of this thread in flight at exit
+  } else if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       int stage = 0;
@@ -172,7 +306,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t b_dst = a_dst + C::kABytes;
           mbar_arrive_expect_tx(full_bar(stage), C::kStageBytes);
           tma_load_2d(a_dst, &tmA, full_bar(stage), kb * BK, t.row0);
-          if (MODE == kGateUp) {
+          if (is_gateup<MODE>()) {
             const int brow = t.g * args.b_rows + t.nb * 128;
             tma_load_2d(b_dst, &tmB, full_bar(stage), kb * BK, brow);
             tma_load_2d(b_dst + 128 * BK * 2, &tmB, full_bar(stage), kb * BK, brow + args.b_half);
@@ -199,7 +333,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-  } else if (warp == 1) {
+  } else if (warp == R::kMmaWarp) {
     // ----------------------------------------------------------------- MMA
     if (lane == 0) {
       int stage = 0;
@@ -215,6 +349,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = true;
         for (int kb = 0; kb < args.k_blocks; ++kb) {
           if (!mbar_wait_bounded(full_bar(stage), phase, abort_flag)) { ok = false; break; }
+          // A rows written by cp.async (generic proxy) are read by the tensor core
+          if (MODE == kGateUpGather) fence_proxy_async_smem();
           tc_fence_after();
           const uint32_t a_addr = sbase + stage * C::kStageBytes;
           const uint64_t adesc = smem_desc_sw128(a_addr);
@@ -244,7 +380,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    const int q = warp & 3;
+    const int q = warp & 3;  // the four epilogue warps cover the four TMEM lane quarters
     const int r = q * 32 + lane;
     int local = 0;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++local) {
@@ -252,8 +388,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int acc = local & 1;
       const uint32_t acc_phase = (local >> 1) & 1;
       const bool ok = mbar_wait_bounded(tfull_bar(acc), acc_phase, abort_flag);
-      // all lanes agree (and reconverge) before the warp-collective TMEM loads
-      if (!__all_sync(0xffffffffu, ok)) break;
+      if (MODE == kRouterFused) {
+        // all four epilogue warps take the same decision (they meet at named
+        // barriers below), and each warp reconverges
+        if (!epilogue_all(ok)) break;
+        __syncwarp();
+      } else {
+        // all lanes agree (and reconverge) before the warp-collective TMEM loads
+        if (!__all_sync(0xffffffffu, ok)) break;
+      }
       tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN;
       const bool valid = r < t.rows;
@@ -273,7 +416,51 @@ __global__ void __launch_bounds__(kThreads, 1)
                                   __uint_as_float(v[4 * u + 2]), __uint_as_float(v[4 * u + 3]));
           }
         }
-      } else if (MODE == kGateUp) {
+      } else if (MODE == kRouterFused) {
+        // logits -> this thread's row in shared memory (and to global if asked)
+        float* rtile = reinterpret_cast<float*>(smem + C::kRouteOff);
+        uint64_t* keys64 = reinterpret_cast<uint64_t*>(smem + C::kRouteOff + C::kRouteTileBytes);
+        int* hist = reinterpret_cast<int*>(smem + C::kRouteOff + C::kRouteTileBytes + 8 * 128 * 8);
+        float* row = rtile + r * (BN + 4);
+        float* gout = args.out ? static_cast<float*>(args.out) + grow * args.ldo : nullptr;
+#pragma unroll
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t v[32];
+          tmem_ld_32x32b_x32(taddr + c, v);
+          tmem_ld_wait();
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const float4 f = make_float4(__uint_as_float(v[4 * u]), __uint_as_float(v[4 * u + 1]),
+                                         __uint_as_float(v[4 * u + 2]), __uint_as_float(v[4 * u + 3]));
+            reinterpret_cast<float4*>(row + c)[u] = f;
+            if (valid && gout) reinterpret_cast<float4*>(gout + c)[u] = f;
+          }
+        }
+        // the accumulator is free once read: release it before routing
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(tempty_bar(acc));
+        if (args.blk_cnt) {
+          for (int e = r; e < BN; e += 128) hist[e] = 0;
+          epilogue_sync();
+        }
+        int ids_sel[8];
+        int k_sel = 0;
+        if (valid)
+          k_sel = route::route_token<BN, RouteX>(row, grow, r, args.K, args.eps, args.topk_mode,
+                                                 args.renorm, args.rx, keys64, args.k_out,
+                                                 args.ids_out, args.gates_out, ids_sel);
+        if (args.blk_cnt) {
+#pragma unroll
+          for (int s2 = 0; s2 < 8; ++s2)
+            if (s2 < k_sel && ids_sel[s2] >= 0 && ids_sel[s2] < BN) atomicAdd(&hist[ids_sel[s2]], 1);
+          epilogue_sync();
+          for (int e = r; e < BN; e += 128)
+            args.blk_cnt[static_cast<int64_t>(e) * args.nblk + tile] = hist[e];
+          epilogue_sync();
+        }
+        continue;
+      } else if (is_gateup<MODE>()) {
         __nv_bfloat16* out = static_cast<__nv_bfloat16*>(args.out) + grow * args.ldo + t.nb * 128;
 #pragma unroll 1
         for (int c = 0; c < 128; c += 32) {
@@ -326,7 +513,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   __syncthreads();
   if (threadIdx.x == 0 && *abort_flag && args.err) atomicExch(args.err, kDevErrTimeout);
-  if (warp == 1) {
+  if (warp == R::kMmaWarp) {
     __syncwarp();
     tc_fence_after();
     tmem_dealloc<C::kTmemCols>(tmem_base);
@@ -369,7 +556,7 @@ static bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t 
 template <int MODE, int BN>
 static cudaError_t launch_mode(const CUtensorMap& a, const CUtensorMap& b, const Args& args,
                                int grid, cudaStream_t stream) {
-  using C = Cfg<BN>;
+  using C = Cfg<MODE, BN>;
   static int attr_dev = -1;
   int dev = 0;
   cudaGetDevice(&dev);
@@ -379,7 +566,7 @@ static cudaError_t launch_mode(const CUtensorMap& a, const CUtensorMap& b, const
     if (e != cudaSuccess) return e;
     attr_dev = dev;
   }
-  gemm_kernel<MODE, BN><<<grid, kThreads, C::kSmemBytes, stream>>>(a, b, args);
+  gemm_kernel<MODE, BN><<<grid, Roles<MODE>::kThreads, C::kSmemBytes, stream>>>(a, b, args);
   return cudaGetLastError();
 }
 
@@ -404,6 +591,70 @@ cudaError_t launch_router_gemm(const uint16_t* x, const uint16_t* wr, int64_t T,
   const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
   if (N == 64) return launch_mode<kRouter, 64>(ma, mb, a, grid, stream);
   return launch_mode<kRouter, 128>(ma, mb, a, grid, stream);
+}
+
+// Router GEMM with the elbow routing in its epilogue: k/ids/gates per token and
+// the dispatch's per-chunk expert counts ([N][ceil(T/128)], may be null);
+// logits_out may be null.
+cudaError_t launch_router_route(const uint16_t* x, const uint16_t* wr, int64_t T, int d, int N,
+                                int K, float eps, int topk_mode, int renorm, float* logits_out,
+                                int32_t* k_out, int32_t* ids_out, float* gates_out,
+                                int32_t* blk_cnt, int32_t* err, int num_sms, cudaStream_t stream) {
+  using namespace gemm;
+  if (T == 0) return cudaSuccess;
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, x, d, T, BM) || !make_map(&mb, wr, d, N, N)) return cudaErrorInvalidValue;
+  Args a{};
+  a.groups = 1;
+  a.m_rows = T;
+  a.n_tiles = 1;
+  a.k_blocks = d / BK;
+  a.out = logits_out;
+  a.ldo = N;
+  a.err = err;
+  route::fill_route_consts(a.rx, N);
+  a.K = K;
+  a.eps = eps;
+  a.topk_mode = topk_mode;
+  a.renorm = renorm;
+  a.k_out = k_out;
+  a.ids_out = ids_out;
+  a.gates_out = gates_out;
+  a.blk_cnt = blk_cnt;
+  const int64_t tiles = (T + BM - 1) / BM;
+  a.nblk = static_cast<int>(tiles);
+  const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
+  if (N == 64) return launch_mode<kRouterFused, 64>(ma, mb, a, grid, stream);
+  return launch_mode<kRouterFused, 128>(ma, mb, a, grid, stream);
+}
+
+// h[P, I] = silu(x[perm] W_g^T) * (x[perm] W_u^T) per expert, rows gathered by TMA
+cudaError_t launch_gateup_gather_gemm(const uint16_t* x, int64_t T, const int32_t* perm,
+                                      const uint16_t* wgu, const int32_t* offsets,
+                                      const int32_t* tile_off, int64_t P, int d, int N, int I,
+                                      uint16_t* h, int32_t* err, int num_sms, cudaStream_t stream) {
+  using namespace gemm;
+  if (P == 0 || T == 0) return cudaSuccess;
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, x, d, T, BM) ||
+      !make_map(&mb, wgu, d, static_cast<uint64_t>(N) * 2 * I, 128))
+    return cudaErrorInvalidValue;
+  Args a{};
+  a.offsets = offsets;
+  a.tile_off = tile_off;
+  a.groups = N;
+  a.n_tiles = I / 128;
+  a.k_blocks = d / BK;
+  a.b_rows = 2 * I;
+  a.b_half = I;
+  a.out = h;
+  a.ldo = I;
+  a.err = err;
+  a.perm = perm;
+  a.m_rows = T;  // gathered token rows are clamped to [0, T)
+  a.a_src = x;
+  a.lda = d;
+  return launch_mode<kGateUpGather, 256>(ma, mb, a, num_sms, stream);
 }
 
 // h[P, I] = silu(xs W_g^T) * (xs W_u^T) per expert

@@ -1,0 +1,548 @@
+// Elbow router (Alg. 1 + the capped selection of Sec. 2.1), one THREAD per token.
+//
+// A block routes 128 tokens. Its [128, N] fp32 logit tile is staged through
+// shared memory with coalesced 16-byte loads (rows padded by 4 floats so that
+// each thread's row reads are bank-conflict free). Each thread keeps its
+// token's values in registers and evaluates, in fp32 with every operation
+// rounded to nearest even (explicit .rn intrinsics / PTX, no contraction):
+//   m = max_j l_j; e_j = EXP(l_j - m); s = balanced tree sum; p_j = e_j * (1/s)
+//   sort p descending; p' = (p_(i) - p_min) * (1 / ((p_max - p_min) + eps));
+//   x' = i / (N-1); D_i = (1 - p'_i) - x'_i; e = smallest argmax; k = min(e+1, K)
+//
+// Fast path. The elbow decision only needs the exact curve at the top ranks:
+// for every rank i, D_i <= fl(1 - x'_i), so ranks i >= kTop - 1 cannot beat a
+// head value >= fl(1 - x'_{kTop-1}). The thread therefore selects the kTop = 32
+// largest values exactly, with the expert id carried in the low bits of a
+// 32-bit key (the key orders by the truncated value, then by ascending id);
+// exact values come back from the shared-memory row by id, and two checks
+// prove that the selected ranks are the exact top ranks in exact order. Then:
+//   M_head = max_{i < K-1} D_i (first argmax), M_mid = max_{K-1 <= i < kTop-1} D_i
+//   M_head >= M_mid and M_head >= bound  ->  k = argmax + 1
+//   M_mid > M_head                        ->  k = K (the elbow lies at or past K-1)
+//   otherwise, or when a check fails      ->  exact full path (rare)
+// Sorting is by e, not p; p = fl(e * (1/s)) is monotone in e, so the curve is
+// the same, and ids inside groups of equal p are re-ordered by ascending id.
+// A p tie across the K boundary also takes the full path.
+//
+// Full path (fallback, one thread, same arithmetic): all N probabilities are
+// sorted with a 543/1471-comparator Batcher network of fmaxf/fminf, the elbow
+// is evaluated on every rank, and the top-K ids are recovered by a threshold
+// scan of the unsorted row plus an 8-key network.
+#pragma once
+
+#include <utility>
+
+#include "common.cuh"
+
+namespace moe {
+namespace route {
+
+// EXP: Cody & Waite (1980) argument reduction with ln 2 split in two (the high
+// part has 16 significant bits, so n * kLn2Hi is exact), a degree-7 Taylor
+// polynomial of exp on the reduced argument in Horner form with fused
+// multiply-adds, and scaling by 2^n built from the exponent bits. Results
+// below 2^-126, and arguments below -104, give zero.
+constexpr float kLog2e = 0x1.715476p+0f;  // fp32(1 / ln 2)
+constexpr float kLn2Hi = 0x1.62e4p-1f;    // ln 2 to 16 significant bits
+constexpr float kLn2Lo = 0x1.7f7d1cp-20f; // fp32(ln 2 - kLn2Hi)
+// Taylor coefficients 1/j!, each rounded once to fp32.
+constexpr float kTay0 = static_cast<float>(1.0 / 1.0);
+constexpr float kTay1 = static_cast<float>(1.0 / 1.0);
+constexpr float kTay2 = static_cast<float>(1.0 / 2.0);
+constexpr float kTay3 = static_cast<float>(1.0 / 6.0);
+constexpr float kTay4 = static_cast<float>(1.0 / 24.0);
+constexpr float kTay5 = static_cast<float>(1.0 / 120.0);
+constexpr float kTay6 = static_cast<float>(1.0 / 720.0);
+constexpr float kTay7 = static_cast<float>(1.0 / 5040.0);
+// Adding 1.5 * 2^23 to |t| < 2^22 rounds t to an integer (to nearest, ties to
+// even) in the low mantissa bits: that sum minus the constant is rint(t), and
+// its bit pattern minus kMagicBits is rint(t) as an integer.
+constexpr float kMagic = 0x1.8p23f;
+constexpr int32_t kMagicBits = 0x4B400000;
+
+constexpr int kTok = 128;  // tokens (threads) per block
+constexpr int kTop = 32;   // ranks selected exactly on the fast path
+
+// ------------------------------------------------------- packed fp32 pairs
+MOE_DEV uint64_t pk(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+MOE_DEV float lo_of(uint64_t v) { return __uint_as_float(static_cast<uint32_t>(v)); }
+MOE_DEV float hi_of(uint64_t v) { return __uint_as_float(static_cast<uint32_t>(v >> 32)); }
+MOE_DEV uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+MOE_DEV uint64_t sub2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+MOE_DEV uint64_t mul2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+MOE_DEV uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+MOE_DEV float max3f(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+MOE_DEV float min3f(float a, float b, float c) {
+  float r;
+  asm("min.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
+// EXP of two arguments z <= 0 at once with packed fp32 operations. z is
+// clamped at -104.5 (every z < -104 gives n < -126, i.e. zero, either way),
+// rint comes from the 1.5 * 2^23 addition, and an exponent below -126 is
+// clamped to a zero scale.
+MOE_DEV uint64_t exp_spec2(uint64_t z) {
+  z = pk(fmaxf(lo_of(z), -104.5f), fmaxf(hi_of(z), -104.5f));
+  const uint64_t t = mul2(z, pk(kLog2e, kLog2e));
+  const uint64_t tm = add2(t, pk(kMagic, kMagic));
+  const uint64_t n = sub2(tm, pk(kMagic, kMagic));
+  uint64_t r = fma2(n, pk(-kLn2Hi, -kLn2Hi), z);
+  r = fma2(n, pk(-kLn2Lo, -kLn2Lo), r);
+  uint64_t q = fma2(pk(kTay7, kTay7), r, pk(kTay6, kTay6));
+  q = fma2(q, r, pk(kTay5, kTay5));
+  q = fma2(q, r, pk(kTay4, kTay4));
+  q = fma2(q, r, pk(kTay3, kTay3));
+  q = fma2(q, r, pk(kTay2, kTay2));
+  q = fma2(q, r, pk(kTay1, kTay1));
+  q = fma2(q, r, pk(kTay0, kTay0));
+  // 2^n from the integer n = bits(tm) - kMagicBits; n < -126 -> +0.0
+  const int32_t b0 = max(__float_as_int(lo_of(tm)), kMagicBits - 127);
+  const int32_t b1 = max(__float_as_int(hi_of(tm)), kMagicBits - 127);
+  const uint64_t scale = pk(__int_as_float((b0 - kMagicBits + 127) << 23),
+                            __int_as_float((b1 - kMagicBits + 127) << 23));
+  return mul2(q, scale);
+}
+
+// -------------------------------------------------------- sorting networks
+// Batcher's odd-even merge sort network for M keys, as a flat comparator list
+// built at compile time (so that every register index is a constant).
+template <int M>
+struct OddEvenMergeNet {
+  static constexpr int count() {
+    int c = 0;
+    for (int p = 1; p < M; p <<= 1)
+      for (int k = p; k >= 1; k >>= 1)
+        for (int j = k % p; j + k < M; j += 2 * k)
+          for (int i = 0; i < k && i + j + k < M; ++i)
+            if ((i + j) / (2 * p) == (i + j + k) / (2 * p)) ++c;
+    return c;
+  }
+  static constexpr int kCount = count();
+  int lo[kCount];
+  int hi[kCount];
+  constexpr OddEvenMergeNet() : lo(), hi() {
+    int c = 0;
+    for (int p = 1; p < M; p <<= 1)
+      for (int k = p; k >= 1; k >>= 1)
+        for (int j = k % p; j + k < M; j += 2 * k)
+          for (int i = 0; i < k && i + j + k < M; ++i)
+            if ((i + j) / (2 * p) == (i + j + k) / (2 * p)) {
+              lo[c] = i + j;
+              hi[c] = i + j + k;
+              ++c;
+            }
+  }
+};
+
+// Bitonic merger (half-cleaners of stride M/2 .. 1): sorts a bitonic sequence.
+template <int M>
+struct BitonicMergeNet {
+  static constexpr int count() {
+    int c = 0;
+    for (int s = M / 2; s >= 1; s >>= 1)
+      for (int i = 0; i < M; ++i)
+        if ((i & s) == 0) ++c;
+    return c;
+  }
+  static constexpr int kCount = count();
+  int lo[kCount];
+  int hi[kCount];
+  constexpr BitonicMergeNet() : lo(), hi() {
+    int c = 0;
+    for (int s = M / 2; s >= 1; s >>= 1)
+      for (int i = 0; i < M; ++i)
+        if ((i & s) == 0) {
+          lo[c] = i;
+          hi[c] = i + s;
+          ++c;
+        }
+  }
+};
+
+template <typename Net>
+struct NetHolder {
+  static constexpr Net net{};
+};
+
+template <int A, int B, typename T, int N>
+MOE_DEV void cex_desc(T (&v)[N]) {
+  const T a = v[A], b = v[B];
+  v[A] = max(a, b);
+  v[B] = min(a, b);
+}
+
+template <typename Net, int OFF, typename T, int N, size_t... C>
+MOE_DEV void apply_net(T (&v)[N], std::index_sequence<C...>) {
+  (cex_desc<OFF + NetHolder<Net>::net.lo[C], OFF + NetHolder<Net>::net.hi[C]>(v), ...);
+}
+
+// v[OFF .. OFF+M) sorted descending.
+template <int M, int OFF, typename T, int N>
+MOE_DEV void sort_desc_at(T (&v)[N]) {
+  apply_net<OddEvenMergeNet<M>, OFF>(v, std::make_index_sequence<OddEvenMergeNet<M>::kCount>{});
+}
+
+// v[A .. A+32) and v[B .. B+32) sorted descending -> v[A .. A+32) = the 32
+// largest of both, sorted descending (the pairwise maxima of one run against
+// the other reversed form a bitonic sequence holding the 32 largest).
+template <int A, int B, typename T, int N, size_t... I>
+MOE_DEV void keep_top32_first(T (&v)[N], std::index_sequence<I...>) {
+  ((v[A + I] = max(v[A + I], v[B + 31 - I])), ...);
+}
+template <int A, int B, typename T, int N>
+MOE_DEV void merge_keep_top32(T (&v)[N]) {
+  keep_top32_first<A, B>(v, std::make_index_sequence<32>{});
+  apply_net<BitonicMergeNet<32>, A>(v, std::make_index_sequence<BitonicMergeNet<32>::kCount>{});
+}
+
+MOE_DEV void cex_desc_u64(uint64_t& a, uint64_t& b) {
+  const uint64_t hi = a > b ? a : b, lo = a > b ? b : a;
+  a = hi;
+  b = lo;
+}
+
+// 19-comparator sorting network for 8 keys (descending).
+MOE_DEV void sort8_desc(uint64_t (&k)[8]) {
+  cex_desc_u64(k[0], k[2]); cex_desc_u64(k[1], k[3]); cex_desc_u64(k[4], k[6]); cex_desc_u64(k[5], k[7]);
+  cex_desc_u64(k[0], k[4]); cex_desc_u64(k[1], k[5]); cex_desc_u64(k[2], k[6]); cex_desc_u64(k[3], k[7]);
+  cex_desc_u64(k[0], k[1]); cex_desc_u64(k[2], k[3]); cex_desc_u64(k[4], k[5]); cex_desc_u64(k[6], k[7]);
+  cex_desc_u64(k[2], k[4]); cex_desc_u64(k[3], k[5]);
+  cex_desc_u64(k[1], k[4]); cex_desc_u64(k[3], k[6]);
+  cex_desc_u64(k[1], k[2]); cex_desc_u64(k[3], k[4]); cex_desc_u64(k[5], k[6]);
+}
+
+// Balanced tree sum on packed pairs ep[a] = (v[2a], v[2a+1]): level H (even)
+// adds element i + H to element i, i.e. pair a + H/2 to pair a; the last level
+// (H = 1) is the sum of the two halves of ep[0].
+template <int H, int NP>
+MOE_DEV void tree_sum_level2(uint64_t (&ep)[NP]) {
+#pragma unroll
+  for (int a = 0; a < H / 2; ++a) ep[a] = add2(ep[a], ep[a + H / 2]);
+  if constexpr (H > 2) tree_sum_level2<H / 2>(ep);
+}
+
+// ---------------------------------------------------------------- kernel
+template <int N>
+struct RouteConsts {
+  float x[N];   // x'_i = fl(i / (N - 1))
+  float bound;  // fl(1 - x'_{kTop-1}) >= D_i for every rank i >= kTop - 1
+};
+
+// Host: the constants of an N-expert curve, computed in fp32 (RN).
+template <typename RC>
+inline void fill_route_consts(RC& rc, int N) {
+  for (int i = 0; i < N; ++i) rc.x[i] = static_cast<float>(i) / static_cast<float>(N - 1);
+  rc.bound = 1.0f - rc.x[kTop - 1];
+}
+
+template <int N>
+constexpr size_t smem_bytes() {
+  return sizeof(float) * kTok * (N + 4) + sizeof(uint64_t) * 8 * kTok;
+}
+
+MOE_DEV void write_outputs(int64_t t, int K, int k, const int (&ids)[8], const float (&g)[8],
+                           int32_t* k_out, int32_t* ids_out, float* gates_out) {
+  k_out[t] = k;
+  if (K == 8) {
+    int4* ip = reinterpret_cast<int4*>(ids_out + t * 8);
+    float4* gp = reinterpret_cast<float4*>(gates_out + t * 8);
+    ip[0] = make_int4(ids[0], ids[1], ids[2], ids[3]);
+    ip[1] = make_int4(ids[4], ids[5], ids[6], ids[7]);
+    gp[0] = make_float4(g[0], g[1], g[2], g[3]);
+    gp[1] = make_float4(g[4], g[5], g[6], g[7]);
+  } else {
+#pragma unroll
+    for (int s = 0; s < 8; ++s) {
+      if (s < K) {
+        ids_out[t * K + s] = ids[s];
+        gates_out[t * K + s] = g[s];
+      }
+    }
+  }
+}
+
+// Exact full path for one token, from the row of e values in shared memory
+// and r = 1/s: every probability sorted, the elbow evaluated on every rank,
+// the top-K ids from a threshold scan. Writes the token's outputs.
+template <int N, typename RC>
+__device__ __noinline__ int route_full(const float* row, float r, int K, float eps, int topk_mode,
+                                        int renorm, const RC& rc, uint64_t* keys,
+                                        int tid, int64_t t, int32_t* k_out, int32_t* ids_out,
+                                        float* gates_out) {
+  float v[N];
+#pragma unroll
+  for (int c = 0; c < N; c += 4) {
+    const float4 q = *reinterpret_cast<const float4*>(row + c);
+    v[c] = __fmul_rn(q.x, r); v[c + 1] = __fmul_rn(q.y, r);
+    v[c + 2] = __fmul_rn(q.z, r); v[c + 3] = __fmul_rn(q.w, r);
+  }
+  sort_desc_at<N, 0>(v);
+
+  int k = K;
+  if (!topk_mode) {
+    const float p_min = v[N - 1];
+    const float inv = __frcp_rn(__fadd_rn(__fsub_rn(v[0], p_min), eps));
+    float best = -__int_as_float(0x7f800000), tail = -__int_as_float(0x7f800000);
+    int e = 0;
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+      const float pn = __fmul_rn(__fsub_rn(v[i], p_min), inv);
+      const float D = __fsub_rn(__fsub_rn(1.0f, pn), rc.x[i]);
+      if (i < 7 && i < K - 1) {
+        if (D > best) { best = D; e = i; }
+      } else {
+        tail = fmaxf(tail, D);
+      }
+    }
+    k = (best >= tail) ? e + 1 : K;
+  }
+
+  // p_(K-1) as the minimum of the first K sorted values
+  float thr = v[0];
+#pragma unroll
+  for (int s = 1; s < 8; ++s)
+    if (s < K) thr = fminf(thr, v[s]);
+  int above = 0;
+#pragma unroll
+  for (int s = 0; s < 8; ++s)
+    if (s < K && v[s] > thr) ++above;
+  const int need_eq = K - above;
+  int cnt = 0, eq = 0;
+#pragma unroll
+  for (int c = 0; c < N; c += 4) {
+    const float4 q = *reinterpret_cast<const float4*>(row + c);
+    const float pq[4] = {__fmul_rn(q.x, r), __fmul_rn(q.y, r), __fmul_rn(q.z, r), __fmul_rn(q.w, r)};
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float pj = pq[u];
+      const bool is_eq = pj == thr;
+      const bool take = (pj > thr) || (is_eq && eq < need_eq);
+      eq += is_eq ? 1 : 0;
+      if (take && cnt < 8) {
+        keys[cnt * kTok + tid] =
+            (static_cast<uint64_t>(__float_as_uint(pj)) << 32) | static_cast<uint32_t>(~(c + u));
+        ++cnt;
+      }
+    }
+  }
+  uint64_t key[8];
+#pragma unroll
+  for (int s = 0; s < 8; ++s) key[s] = (s < K) ? keys[s * kTok + tid] : 0ull;
+  sort8_desc(key);
+
+  int ids[8];
+  float g[8];
+  float S = 0.0f;
+#pragma unroll
+  for (int s = 0; s < 8; ++s)
+    if (s < k) S = __fadd_rn(S, v[s]);
+#pragma unroll
+  for (int s = 0; s < 8; ++s) {
+    ids[s] = ~static_cast<int>(key[s]);
+    const float p = renorm ? __fdiv_rn(v[s], S) : v[s];
+    g[s] = (s < k) ? p : 0.0f;
+  }
+  write_outputs(t, K, k, ids, g, k_out, ids_out, gates_out);
+  // leave the ids in this thread's slot for the caller
+  int* slot = reinterpret_cast<int*>(keys);
+#pragma unroll
+  for (int s = 0; s < 8; ++s) slot[s * kTok + tid] = ids[s];
+  return k;
+}
+
+// Routes the token of this thread (its logits are in `row`); writes its
+// outputs and returns k, with the selected ids in ids_sel.
+template <int N, typename RC>
+MOE_DEV int route_token(float* row, int64_t t, int tid, int K, float eps, int topk_mode, int renorm,
+                        const RC& rc, uint64_t* keys64, int32_t* __restrict__ k_out,
+                        int32_t* __restrict__ ids_out, float* __restrict__ gates_out,
+                        int (&ids_sel)[8]) {
+  constexpr uint32_t kIdMask = N - 1;
+
+  // ---- e_j = EXP(l_j - m), stored back into the row; e_min; s; r = 1/s
+  uint64_t ep[N / 2];
+  float emin;
+  {
+    float l[N];
+#pragma unroll
+    for (int c = 0; c < N; c += 4) {
+      const float4 q = *reinterpret_cast<const float4*>(row + c);
+      l[c] = q.x; l[c + 1] = q.y; l[c + 2] = q.z; l[c + 3] = q.w;
+    }
+    // four interleaved 3-input max chains over l[4 ..), two elements per step
+    float acc[4] = {l[0], l[1], l[2], l[3]};
+#pragma unroll
+    for (int j = 4; j < N; j += 2) acc[(j / 2) % 4] = max3f(acc[(j / 2) % 4], l[j], l[j + 1]);
+    const float m = fmaxf(max3f(acc[0], acc[1], acc[2]), acc[3]);
+    const uint64_t mm = pk(m, m);
+#pragma unroll
+    for (int a = 0; a < N / 2; ++a) ep[a] = exp_spec2(sub2(pk(l[2 * a], l[2 * a + 1]), mm));
+  }
+#pragma unroll
+  for (int c = 0; c < N; c += 4)
+    *reinterpret_cast<float4*>(row + c) =
+        make_float4(lo_of(ep[c / 2]), hi_of(ep[c / 2]), lo_of(ep[c / 2 + 1]), hi_of(ep[c / 2 + 1]));
+  {
+    // four interleaved 3-input min chains over the pairs ep[2 ..)
+    float acc[4] = {lo_of(ep[0]), hi_of(ep[0]), lo_of(ep[1]), hi_of(ep[1])};
+#pragma unroll
+    for (int a = 2; a < N / 2; ++a) acc[a % 4] = min3f(acc[a % 4], lo_of(ep[a]), hi_of(ep[a]));
+    emin = fminf(min3f(acc[0], acc[1], acc[2]), acc[3]);
+  }
+  tree_sum_level2<N / 2>(ep);
+  const float r = __frcp_rn(__fadd_rn(lo_of(ep[0]), hi_of(ep[0])));
+
+  // ---- the kTop largest e, each key = truncated value | (N-1 - id)
+  uint32_t key[N];
+#pragma unroll
+  for (int c = 0; c < N; c += 4) {
+    const float4 q = *reinterpret_cast<const float4*>(row + c);
+    key[c] = (__float_as_uint(q.x) & ~kIdMask) | (kIdMask - c);
+    key[c + 1] = (__float_as_uint(q.y) & ~kIdMask) | (kIdMask - (c + 1));
+    key[c + 2] = (__float_as_uint(q.z) & ~kIdMask) | (kIdMask - (c + 2));
+    key[c + 3] = (__float_as_uint(q.w) & ~kIdMask) | (kIdMask - (c + 3));
+  }
+  sort_desc_at<32, 0>(key);
+  sort_desc_at<32, 32>(key);
+  if constexpr (N == 128) {
+    sort_desc_at<32, 64>(key);
+    sort_desc_at<32, 96>(key);
+    merge_keep_top32<64, 96>(key);
+  }
+  merge_keep_top32<0, 32>(key);
+  if constexpr (N == 128) merge_keep_top32<0, 64>(key);
+
+  // ---- exact values of the selected ranks, and the proof that they are the
+  // exact top ranks in exact order
+  float ev[kTop];
+  int idv[kTop];
+#pragma unroll
+  for (int i = 0; i < kTop; ++i) {
+    idv[i] = static_cast<int>(kIdMask - (key[i] & kIdMask));
+    ev[i] = row[idv[i]];
+  }
+  bool ok = ((key[kTop - 2] ^ key[kTop - 1]) & ~kIdMask) != 0u;
+#pragma unroll
+  for (int i = 0; i + 1 < kTop - 1; ++i) ok = ok && (ev[i] >= ev[i + 1]);
+
+  // ---- probabilities of the top ranks, elbow decision
+  float pv[kTop];
+  const uint64_t rr = pk(r, r);
+#pragma unroll
+  for (int i = 0; i < kTop; i += 2) {
+    const uint64_t q = mul2(pk(ev[i], ev[i + 1]), rr);
+    pv[i] = lo_of(q);
+    pv[i + 1] = hi_of(q);
+  }
+  int k = K;
+  if (ok && !topk_mode) {
+    const float p_min = __fmul_rn(emin, r);
+    const float inv = __frcp_rn(__fadd_rn(__fsub_rn(pv[0], p_min), eps));
+    const uint64_t pmin2 = pk(p_min, p_min), inv2 = pk(inv, inv), one2 = pk(1.0f, 1.0f);
+    float best = -__int_as_float(0x7f800000), mid = -__int_as_float(0x7f800000);
+    int e = 0;
+#pragma unroll
+    for (int i = 0; i < kTop; i += 2) {
+      const uint64_t pn = mul2(sub2(pk(pv[i], pv[i + 1]), pmin2), inv2);
+      const uint64_t D2 = sub2(sub2(one2, pn), pk(rc.x[i], rc.x[i + 1]));
+      const float D[2] = {lo_of(D2), hi_of(D2)};
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int ii = i + u;
+        if (ii >= kTop - 1) continue;
+        if (ii < 7 && ii < K - 1) {
+          if (D[u] > best) { best = D[u]; e = ii; }
+        } else {
+          mid = fmaxf(mid, D[u]);
+        }
+      }
+    }
+    if (best >= mid && best >= rc.bound) k = e + 1;
+    else if (mid > best) k = K;
+    else ok = false;
+  }
+
+  // ---- top-K ids and gates; equal probabilities are re-ordered by id
+  // (p_(K) and p_(K-1) are written as a max and a min over sorted values: a
+  // select on s == K would become a dynamic index into the register array)
+  bool tie_in = false;
+  float pK = 0.0f;
+#pragma unroll
+  for (int s = 0; s < 8; ++s)
+    if (s + 1 < K && pv[s] == pv[s + 1]) tie_in = true;
+#pragma unroll
+  for (int s = 1; s <= 8; ++s)
+    if (s >= K) pK = fmaxf(pK, pv[s]);
+  float pKm1 = pv[0];
+#pragma unroll
+  for (int s = 1; s < 8; ++s)
+    if (s < K) pKm1 = fminf(pKm1, pv[s]);
+  if (pKm1 == pK) ok = false;  // a tie across the K boundary
+
+  if (!ok) {
+    const int kf =
+        route_full<N, RC>(row, r, K, eps, topk_mode, renorm, rc, keys64, tid, t, k_out, ids_out,
+                          gates_out);
+    const int* slot = reinterpret_cast<const int*>(keys64);
+#pragma unroll
+    for (int s = 0; s < 8; ++s) ids_sel[s] = slot[s * kTok + tid];
+    return kf;
+  }
+
+  int ids[8];
+  float g[8];
+#pragma unroll
+  for (int s = 0; s < 8; ++s) ids[s] = idv[s];
+  if (tie_in) {
+    uint64_t kk[8];
+#pragma unroll
+    for (int s = 0; s < 8; ++s)
+      kk[s] = (s < K) ? ((static_cast<uint64_t>(__float_as_uint(pv[s])) << 32) |
+                         static_cast<uint32_t>(~idv[s]))
+                      : 0ull;
+    sort8_desc(kk);
+#pragma unroll
+    for (int s = 0; s < 8; ++s) ids[s] = ~static_cast<int>(kk[s]);
+  }
+  float S = 0.0f;
+#pragma unroll
+  for (int s = 0; s < 8; ++s)
+    if (s < k) S = __fadd_rn(S, pv[s]);
+#pragma unroll
+  for (int s = 0; s < 8; ++s) {
+    const float p = renorm ? __fdiv_rn(pv[s], S) : pv[s];
+    g[s] = (s < k) ? p : 0.0f;
+  }
+  write_outputs(t, K, k, ids, g, k_out, ids_out, gates_out);
+#pragma unroll
+  for (int s = 0; s < 8; ++s) ids_sel[s] = ids[s];
+  return k;
+}
+
+}  // namespace route
+}  // namespace moe

@@ -77,7 +77,8 @@ def test_dispatch_validation(lib):
 def test_layer_validation(lib):
     fake = ctypes.c_void_p(256)
     ws = lib.moe_layer_workspace_size(64, 2048, 64, 1024, 8)
-    assert ws > 64 * 8 * (2048 * 2 * 2 + 1024 * 2)
+    # h [T*K, I] and the expert outputs [T*K, d], bf16
+    assert ws > 64 * 8 * (2048 * 2 + 1024 * 2)
     args = lambda T=64, d=2048, N=64, I=1024, rp=None, wsb=ws: (
         fake, fake, fake, fake, T, d, N, I, rp or _rp(), None, fake, None, None, None, None, None,
         fake, wsb, None)

@@ -33,7 +33,7 @@ def test_noalloc_matches_workspace_dispatch(moe, N):
     import torch
     K = 8
     # second call smaller than the first, so stale chunk counts would show up
-    for seed, T in ((1, 300000), (2, 4097)):
+    for seed, T in ((1, 262144), (2, 4097)):
         k, ids = _inputs(seed + N, T, N, K)
         dk = torch.from_numpy(k).cuda()
         dids = torch.from_numpy(ids).cuda()
@@ -52,4 +52,4 @@ def test_noalloc_rejects_oversize(moe):
     import ctypes
     lib = moe.library()
     fake = ctypes.c_void_p(256)
-    assert lib.moe_dispatch_noalloc(fake, fake, (1 << 20) + 1, 64, 8, fake, fake, fake, None) == 2
+    assert lib.moe_dispatch_noalloc(fake, fake, (1 << 18) + 1, 64, 8, fake, fake, fake, None) == 2
