@@ -1,7 +1,8 @@
 """Benchmark of the elbow-routed MoE layer on GB300.
 
-One step = one MoE layer forward (router GEMM, elbow routing, dispatch,
-gather, grouped SwiGLU gate/up GEMM, grouped down GEMM, combine) over the
+One step = one MoE layer forward (router GEMM with the elbow routing in its
+epilogue, dispatch, grouped SwiGLU gate/up GEMM gathering its token rows,
+grouped down GEMM, combine) over the
 16,384-token OLMoE-shaped prefill batch (d = 2048, 64 experts, I = 1024,
 K = 8), inputs resident in HBM. `value` = tokens/s in elbow mode; the same
 kernels in fixed top-8 mode are reported beside it. Per-kernel CUDA-event
@@ -32,9 +33,9 @@ sys.path.insert(0, ROOT)
 METRIC = "MoE-layer tokens/s elbow vs fixed top-8; route GB/s & GEMM tensor-pipe % of peak"
 WORKLOAD = "layer_t16k"
 ROUTE_WORKLOAD = "route_t1m"
-# steps per launch sequence of moe_layer_forward (router GEMM, route, dispatch
-# count/scan/scatter, gather, gate/up GEMM, down GEMM, combine)
-KERNELS_PER_STEP = 9
+# kernels per moe_layer_forward: router GEMM with fused routing, dispatch
+# scan and scatter, gathered gate/up GEMM, down GEMM, combine
+KERNELS_PER_STEP = 6
 
 
 def parse():
@@ -279,11 +280,12 @@ def run_ours(args, rank, world, local, pg):
                  "elbow_speedup": ms_topk / ms_elbow},
         "routing": {"mean_k": sum_k / T, "k_hist": np.bincount(kk, minlength=K + 1)[1:].tolist(),
                     "expert_load_min": int(load.min()), "expert_load_max": int(load.max())},
-        "roofline": {"kernel": "grouped gate/up GEMM + SwiGLU (tcgen05)", "bound": "tensor",
+        "roofline": {"kernel": "grouped gate/up GEMM + SwiGLU, gathered rows (tcgen05)",
+                     "bound": "tensor",
                      "achieved": gu_tf, "peak": pk["bf16_sus"], "unit": "TFLOP/s",
-                     "frac": gu_tf / pk["bf16_sus"], "traffic": ncu_traffic("gemm_gate_up_layer_t16k"),
+                     "frac": gu_tf / pk["bf16_sus"], "traffic": ncu_traffic("gemm_gate_up_gathered_layer_t16k"),
                      "traffic_unit": "bytes per launch (ncu dram read + write)",
-                     "algorithmic_bytes": 2 * sum_k * d + 2 * N * 2 * I * d + 2 * sum_k * I,
+                     "algorithmic_bytes": 2 * T * d + 2 * N * 2 * I * d + 2 * sum_k * I,
                      "peak_source": f"{pk['source']} bf16 dense, sustained",
                      "frac_of_burst": gu_tf / pk["bf16"]},
         "kernels": kern,
@@ -300,32 +302,31 @@ def run_ours(args, rank, world, local, pg):
 
 def kernel_breakdown(moe, x, wr, wgu, wd, T, d, N, I, K, args, stream, dev):
     """Average duration of each kernel of the layer, CUDA events between the
-    step-level calls on one stream, over `steps` back-to-back steps."""
+    step-level calls (the same kernels moe_layer_forward launches, in its
+    order) on one stream, over back-to-back steps."""
     import torch
-    names = ["router_gemm", "route", "dispatch", "gather", "gate_up", "down", "combine"]
+    names = ["router_route", "dispatch", "gate_up", "down", "combine"]
     acc = {n: 0.0 for n in names}
     err = torch.zeros(1, dtype=torch.int32, device=dev)
     P = T * K
     steps = max(10, args.steps // 4)
     dws = torch.empty(moe.dispatch_workspace_size(T, N, K), dtype=torch.uint8, device=dev)
+    cc = moe.dispatch_chunk_counts(dws, T, N, K)
     for it in range(steps + 3):
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)]
         ev[0].record(stream)
-        lg = moe.router_logits(x, wr, err=err)
+        k, ids, gates, _, _ = moe.router_route(x, wr, K=K, with_logits=False, chunk_counts=cc,
+                                               err=err)
         ev[1].record(stream)
-        k, ids, gates = moe.elbow_route(lg, K=K)
+        off, perm, pp = moe.moe_dispatch_counted(k, ids, N, dws)
         ev[2].record(stream)
-        off, perm, pp, _ = moe.moe_dispatch(k, ids, N, ws=dws)
-        ev[3].record(stream)
-        xs = moe.gather_rows(x, perm, off, P)
-        ev[4].record(stream)
         toff = moe.dispatch_tile_offsets(dws, T, N, K)
-        h = moe.expert_gate_up(xs, wgu, off, toff, err=err)
-        ev[5].record(stream)
+        h = moe.expert_gate_up_gathered(x, perm, wgu, off, toff, P, err=err)
+        ev[3].record(stream)
         o = moe.expert_down(h, wd, off, toff, err=err)
-        ev[6].record(stream)
+        ev[4].record(stream)
         moe.combine(o, k, pp, gates)
-        ev[7].record(stream)
+        ev[5].record(stream)
         torch.cuda.synchronize()
         if it >= 3:
             for i, n in enumerate(names):

@@ -216,6 +216,17 @@ moe_status moe_expert_down(const uint16_t* h, const uint16_t* w_down, const int3
  * moe_dispatch on that workspace wrote. */
 const int32_t* moe_dispatch_tile_offsets(const void* ws, int64_t T, int N, int K);
 
+/* Device pointer, inside a moe_dispatch workspace, of the [N][ceil(T/128)]
+ * int32 per-chunk expert counts: pass it as moe_router_route's chunk_counts,
+ * then call moe_dispatch_counted, which skips its own counting pass. */
+int32_t* moe_dispatch_chunk_counts(void* ws, int64_t T, int N, int K);
+
+/* moe_dispatch whose per-chunk expert counts are already in the workspace
+ * (written there by moe_router_route); otherwise identical. */
+moe_status moe_dispatch_counted(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
+                                int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
+                                size_t ws_bytes, void* stream);
+
 /* Gather rows: xs[r] = x[perm[r]] for r < offsets[N] (x [T, d] bf16,
  * xs [P, d] bf16, P >= offsets[N]). */
 moe_status moe_gather_rows(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int64_t T,

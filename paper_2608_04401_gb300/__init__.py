@@ -68,6 +68,8 @@ def library():
             "moe_dispatch": ([P, P, i64, i32, i32, P, P, P, P, sz, P], i32),
             "moe_dispatch_tile_offsets": ([P, i64, i32, i32], P),
             "moe_dispatch_noalloc": ([P, P, i64, i32, i32, P, P, P, P], i32),
+            "moe_dispatch_chunk_counts": ([P, i64, i32, i32], P),
+            "moe_dispatch_counted": ([P, P, i64, i32, i32, P, P, P, P, sz, P], i32),
             "moe_layer_workspace_size": ([i64, i32, i32, i32, i32], sz),
             "moe_layer_forward": ([P, P, P, P, i64, i32, i32, i32, RP, P, P, P, P, P, P, P, P, sz, P],
                                   i32),
@@ -162,6 +164,29 @@ def moe_dispatch(k, ids, N: int, ws=None, stream=None):
     return offsets, perm, pair_pos, ws
 
 
+def dispatch_chunk_counts(ws, T: int, N: int, K: int):
+    """View of the [N, ceil(T/128)] per-chunk expert counts inside a dispatch workspace."""
+    torch = _torch()
+    ptr = library().moe_dispatch_chunk_counts(_p(ws), T, N, K)
+    off = ptr - ws.data_ptr()
+    nblk = (T + 127) // 128
+    return ws[off: off + 4 * N * nblk].view(torch.int32).view(N, nblk)
+
+
+def moe_dispatch_counted(k, ids, N: int, ws, stream=None):
+    """moe_dispatch using the per-chunk counts already in ws (from router_route)."""
+    torch = _torch()
+    lib = library()
+    T, K = ids.shape
+    dev = ids.device
+    offsets = torch.empty(N + 1, dtype=torch.int32, device=dev)
+    perm = torch.empty(max(1, T * K), dtype=torch.int32, device=dev)
+    pair_pos = torch.empty(T, K, dtype=torch.int32, device=dev)
+    _check(lib.moe_dispatch_counted(_p(k), _p(ids), T, N, K, _p(offsets), _p(perm), _p(pair_pos),
+                                    _p(ws), ws.numel(), _stream(stream)), "moe_dispatch_counted")
+    return offsets, perm, pair_pos
+
+
 def moe_dispatch_noalloc(k, ids, N: int, offsets=None, perm=None, pair_pos=None, stream=None):
     """moe_dispatch without a workspace (the library's fixed scratch array is used).
     Output buffers may be passed in; returns (offsets, perm, pair_pos)."""
@@ -250,7 +275,7 @@ def router_logits(x, w_router, err=None, stream=None):
 
 def router_route(x, w_router, K: int = 8, eps: float = 1e-8, mode: int = MODE_ELBOW,
                  renorm: int = 0, with_logits: bool = True, with_counts: bool = True, err=None,
-                 stream=None):
+                 chunk_counts=None, stream=None):
     """Router GEMM with the elbow routing in its epilogue. Returns
     (k, ids, gates, logits or None, chunk_counts [N, ceil(T/128)] or None)."""
     torch = _torch()
@@ -263,8 +288,9 @@ def router_route(x, w_router, K: int = 8, eps: float = 1e-8, mode: int = MODE_EL
     ids = torch.empty(T, K, dtype=torch.int32, device=dev)
     gates = torch.empty(T, K, dtype=torch.float32, device=dev)
     lg = torch.empty(T, N, dtype=torch.float32, device=dev) if with_logits else None
-    cc = (torch.zeros(N, (T + 127) // 128, dtype=torch.int32, device=dev)
-          if with_counts else None)
+    cc = chunk_counts
+    if cc is None and with_counts:
+        cc = torch.zeros(N, (T + 127) // 128, dtype=torch.int32, device=dev)
     _check(library().moe_router_route(_p(x), _p(w_router), T, d, N, _params(K, eps, mode, renorm),
                                       _p(lg), _p(k), _p(ids), _p(gates), _p(cc), _p(err),
                                       _stream(stream)), "moe_router_route")

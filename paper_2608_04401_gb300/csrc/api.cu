@@ -154,6 +154,27 @@ const int32_t* moe_dispatch_tile_offsets(const void* ws, int64_t T, int N, int K
   return moe::dispatch_tile_off(const_cast<void*>(ws), T, N);
 }
 
+int32_t* moe_dispatch_chunk_counts(void* ws, int64_t T, int N, int K) {
+  (void)T;
+  (void)K;
+  if (!ws || !supported_n(N)) return nullptr;
+  return moe::dispatch_counts(ws);
+}
+
+moe_status moe_dispatch_counted(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
+                                int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
+                                size_t ws_bytes, void* stream) {
+  if (T < 0 || T > kMaxTokens) return MOE_ERR_INVALID_ARG;
+  if (!supported_n(N) || K < 1 || K > 8 || K > N) return MOE_ERR_UNSUPPORTED;
+  if (!offsets || !ws) return MOE_ERR_INVALID_ARG;
+  if (T > 0 && (!k || !ids || !perm || !pair_pos)) return MOE_ERR_INVALID_ARG;
+  if (ws_bytes < moe::dispatch_ws_bytes(T, N)) return MOE_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u)) return MOE_ERR_INVALID_ARG;
+  if (T > 0 && !aligned16(ids)) return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_dispatch(k, ids, T, N, K, offsets, perm, pair_pos, ws, nullptr,
+                                          true, static_cast<cudaStream_t>(stream)));
+}
+
 moe_status moe_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
                         int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
                         size_t ws_bytes, void* stream) {

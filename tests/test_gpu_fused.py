@@ -70,3 +70,21 @@ def test_gate_up_gathered_matches_dense(moe, N, T):
     assert int(err.item()) == 0
     n = int(off[-1].item())
     assert torch.equal(h_dense[:n].view(torch.int16), h_gath[:n].view(torch.int16))
+
+
+@pytest.mark.parametrize("T,N", [(64, 64), (5000, 64), (3000, 128)])
+def test_dispatch_counted_matches_dispatch(moe, T, N):
+    """Router counts written straight into the dispatch workspace give the
+    same dispatch as counting again."""
+    import torch
+    inp = synth.layer_inputs(T=T, d=512, N=N, I=128, seed=T * 3 + N, with_experts=False)
+    x, wr = to_dev_bf16(inp["x"]), to_dev_bf16(inp["w_router"])
+    ws = torch.empty(moe.dispatch_workspace_size(T, N, 8), dtype=torch.uint8, device="cuda")
+    cc = moe.dispatch_chunk_counts(ws, T, N, 8)
+    k, ids, gates, _, _ = moe.router_route(x, wr, with_logits=False, chunk_counts=cc)
+    off_a, perm_a, pp_a = moe.moe_dispatch_counted(k, ids, N, ws)
+    off_b, perm_b, pp_b, _ = moe.moe_dispatch(k, ids, N)
+    torch.cuda.synchronize()
+    assert torch.equal(off_a, off_b) and torch.equal(pp_a, pp_b)
+    n = int(off_b[-1].item())
+    assert torch.equal(perm_a[:n], perm_b[:n])
