@@ -229,52 +229,75 @@ __global__ void __launch_bounds__(256) gather_kernel(const uint4* __restrict__ x
 }
 
 // y_t = sum_{s<k_t} g_{t,s} * o[pair_pos[t,s]] (+ residual_t); fp32 in s order.
-__global__ void __launch_bounds__(256) combine_kernel(const uint4* __restrict__ o,
-                                                      const int32_t* __restrict__ k,
-                                                      const int32_t* __restrict__ pair_pos,
-                                                      const float* __restrict__ gates,
-                                                      const uint4* residual, int64_t T, int d8,
-                                                      int K, uint4* y) {
-  for (int64_t t = blockIdx.x; t < T; t += gridDim.x) {
+// One warp per token. The token's k positions and gates are read once (lane s
+// holds pair s) and broadcast by shuffles; the row is processed in slabs of
+// 256 sixteen-byte chunks, lane l holding chunks l + 32c (c < 8) of the slab,
+// so each of the k rows is fetched with eight independent coalesced loads
+// per lane before it is accumulated.
+constexpr int kCombineWarps = 4;
+
+__global__ void __launch_bounds__(32 * kCombineWarps) combine_kernel(
+    const uint4* __restrict__ o, const int32_t* __restrict__ k, const int32_t* __restrict__ pair_pos,
+    const float* __restrict__ gates, const uint4* residual, int64_t T, int d8, int K, uint4* y) {
+  const int lane = threadIdx.x & 31;
+  const int64_t nwarps = static_cast<int64_t>(gridDim.x) * kCombineWarps;
+  const int64_t cap = T * K;
+  for (int64_t t = static_cast<int64_t>(blockIdx.x) * kCombineWarps + threadIdx.x / 32; t < T;
+       t += nwarps) {
     const int kt = min(k[t], K);
-    int pos[8];
-    float g[8];
+    const int my_pos = lane < kt ? static_cast<int>(min_of<int64_t>(max(pair_pos[t * K + lane], 0), cap - 1)) : 0;
+    const float my_g = lane < kt ? gates[t * K + lane] : 0.0f;
+    for (int slab = 0; slab < d8; slab += 256) {
+      float acc[8][8];
 #pragma unroll
-    for (int s = 0; s < 8; ++s) {
-      pos[s] = (s < kt) ? min(max(pair_pos[t * K + s], 0), static_cast<int>(T * K - 1)) : 0;
-      g[s] = (s < kt) ? gates[t * K + s] : 0.0f;
-    }
-    for (int c = threadIdx.x; c < d8; c += blockDim.x) {
-      float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+      for (int c = 0; c < 8; ++c)
+#pragma unroll
+        for (int u = 0; u < 8; ++u) acc[c][u] = 0.0f;
 #pragma unroll
       for (int s = 0; s < 8; ++s) {
+        const int p = __shfl_sync(0xffffffffu, my_pos, s);
+        const float g = __shfl_sync(0xffffffffu, my_g, s);
         if (s < kt) {
-          const uint4 v = o[static_cast<int64_t>(pos[s]) * d8 + c];
+          const uint4* row = o + static_cast<int64_t>(p) * d8 + slab;
+          uint4 v[8];
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            const int ci = slab + lane + 32 * c;
+            v[c] = ci < d8 ? row[lane + 32 * c] : make_uint4(0, 0, 0, 0);
+          }
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v[c]);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+              const float2 f = __bfloat1622float2(h[u]);
+              acc[c][2 * u] = fmaf(g, f.x, acc[c][2 * u]);
+              acc[c][2 * u + 1] = fmaf(g, f.y, acc[c][2 * u + 1]);
+            }
+          }
+        }
+      }
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        const int ci = slab + lane + 32 * c;
+        if (ci >= d8) continue;
+        if (residual) {
+          const uint4 v = residual[t * d8 + ci];
           const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
             const float2 f = __bfloat1622float2(h[u]);
-            acc[2 * u] = fmaf(g[s], f.x, acc[2 * u]);
-            acc[2 * u + 1] = fmaf(g[s], f.y, acc[2 * u + 1]);
+            acc[c][2 * u] += f.x;
+            acc[c][2 * u + 1] += f.y;
           }
         }
+        uint4 out;
+        out.x = pack_bf16x2(acc[c][0], acc[c][1]);
+        out.y = pack_bf16x2(acc[c][2], acc[c][3]);
+        out.z = pack_bf16x2(acc[c][4], acc[c][5]);
+        out.w = pack_bf16x2(acc[c][6], acc[c][7]);
+        y[t * d8 + ci] = out;
       }
-      if (residual) {
-        const uint4 v = residual[t * d8 + c];
-        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const float2 f = __bfloat1622float2(h[u]);
-          acc[2 * u] += f.x;
-          acc[2 * u + 1] += f.y;
-        }
-      }
-      uint4 out;
-      out.x = pack_bf16x2(acc[0], acc[1]);
-      out.y = pack_bf16x2(acc[2], acc[3]);
-      out.z = pack_bf16x2(acc[4], acc[5]);
-      out.w = pack_bf16x2(acc[6], acc[7]);
-      y[t * d8 + c] = out;
     }
   }
 }
@@ -356,10 +379,10 @@ cudaError_t launch_combine(const uint16_t* o, const int32_t* k, const int32_t* p
                            const float* gates, const uint16_t* residual, int64_t T, int d, int K,
                            uint16_t* y, int num_sms, cudaStream_t stream) {
   if (T == 0) return cudaSuccess;
-  int64_t blocks = T;
-  const int64_t cap = static_cast<int64_t>(num_sms) * 64;
+  int64_t blocks = (T + disp::kCombineWarps - 1) / disp::kCombineWarps;
+  const int64_t cap = static_cast<int64_t>(num_sms) * 16;
   if (blocks > cap) blocks = cap;
-  disp::combine_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
+  disp::combine_kernel<<<static_cast<unsigned>(blocks), 32 * disp::kCombineWarps, 0, stream>>>(
       reinterpret_cast<const uint4*>(o), k, pair_pos, gates,
       reinterpret_cast<const uint4*>(residual), T, d / 8, K, reinterpret_cast<uint4*>(y));
   return cudaGetLastError();

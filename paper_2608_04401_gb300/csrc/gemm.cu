@@ -73,7 +73,9 @@ struct Cfg {
   static constexpr int kRouteTileBytes = 128 * (BN + 4) * 4;
   static constexpr int kRouteBytes =
       MODE == kRouterFused ? kRouteTileBytes + 8 * 128 * 8 + BN * 4 : 0;
-  static constexpr int kStages = (208 * 1024 - kRouteBytes) / kStageBytes;
+  // kDown: per epilogue warp two 32 x 32 bf16 staging tiles for TMA stores
+  static constexpr int kEpiBytes = MODE == kDown ? 4 * 2 * 32 * 64 : 0;
+  static constexpr int kStages = (208 * 1024 - kRouteBytes - kEpiBytes) / kStageBytes;
   static constexpr int kTmemCols = (2 * BN <= 64) ? 64 : (2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512));
   static constexpr int kBarOff = kStages * kStageBytes;
   // barriers: full[S], empty[S], tfull[2], tempty[2], drain
@@ -82,7 +84,8 @@ struct Cfg {
   static constexpr int kTableOff = kMiscOff + 16;
   static constexpr int kMaxGroups = 128;
   static constexpr int kRouteOff = (kTableOff + 2 * (kMaxGroups + 1) * 4 + 15) & ~15;
-  static constexpr int kSmemBytes = kRouteOff + kRouteBytes + 1024;  // + align slack
+  static constexpr int kEpiOff = (kRouteOff + kRouteBytes + 127) & ~127;
+  static constexpr int kSmemBytes = kEpiOff + kEpiBytes + 1024;  // + align slack
   static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 };
 
@@ -156,6 +159,23 @@ MOE_DEV void cp_async_wait_group() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
+// TMA store of a shared-memory box to global, tracked by bulk groups.
+MOE_DEV void tma_store_2d(const CUtensorMap* map, uint32_t src, int c0, int c1) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(src), "r"(c0), "r"(c1)
+               : "memory");
+}
+MOE_DEV void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+template <int N>
+MOE_DEV void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+template <int N>
+MOE_DEV void bulk_wait() {
+  asm volatile("cp.async.bulk.wait_group %0;" ::"n"(N) : "memory");
+}
+
 // Named barrier among the four epilogue warps.
 MOE_DEV void epilogue_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
@@ -176,6 +196,7 @@ MOE_DEV bool epilogue_all(bool v) {
 template <int MODE, int BN>
 __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                const __grid_constant__ CUtensorMap tmC,
                 const __grid_constant__ Args args) {
   using C = Cfg<MODE, BN>;
   using R = Roles<MODE>;
@@ -381,6 +402,7 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
   } else {
     // ------------------------------------------------------------ epilogue
     const int q = warp & 3;  // the four epilogue warps cover the four TMEM lane quarters
+    int epi_buf = 0;         // kDown: which of this warp's two staging tiles is next
     const int r = q * 32 + lane;
     int local = 0;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++local) {
@@ -484,24 +506,46 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
           }
         }
       } else {
+        // Output rows are written 32 x 32 at a time: when all 32 rows of this
+        // warp belong to the tile's expert, through a staging tile in shared
+        // memory and a TMA store (coalesced, asynchronous); otherwise (the
+        // ragged last tile of an expert) row by row from registers.
         __nv_bfloat16* out = static_cast<__nv_bfloat16*>(args.out) + grow * args.ldo + t.nb * BN;
+        const bool full_warp = __all_sync(0xffffffffu, valid);
 #pragma unroll 1
         for (int c = 0; c < BN; c += 32) {
           uint32_t v[32];
           tmem_ld_32x32b_x32(taddr + c, v);
           tmem_ld_wait();
-          if (valid) {
+          uint4 w4[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            uint32_t w[4];
+#pragma unroll
+            for (int z = 0; z < 4; ++z) {
+              const int i0 = 8 * u + 2 * z;
+              w[z] = pack_bf16x2(__uint_as_float(v[i0]), __uint_as_float(v[i0 + 1]));
+            }
+            w4[u] = make_uint4(w[0], w[1], w[2], w[3]);
+          }
+          if (MODE == kDown && full_warp) {
+            uint8_t* sb = smem + C::kEpiOff + (q * 2 + epi_buf) * 2048;
+            // the store issued from this buffer two chunks ago has read it
+            if (lane == 0) bulk_wait_read<1>();
+            __syncwarp();
+#pragma unroll
+            for (int u = 0; u < 4; ++u) reinterpret_cast<uint4*>(sb + lane * 64)[u] = w4[u];
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+              tma_store_2d(&tmC, smem_u32(sb), t.nb * BN + c, t.row0 + q * 32);
+              bulk_commit();
+            }
+            epi_buf ^= 1;
+          } else if (valid) {
             uint4* o4 = reinterpret_cast<uint4*>(out + c);
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              uint32_t w[4];
-#pragma unroll
-              for (int z = 0; z < 4; ++z) {
-                const int i0 = 8 * u + 2 * z;
-                w[z] = pack_bf16x2(__uint_as_float(v[i0]), __uint_as_float(v[i0 + 1]));
-              }
-              o4[u] = make_uint4(w[0], w[1], w[2], w[3]);
-            }
+            for (int u = 0; u < 4; ++u) o4[u] = w4[u];
           }
         }
       }
@@ -509,6 +553,7 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty_bar(acc));
     }
+    if (MODE == kDown && lane == 0) bulk_wait<0>();  // every TMA store has completed
   }
 
   __syncthreads();
@@ -553,9 +598,23 @@ static bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t 
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 2-D bf16 tensor [outer, inner], box [box_outer, box_inner], no swizzle.
+static bool make_map_plain(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer,
+                           uint32_t box_inner, uint32_t box_outer) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+            CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int MODE, int BN>
-static cudaError_t launch_mode(const CUtensorMap& a, const CUtensorMap& b, const Args& args,
-                               int grid, cudaStream_t stream) {
+static cudaError_t launch_mode(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
+                               const Args& args, int grid, cudaStream_t stream) {
   using C = Cfg<MODE, BN>;
   static int attr_dev = -1;
   int dev = 0;
@@ -566,7 +625,7 @@ static cudaError_t launch_mode(const CUtensorMap& a, const CUtensorMap& b, const
     if (e != cudaSuccess) return e;
     attr_dev = dev;
   }
-  gemm_kernel<MODE, BN><<<grid, Roles<MODE>::kThreads, C::kSmemBytes, stream>>>(a, b, args);
+  gemm_kernel<MODE, BN><<<grid, Roles<MODE>::kThreads, C::kSmemBytes, stream>>>(a, b, c, args);
   return cudaGetLastError();
 }
 
@@ -589,8 +648,8 @@ cudaError_t launch_router_gemm(const uint16_t* x, const uint16_t* wr, int64_t T,
   a.err = err;
   const int64_t tiles = (T + BM - 1) / BM;
   const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
-  if (N == 64) return launch_mode<kRouter, 64>(ma, mb, a, grid, stream);
-  return launch_mode<kRouter, 128>(ma, mb, a, grid, stream);
+  if (N == 64) return launch_mode<kRouter, 64>(ma, mb, ma, a, grid, stream);
+  return launch_mode<kRouter, 128>(ma, mb, ma, a, grid, stream);
 }
 
 // Router GEMM with the elbow routing in its epilogue: k/ids/gates per token and
@@ -624,8 +683,8 @@ cudaError_t launch_router_route(const uint16_t* x, const uint16_t* wr, int64_t T
   const int64_t tiles = (T + BM - 1) / BM;
   a.nblk = static_cast<int>(tiles);
   const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
-  if (N == 64) return launch_mode<kRouterFused, 64>(ma, mb, a, grid, stream);
-  return launch_mode<kRouterFused, 128>(ma, mb, a, grid, stream);
+  if (N == 64) return launch_mode<kRouterFused, 64>(ma, mb, ma, a, grid, stream);
+  return launch_mode<kRouterFused, 128>(ma, mb, ma, a, grid, stream);
 }
 
 // h[P, I] = silu(x[perm] W_g^T) * (x[perm] W_u^T) per expert, rows gathered by TMA
@@ -654,7 +713,7 @@ cudaError_t launch_gateup_gather_gemm(const uint16_t* x, int64_t T, const int32_
   a.m_rows = T;  // gathered token rows are clamped to [0, T)
   a.a_src = x;
   a.lda = d;
-  return launch_mode<kGateUpGather, 256>(ma, mb, a, num_sms, stream);
+  return launch_mode<kGateUpGather, 256>(ma, mb, ma, a, num_sms, stream);
 }
 
 // h[P, I] = silu(xs W_g^T) * (xs W_u^T) per expert
@@ -678,7 +737,7 @@ cudaError_t launch_gateup_gemm(const uint16_t* xs, const uint16_t* wgu, const in
   a.out = h;
   a.ldo = I;
   a.err = err;
-  return launch_mode<kGateUp, 256>(ma, mb, a, num_sms, stream);
+  return launch_mode<kGateUp, 256>(ma, mb, ma, a, num_sms, stream);
 }
 
 // o[P, d] = h W_d[e]^T per expert
@@ -700,7 +759,9 @@ cudaError_t launch_down_gemm(const uint16_t* h, const uint16_t* wd, const int32_
   a.out = o;
   a.ldo = d;
   a.err = err;
-  return launch_mode<kDown, 256>(ma, mb, a, num_sms, stream);
+  CUtensorMap mc;  // o [P, d], boxes of 32 x 32, no swizzle (TMA stores)
+  if (!make_map_plain(&mc, o, d, P, 32, 32)) return cudaErrorInvalidValue;
+  return launch_mode<kDown, 256>(ma, mb, mc, a, num_sms, stream);
 }
 
 }  // namespace moe
