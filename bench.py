@@ -363,12 +363,25 @@ def route_stress(moe, args, stream, dev, pk):
     def disp():
         lib.moe_dispatch(P(k), P(ids), T, N, K, P(off), P(perm), P(pp), P(dws), dws.numel(), s)
 
+    cc = moe.dispatch_chunk_counts(dws, T, N, K)
+
+    def route_counted():
+        lib.elbow_route_with_counts(P(lg), T, N, rp, P(k), P(ids), P(gates), P(cc), s)
+
+    def disp_counted():
+        lib.moe_dispatch_counted(P(k), P(ids), T, N, K, P(off), P(perm), P(pp), P(dws),
+                                 dws.numel(), s)
+
     for _ in range(3):
         route()
         disp()
+        route_counted()
+        disp_counted()
     n = max(20, args.steps // 4)
     ms_r = time_steps(route, n, stream, None)
     ms_d = time_steps(disp, n, stream, None)
+    ms_rc = time_steps(route_counted, n, stream, None)
+    ms_dc = time_steps(disp_counted, n, stream, None)
     sum_k = int(k.sum().item())
     # algorithmic bytes: route reads N fp32 logits, writes k + K ids + K gates
     br = T * (4 * N + 4 + 8 * K)
@@ -380,6 +393,10 @@ def route_stress(moe, args, stream, dev, pk):
             "route": {"ms": ms_r, "GBps": gr, "frac": gr / pk["hbm"], "bytes": br,
                       "tokens_per_s": T / (ms_r * 1e-3)},
             "dispatch": {"ms": ms_d, "GBps": gd, "frac": gd / pk["hbm"], "bytes": bd},
+            "pipeline": {"route_with_counts_ms": ms_rc, "dispatch_counted_ms": ms_dc,
+                         "GBps": (br + bd) / ((ms_rc + ms_dc) * 1e-3) / 1e9,
+                         "frac": (br + bd) / ((ms_rc + ms_dc) * 1e-3) / 1e9 / pk["hbm"],
+                         "note": "router writes the per-chunk counts; dispatch skips counting"},
             "peak_GBps": pk["hbm"], "peak_source": pk["source"] + " HBM copy",
             "mean_k": sum_k / T}
 

@@ -85,6 +85,14 @@ const char* moe_status_string(moe_status s);
 moe_status elbow_route(const float* logits, int64_t T, int N, const moe_route_params* rp,
                        int32_t* k_out, int32_t* ids_out, float* gates_out, void* stream);
 
+/* elbow_route that also counts, for the dispatch, the selected pairs of each
+ * expert in each chunk of 128 tokens: chunk_counts [N][ceil(T/128)] int32
+ * (pass moe_dispatch_chunk_counts(ws) and follow with moe_dispatch_counted,
+ * which then skips its own counting pass over k and ids). */
+moe_status elbow_route_with_counts(const float* logits, int64_t T, int N,
+                                   const moe_route_params* rp, int32_t* k_out, int32_t* ids_out,
+                                   float* gates_out, int32_t* chunk_counts, void* stream);
+
 /*
  * moe_dispatch - token-to-expert grouping of the selected (t, s < k_t) pairs,
  * as the MoE block of App. A.4 sends each token to its selected experts.

@@ -64,6 +64,7 @@ def library():
         sig = {
             "moe_status_string": ([i32], ctypes.c_char_p),
             "elbow_route": ([P, i64, i32, RP, P, P, P, P], i32),
+            "elbow_route_with_counts": ([P, i64, i32, RP, P, P, P, P, P], i32),
             "moe_dispatch_workspace_size": ([i64, i32, i32], sz),
             "moe_dispatch": ([P, P, i64, i32, i32, P, P, P, P, sz, P], i32),
             "moe_dispatch_tile_offsets": ([P, i64, i32, i32], P),
@@ -137,6 +138,23 @@ def elbow_route(logits, K: int = 8, eps: float = 1e-8, mode: int = MODE_ELBOW, r
     gates = torch.empty(T, K, dtype=torch.float32, device=logits.device)
     _check(lib.elbow_route(_p(logits), T, N, _params(K, eps, mode, renorm), _p(k), _p(ids),
                            _p(gates), _stream(stream)), "elbow_route")
+    return k, ids, gates
+
+
+def elbow_route_with_counts(logits, chunk_counts, K: int = 8, eps: float = 1e-8,
+                            mode: int = MODE_ELBOW, renorm: int = 0, stream=None):
+    """elbow_route that also writes the per-chunk expert counts (an int32 tensor of
+    [N, ceil(T/128)], e.g. dispatch_chunk_counts(ws, ...)). Returns (k, ids, gates)."""
+    torch = _torch()
+    lib = library()
+    _cuda(logits, torch.float32, "logits")
+    T, N = logits.shape
+    k = torch.empty(T, dtype=torch.int32, device=logits.device)
+    ids = torch.empty(T, K, dtype=torch.int32, device=logits.device)
+    gates = torch.empty(T, K, dtype=torch.float32, device=logits.device)
+    _check(lib.elbow_route_with_counts(_p(logits), T, N, _params(K, eps, mode, renorm), _p(k),
+                                       _p(ids), _p(gates), _p(chunk_counts), _stream(stream)),
+           "elbow_route_with_counts")
     return k, ids, gates
 
 

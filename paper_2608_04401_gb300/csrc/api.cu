@@ -142,6 +142,23 @@ moe_status elbow_route(const float* logits, int64_t T, int N, const moe_route_pa
                                              static_cast<cudaStream_t>(stream)));
 }
 
+moe_status elbow_route_with_counts(const float* logits, int64_t T, int N,
+                                   const moe_route_params* rp, int32_t* k_out, int32_t* ids_out,
+                                   float* gates_out, int32_t* chunk_counts, void* stream) {
+  if (T < 0 || T > kMaxTokens) return MOE_ERR_INVALID_ARG;
+  if (!supported_n(N)) return MOE_ERR_UNSUPPORTED;
+  moe_status st = check_route_params(rp, N);
+  if (st != MOE_OK) return st;
+  if (T == 0) return MOE_OK;
+  if (!logits || !k_out || !ids_out || !gates_out || !chunk_counts) return MOE_ERR_INVALID_ARG;
+  if (!aligned16(logits) || !aligned16(ids_out) || !aligned16(gates_out) ||
+      (reinterpret_cast<uintptr_t>(k_out) & 3u) || (reinterpret_cast<uintptr_t>(chunk_counts) & 3u))
+    return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_elbow_route(logits, T, N, rp->K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
+                                             rp->renorm, k_out, ids_out, gates_out, chunk_counts,
+                                             static_cast<cudaStream_t>(stream)));
+}
+
 size_t moe_dispatch_workspace_size(int64_t T, int N, int K) {
   (void)K;
   if (T < 0 || !supported_n(N)) return 0;

@@ -21,7 +21,7 @@ namespace disp {
 
 constexpr int kChunk = 128;  // tokens per chunk = threads per block
 constexpr int kWarps = kChunk / 32;
-constexpr int kScanThreads = 256;
+constexpr int kScanThreads = 1024;
 
 // Expert-membership bit masks of one token's selection (experts 0..63, 64..127).
 MOE_DEV void load_selection(const int32_t* __restrict__ k, const int32_t* __restrict__ ids,
@@ -78,39 +78,49 @@ __global__ void __launch_bounds__(kChunk) count_kernel(const int32_t* __restrict
 }
 
 // Block e: exclusive prefix sum of cnt[e][0 .. nblk) in place; total -> totals[e].
-// Thread i owns the contiguous range [i * per, (i + 1) * per): it sums it with
-// independent loads, the block scans the per-thread sums once, and each thread
-// rewrites its range with the running prefix.
+// Warp w owns a contiguous segment of the chunks, read in coalesced 32-chunk
+// slices: a first pass sums the segment, the block scans the warp sums, and a
+// second pass rescans each slice (eight slices loaded ahead) with the carry.
 __global__ void __launch_bounds__(kScanThreads) scan_kernel(int32_t* __restrict__ cnt, int nblk,
                                                             int32_t* __restrict__ totals) {
-  __shared__ int warp_sum[kScanThreads / 32];
+  constexpr int kW = kScanThreads / 32;
+  __shared__ int warp_sum[kW];
   int32_t* col = cnt + static_cast<int64_t>(blockIdx.x) * nblk;
   const int lane = threadIdx.x % 32, warp = threadIdx.x / 32;
-  const int per = (nblk + kScanThreads - 1) / kScanThreads;
-  const int b0 = threadIdx.x * per;
-  const int b1 = min(nblk, b0 + per);
+  const int seg = (((nblk + kW - 1) / kW) + 31) & ~31;
+  const int s0 = warp * seg;
+  const int s1 = min(nblk, s0 + seg);
   int sum = 0;
-#pragma unroll 8
-  for (int b = b0; b < b1; ++b) sum += col[b];
-  int x = sum;
+  for (int b = s0 + lane; b < s1; b += 32) sum += col[b];
 #pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, x, o);
-    if (lane >= o) x += y;
-  }
-  if (lane == 31) warp_sum[warp] = x;
+  for (int o = 16; o >= 1; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+  if (lane == 0) warp_sum[warp] = sum;
   __syncthreads();
-  int run = x - sum;
-  int total = 0;
+  int carry = 0, total = 0;
 #pragma unroll
-  for (int w = 0; w < kScanThreads / 32; ++w) {
-    if (w < warp) run += warp_sum[w];
+  for (int w = 0; w < kW; ++w) {
+    if (w < warp) carry += warp_sum[w];
     total += warp_sum[w];
   }
-  for (int b = b0; b < b1; ++b) {
-    const int v = col[b];
-    col[b] = run;
-    run += v;
+  for (int base = s0; base < s1; base += 8 * 32) {
+    int v[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int b = base + 32 * j + lane;
+      v[j] = b < s1 ? col[b] : 0;
+    }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      int x = v[j];
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+      }
+      const int b = base + 32 * j + lane;
+      if (b < s1) col[b] = carry + x - v[j];
+      carry += __shfl_sync(0xffffffffu, x, 31);
+    }
   }
   if (threadIdx.x == 0) totals[blockIdx.x] = total;
 }
@@ -147,8 +157,11 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
     int32_t* __restrict__ tile_off, int32_t* __restrict__ offsets_copy) {
   __shared__ int exp_off[N];
   __shared__ uint32_t bal[kWarps][N];
-  __shared__ int wbase[kWarps][N];
+  __shared__ int wbase[kWarps][N];   // global position of each warp's first pair per expert
+  __shared__ int lbase[kWarps][N];   // the same inside this chunk's expert-sorted pair list
   __shared__ int warp_tmp[kWarps];
+  __shared__ int s_tok[kChunk * 8];  // the chunk's pairs sorted by expert: token
+  __shared__ int s_gpos[kChunk * 8]; //                                     and global position
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int tid = threadIdx.x;
 
@@ -184,12 +197,24 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
     if (lane == (e & 31)) bal[warp][e] = b;
   }
   __syncthreads();
-  for (int e = tid; e < N; e += kChunk) {
-    int acc = exp_off[e] + base[static_cast<int64_t>(e) * nblk + blockIdx.x];
+  // this chunk's count per expert, and its exclusive scan over the experts
+  int c_e = 0;
+  if (tid < N) {
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) c_e += __popc(bal[w][tid]);
+  }
+  int chunk_pairs;
+  const int chunk_off = block_exclusive_scan_small<N>(c_e, warp_tmp, chunk_pairs);
+  if (tid < N) {
+    int acc = exp_off[tid] + base[static_cast<int64_t>(tid) * nblk + blockIdx.x];
+    int lacc = chunk_off;
 #pragma unroll
     for (int w = 0; w < kWarps; ++w) {
-      wbase[w][e] = acc;
-      acc += __popc(bal[w][e]);
+      wbase[w][tid] = acc;
+      lbase[w][tid] = lacc;
+      const int c = __popc(bal[w][tid]);
+      acc += c;
+      lacc += c;
     }
   }
   __syncthreads();
@@ -200,15 +225,25 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
       if (s < K) {
         if (s < kt) {
           const int e = my[s];
-          const int pos = wbase[warp][e] + __popc(bal[warp][e] & lt_mask);
-          // positions stay below T*K when the counts match the ids
-          if (pos >= 0 && static_cast<int64_t>(pos) < T * K) perm[pos] = static_cast<int32_t>(t);
+          const int below = __popc(bal[warp][e] & lt_mask);
+          const int pos = wbase[warp][e] + below;
+          const int lpos = lbase[warp][e] + below;
+          s_tok[lpos] = static_cast<int32_t>(t);
+          s_gpos[lpos] = pos;
           pair_pos[t * K + s] = pos;
         } else {
           pair_pos[t * K + s] = -1;
         }
       }
     }
+  }
+  __syncthreads();
+  // write perm from the expert-sorted list: consecutive threads write
+  // consecutive positions inside each expert's run
+  for (int i = tid; i < chunk_pairs; i += kChunk) {
+    const int pos = s_gpos[i];
+    // positions stay below T*K when the counts match the ids
+    if (pos >= 0 && static_cast<int64_t>(pos) < T * K) perm[pos] = s_tok[i];
   }
 }
 

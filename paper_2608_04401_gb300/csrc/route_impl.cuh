@@ -368,10 +368,11 @@ __device__ __noinline__ int route_full(const float* row, float r, int K, float e
     g[s] = (s < k) ? p : 0.0f;
   }
   write_outputs(t, K, k, ids, g, k_out, ids_out, gates_out);
-  // leave the ids in this thread's slot for the caller
-  int* slot = reinterpret_cast<int*>(keys);
+  // leave the ids for the caller in this thread's own 8-byte key slots
+  // (keys[s * kTok + tid]; a 4-byte view of that array would overlap the
+  // slots of other threads, which may still be staging their keys)
 #pragma unroll
-  for (int s = 0; s < 8; ++s) slot[s * kTok + tid] = ids[s];
+  for (int s = 0; s < 8; ++s) keys[s * kTok + tid] = static_cast<uint32_t>(ids[s]);
   return k;
 }
 
@@ -508,9 +509,8 @@ MOE_DEV int route_token(float* row, int64_t t, int tid, int K, float eps, int to
     const int kf =
         route_full<N, RC>(row, r, K, eps, topk_mode, renorm, rc, keys64, tid, t, k_out, ids_out,
                           gates_out);
-    const int* slot = reinterpret_cast<const int*>(keys64);
 #pragma unroll
-    for (int s = 0; s < 8; ++s) ids_sel[s] = slot[s * kTok + tid];
+    for (int s = 0; s < 8; ++s) ids_sel[s] = static_cast<int>(keys64[s * kTok + tid]);
     return kf;
   }
 

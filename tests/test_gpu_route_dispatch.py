@@ -66,6 +66,11 @@ def test_route_edge_cases(moe):
     r = np.zeros(N); r[::2] = 1e-7; rows.append(r)   # distinct logits, equal probabilities
     r = np.linspace(-60, 30, N); rows.append(r)      # wide range
     rng = np.random.default_rng(0)
+    # logit ranges around 86 (the unclamped exponential's domain ends there)
+    # and around the exponential's underflow limits (-87.3, -104)
+    for zlow in (-85.99, -86.0, -86.01, -87.0, -87.4, -87.8, -103.9, -104.0, -104.3, -104.6):
+        r = rng.uniform(-3.0, 0.0, N); r[0] = 0.0; r[7] = zlow; rows.append(r)
+        r = rng.uniform(zlow, zlow + 1.5, N); r[3] = 0.0; r[4] = -0.5; rows.append(r)
     q = np.round(rng.standard_normal((200, N)) * 2) / 2   # many exact ties
     lg = np.concatenate([np.array(rows), q]).astype(np.float32)
     for K in (8, 2):
@@ -165,3 +170,24 @@ def test_dispatch_full_stress(moe):
     lg = synth.boosted_logits(rng, w["T"], w["N"])
     r = oracle.route(lg, K=8)
     _dispatch_both(moe, r["k"], r["ids"], w["N"])
+
+
+@pytest.mark.parametrize("N,T", [(64, 1000), (128, 3000), (64, 70000)])
+def test_route_with_counts_then_counted_dispatch(moe, N, T):
+    """The router's per-chunk counts let the dispatch skip its counting pass;
+    routing and dispatch stay bit-exact against the oracle."""
+    import torch
+    rng = np.random.default_rng(N + T)
+    lg = synth.boosted_logits(rng, T, N)
+    ws = torch.empty(moe.dispatch_workspace_size(T, N, 8), dtype=torch.uint8, device="cuda")
+    cc = moe.dispatch_chunk_counts(ws, T, N, 8)
+    k, ids, gates = moe.elbow_route_with_counts(to_dev(lg), cc)
+    off, perm, pp = moe.moe_dispatch_counted(k, ids, N, ws)
+    torch.cuda.synchronize()
+    ref = oracle.route(lg, K=8)
+    _assert_route_equal((k.cpu().numpy(), ids.cpu().numpy(), gates.cpu().numpy()), ref)
+    d = oracle.dispatch(ref["k"], ref["ids"], N)
+    assert np.array_equal(off.cpu().numpy(), d["offsets"])
+    n = int(d["offsets"][-1])
+    assert np.array_equal(perm.cpu().numpy()[:n], d["perm"])
+    assert np.array_equal(pp.cpu().numpy(), d["pair_pos"])
