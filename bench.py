@@ -239,6 +239,7 @@ def run_ours(args, rank, world, local, pg):
     kern["down"].update(tflops=dn_tf, frac=dn_tf / pk["bf16_sus"])
 
     route = route_stress(moe, args, stream, dev, pk)
+    others = other_configs(moe, args, stream, dev, pk, pg)
 
     # end to end through the public API with host buffers
     xh = torch.empty(T, d, dtype=torch.bfloat16, pin_memory=True)
@@ -290,6 +291,7 @@ def run_ours(args, rank, world, local, pg):
                      "frac_of_burst": gu_tf / pk["bf16"]},
         "kernels": kern,
         "route_stress": route,
+        "other_configs": others,
         "e2e": {"value": world * T / (ms_e2e * 1e-3), "unit": "tokens/s", "ms_per_step": ms_e2e,
                 "h2d_bytes_per_step": T * d * 2, "d2h_bytes_per_step": T * d * 2},
         "gpu_launches": KERNELS_PER_STEP * args.steps * 2,
@@ -312,6 +314,9 @@ def kernel_breakdown(moe, x, wr, wgu, wd, T, d, N, I, K, args, stream, dev):
     steps = max(10, args.steps // 4)
     dws = torch.empty(moe.dispatch_workspace_size(T, N, K), dtype=torch.uint8, device=dev)
     cc = moe.dispatch_chunk_counts(dws, T, N, K)
+    # all steps are enqueued back to back (the host runs ahead of the GPU), so
+    # each interval between two events is device time, not launch latency
+    evs = []
     for it in range(steps + 3):
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)]
         ev[0].record(stream)
@@ -327,13 +332,119 @@ def kernel_breakdown(moe, x, wr, wgu, wd, T, d, N, I, K, args, stream, dev):
         ev[4].record(stream)
         moe.combine(o, k, pp, gates)
         ev[5].record(stream)
-        torch.cuda.synchronize()
         if it >= 3:
-            for i, n in enumerate(names):
-                acc[n] += ev[i].elapsed_time(ev[i + 1])
+            evs.append(ev)
+    torch.cuda.synchronize()
+    for ev in evs:
+        for i, n in enumerate(names):
+            acc[n] += ev[i].elapsed_time(ev[i + 1])
     assert int(err.item()) == 0, "device timeout in a GEMM"
     tot = sum(acc.values())
     return {n: {"ms": acc[n] / steps, "share": acc[n] / tot} for n in names}
+
+
+def dev_experts(N, d, I, seed, dev):
+    """Expert weights ~ N(0, 0.02^2), drawn on the device (seeded) and stored bf16."""
+    import torch
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+    wgu = torch.empty(N, 2 * I, d, dtype=torch.bfloat16, device=dev)
+    wd = torch.empty(N, d, I, dtype=torch.bfloat16, device=dev)
+    for w in (wgu, wd):
+        for e in range(N):
+            w[e].copy_(torch.randn(w.shape[1:], generator=g, device=dev) * 0.02)
+    return wgu, wd
+
+
+def time_layer_modes(moe, x, wr, wgu, wd, K, steps, stream, pg, residual=None):
+    """ms per moe_layer_forward in elbow and in top-K mode; sum k of the elbow batch."""
+    import torch
+    T, d = x.shape
+    N = wr.shape[0]
+    I = wgu.shape[1] // 2
+    ws = torch.empty(moe.layer_workspace_size(T, d, N, I, K), dtype=torch.uint8, device=x.device)
+    y = torch.empty(T, d, dtype=torch.bfloat16, device=x.device)
+    out = {}
+    for name, mode in (("elbow", moe.MODE_ELBOW), ("topk", moe.MODE_TOPK)):
+        def step():
+            moe.moe_layer_forward(x, wr, wgu, wd, K=K, mode=mode, residual=residual, y=y, ws=ws)
+        for _ in range(3):
+            step()
+        out[name] = time_steps(step, steps, stream, pg)
+    moe.read_device_error(ws)
+    _, it = moe.moe_layer_forward(x, wr, wgu, wd, K=K, y=y, ws=ws, return_intermediates=True)
+    out["sum_k"] = int(it["k"].sum().item())
+    out["touched"] = int((np.diff(it["offsets"].cpu().numpy()) > 0).sum())
+    return out
+
+
+def other_configs(moe, args, stream, dev, pk, pg):
+    """The small (64-token), wide-router (N = 128) and 16-layer-stack workloads,
+    timed with the same kernels in elbow and fixed top-8 mode. Expert weights
+    are drawn on the device; tokens and routers follow the synthetic recipe."""
+    import torch
+    from paper_2608_04401_gb300 import synth
+    res = {}
+    steps = max(20, args.steps // 4)
+    for name in ("layer_t64", "layer_wide"):
+        w = synth.WORKLOADS[name]
+        T, d, N, I, K = w["T"], w["d"], w["N"], w["I"], w["K"]
+        inp = synth.layer_inputs(T=T, d=d, N=N, I=I, seed=w["seed"],
+                                 flat_frac=w.get("flat_frac", 0.0), with_experts=False)
+        x, wr = bf16_dev(inp["x"], dev), bf16_dev(inp["w_router"], dev)
+        wgu, wd = dev_experts(N, d, I, w["seed"], dev)
+        r = time_layer_modes(moe, x, wr, wgu, wd, K, steps, stream, pg)
+        flops = 6.0 * d * I * r["sum_k"]
+        # bytes: the touched experts' weights, x and y
+        wbytes = r["touched"] * 3 * d * I * 2 + 2 * T * d * 2
+        res[name] = {
+            "workload": f"T={T}, d_model={d}, N={N}, I={I}, K={K}"
+                        + (f", {int(100 * w['flat_frac'])}% flat tokens" if "flat_frac" in w else ""),
+            "elbow_ms": r["elbow"], "topk_ms": r["topk"], "elbow_speedup": r["topk"] / r["elbow"],
+            "tokens_per_s": T / (r["elbow"] * 1e-3), "mean_k": r["sum_k"] / T,
+            "experts_touched": r["touched"],
+            "tflops": flops / (r["elbow"] * 1e-3) / 1e12,
+            "weight_hbm_frac": wbytes / (r["elbow"] * 1e-3) / 1e9 / pk["hbm"],
+        }
+        del wgu, wd
+        torch.cuda.empty_cache()
+    # 16-layer stack with the residual add between layers
+    w = synth.WORKLOADS["stack16_t4k"]
+    T, d, N, I, K, L = w["T"], w["d"], w["N"], w["I"], w["K"], w["L"]
+    x0_bits, routers = synth.stack_inputs(T, d, N, L, w["seed"])
+    layers = [(bf16_dev(routers[l], dev),) + dev_experts(N, d, I, synth.stack_expert_seed(w["seed"], l), dev)
+              for l in range(L)]
+    x0 = bf16_dev(x0_bits, dev)
+    ws = torch.empty(moe.layer_workspace_size(T, d, N, I, K), dtype=torch.uint8, device=dev)
+    bufs = [torch.empty(T, d, dtype=torch.bfloat16, device=dev) for _ in range(2)]
+    out = {}
+    for name, mode in (("elbow", moe.MODE_ELBOW), ("topk", moe.MODE_TOPK)):
+        def stack():
+            cur = x0
+            for l, (wr, wgu, wd) in enumerate(layers):
+                nxt = bufs[l % 2]
+                moe.moe_layer_forward(cur, wr, wgu, wd, K=K, mode=mode, residual=cur, y=nxt, ws=ws)
+                cur = nxt
+        for _ in range(2):
+            stack()
+        out[name] = time_steps(stack, max(5, steps // 4), stream, pg)
+    moe.read_device_error(ws)
+    mean_k = []
+    cur = x0
+    for l, (wr, wgu, wd) in enumerate(layers):
+        nxt = bufs[l % 2]
+        _, it = moe.moe_layer_forward(cur, wr, wgu, wd, K=K, residual=cur, y=nxt, ws=ws,
+                                      return_intermediates=True)
+        mean_k.append(round(float(it["k"].float().mean().item()), 3))
+        cur = nxt
+    res["stack16_t4k"] = {
+        "workload": f"{L} layers, T={T}, d_model={d}, N={N}, I={I}, K={K}, residual add",
+        "elbow_ms": out["elbow"], "topk_ms": out["topk"], "elbow_speedup": out["topk"] / out["elbow"],
+        "tokens_per_s": T / (out["elbow"] * 1e-3), "mean_k_per_layer": mean_k,
+    }
+    del layers
+    torch.cuda.empty_cache()
+    return res
 
 
 def route_stress(moe, args, stream, dev, pk):

@@ -41,6 +41,8 @@ __all__ = [
     "tokens",
     "expert_weights",
     "boosted_logits",
+    "stack_inputs",
+    "stack_expert_seed",
     "layer_inputs",
 ]
 
@@ -130,6 +132,22 @@ def expert_weights(seed: int, N: int, d: int, I: int):
     with ThreadPoolExecutor(max_workers=min(16, os.cpu_count() or 1)) as ex:
         list(ex.map(one, range(N)))
     return wgu, wd
+
+
+def stack_inputs(T: int, d: int, N: int, L: int, seed: int):
+    """Inputs of an L-layer stack: the tokens x_0 and layer 0's router follow the
+    layer recipe (seed); layer l >= 1 draws its own router from
+    PCG64(SeedSequence([seed, l])). Experts: expert_weights(seed * 100 + l, ...)."""
+    first = layer_inputs(T=T, d=d, N=N, I=0, seed=seed, with_experts=False)
+    routers = [first["w_router"]]
+    for l in range(1, L):
+        g = np.random.Generator(np.random.PCG64(np.random.SeedSequence([seed, l])))
+        routers.append(router_weights(g, N, d)[0])
+    return first["x"], routers
+
+
+def stack_expert_seed(seed: int, l: int) -> int:
+    return seed * 100 + l
 
 
 def boosted_logits(rng: np.random.Generator, T: int, N: int, chunk: int = 1 << 17):
