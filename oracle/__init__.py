@@ -11,7 +11,8 @@ Functions and the passages they follow:
   router_logits  l(x) = W_r x of Sec. 2, fp64 accumulation rounded to fp32
   layer_rows     the whole MoE layer forward (App. A.4) for chosen tokens, fp64
   load_balance   L_i, q_i, delta and the bounds of Theorem 1 / Corollaries 1-2
-                 (App. A.3)
+                 (App. A.3), the percentage changes of Sec. 4.3
+  elbow_angle    the uncapped elbow index and the elbow angle of Sec. 3.1
   exp / exp_max_ulp  the fp32 routing exponential and its error sweep
 The readings taken where the paper is silent or garbled are listed in the
 header of elbow_oracle.c.
@@ -62,6 +63,10 @@ def _load():
         lib.oracle_exp_max_ulp.restype = ctypes.c_double
         lib.oracle_route.argtypes = [P, i64, i32, i32, f32, i32, i32, P, P, P, P, P]
         lib.oracle_route.restype = i32
+        lib.oracle_elbow_angle.argtypes = [P, i64, i32, f32, P, P]
+        lib.oracle_elbow_angle.restype = i32
+        lib.oracle_angle_deg.argtypes = [i32, i32, f32]
+        lib.oracle_angle_deg.restype = ctypes.c_double
         lib.oracle_dispatch.argtypes = [P, P, i64, i32, i32, P, P, P]
         lib.oracle_dispatch.restype = i32
         lib.oracle_router_logits.argtypes = [P, P, i64, i32, i32, P, i64, P]
@@ -177,6 +182,24 @@ def layer_rows(x_bits, w_router_bits, w_gate_up_bits, w_down_bits, rows=None, K:
     return dict(y=y, logits=lg, k=k, ids=ids, gates=gates)
 
 
+def elbow_angle(logits, eps: float = 1e-8):
+    """Per token of fp32 logits [T, N]: the uncapped elbow index (argmax of D
+    over all ranks) and the elbow angle in degrees (Sec. 3.1, reading R11)."""
+    lib = _load()
+    lg = _c(logits, np.float32)
+    T, N = lg.shape
+    e = np.empty(T, np.int32)
+    th = np.empty(T, np.float32)
+    if lib.oracle_elbow_angle(_ptr(lg), T, N, eps, _ptr(e), _ptr(th)) != 0:
+        raise ValueError("oracle_elbow_angle: unsupported arguments")
+    return dict(elbow=e, theta=th)
+
+
+def angle_deg(e: int, N: int, pn_e: float) -> float:
+    """The elbow angle (degrees, fp64) at rank e of an N-point curve with p'_e = pn_e."""
+    return float(_load().oracle_angle_deg(int(e), int(N), float(np.float32(pn_e))))
+
+
 def load_balance(k_elb, ids, N: int):
     """Expert loads under elbow-K and top-K routing of the same tokens (App. A.3).
 
@@ -199,6 +222,7 @@ def load_balance(k_elb, ids, N: int):
     q_elb = L_elb / L_elb.sum()
     delta = 1.0 - k_elb.mean() / K
     cv2 = lambda q: N * float(np.dot(q, q)) - 1.0
+    cv_top, cv_elb = np.sqrt(max(cv2(q_top), 0.0)), np.sqrt(max(cv2(q_elb), 0.0))
     return dict(
         L_top=L_top, L_elb=L_elb, q_top=q_top, q_elb=q_elb, delta=delta,
         l1=float(np.abs(q_elb - q_top).sum()),
@@ -206,4 +230,7 @@ def load_balance(k_elb, ids, N: int):
         max_change=abs(q_elb.max() - q_top.max()),
         cv2_change=abs(cv2(q_elb) - cv2(q_top)),
         cv2_bound=2 * N * delta / (1 - delta) ** 2,
+        # the percentages of Sec. 4.3
+        top1_share_change_pct=(q_top.max() - q_elb.max()) / q_top.max() * 100.0,
+        cv_change_pct=(cv_top - cv_elb) / cv_top * 100.0 if cv_top > 0 else 0.0,
     )

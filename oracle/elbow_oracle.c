@@ -42,6 +42,11 @@
  *   R7  Expert MLP: SwiGLU, y_e = W_down (silu(W_gate x) * (W_up x)),
  *       silu(z) = z / (1 + exp(-z)), evaluated in fp64 on the bf16 inputs.
  *
+ *   R11 Elbow angle (Sec. 3.1): the printed points (0,0), (x'_e, p'_e), (1,1)
+ *       are read on the curve y' = 1 - p' that R1's chord uses (p' itself
+ *       runs from (0,1) to (1,0)); theta is evaluated in fp64 from the fp32
+ *       x'_e and p'_e, and is 180 degrees when the elbow is an end point.
+ *
  * EXP, the routing exponential (written for this project from Cody & Waite's
  * argument reduction, 1980, and the Taylor series of exp):
  *   if !(z >= -104) return 0;  if z > 88 return +inf
@@ -129,7 +134,8 @@ double oracle_exp_max_ulp(float lo, float hi, float* worst_z) {
 
 /* Algorithm 1 plus capped selection for one token. Returns k. */
 static int route_one(const float* l, int N, int K, float eps, int mode, int renorm,
-                     int32_t* ids, float* gates, float* sorted_p, int32_t* elbow_e) {
+                     int32_t* ids, float* gates, float* sorted_p, int32_t* elbow_e,
+                     float* elbow_pn) {
   float e[ORACLE_MAX_N], p[ORACLE_MAX_N], v[ORACLE_MAX_N];
   int idx[ORACLE_MAX_N];
 
@@ -162,7 +168,7 @@ static int route_one(const float* l, int N, int K, float eps, int mode, int reno
   float den = (p_max - p_min) + eps;
   float inv = 1.0f / den;
   int e_arg = 0;
-  float d_best = 0.0f;
+  float d_best = 0.0f, pn_best = 0.0f;
   for (int i = 0; i < N; ++i) {
     float pn = (p[idx[i]] - p_min) * inv;
     float xn = (float)i / (float)(N - 1);
@@ -170,9 +176,11 @@ static int route_one(const float* l, int N, int K, float eps, int mode, int reno
     if (i == 0 || D > d_best) {
       d_best = D;
       e_arg = i;
+      pn_best = pn;
     }
   }
   if (elbow_e) *elbow_e = e_arg;
+  if (elbow_pn) *elbow_pn = pn_best;
 
   /* k(x) = min(e(x), K) with e(x) = argmax + 1 (R2); fixed top-K: k = K */
   int k = (mode == 1) ? K : (e_arg + 1 < K ? e_arg + 1 : K);
@@ -201,7 +209,46 @@ int oracle_route(const float* logits, int64_t T, int N, int K, float eps, int mo
   for (int64_t t = 0; t < T; ++t) {
     k_out[t] = route_one(logits + t * N, N, K, eps, mode, renorm, ids_out + t * K,
                          gates_out + t * K, sorted_p_out ? sorted_p_out + t * N : NULL,
-                         elbow_out ? elbow_out + t : NULL);
+                         elbow_out ? elbow_out + t : NULL, NULL);
+  }
+  return 0;
+}
+
+/* Elbow angle (Sec. 3.1): the angle at the elbow point between the first and
+ * the last point of the normalised curve. With the deviation read as below
+ * the chord (R1), the normalised curve is (x'_i, y'_i) = (i/(N-1), 1 - p'_i),
+ * from (0,0) to (1,1); at the elbow e, v1 = (0,0) - (x'_e, y'_e) and
+ * v2 = (1,1) - (x'_e, y'_e), theta = arccos(v1.v2 / (|v1| |v2|)) (R11).
+ * x'_e and p'_e are the fp32 values of the elbow step; the angle is evaluated
+ * in fp64 and returned in degrees. A zero-length v1 or v2 (the elbow on an end
+ * point) gives 180 degrees (no bend). */
+static const double ORACLE_PI = 3.14159265358979323846;
+
+double oracle_angle_deg(int e, int N, float pn_e) {
+  double x = (double)((float)e / (float)(N - 1));
+  double y = 1.0 - (double)pn_e;
+  double ax = -x, ay = -y, bx = 1.0 - x, by = 1.0 - y;
+  double na = sqrt(ax * ax + ay * ay), nb = sqrt(bx * bx + by * by);
+  if (na == 0.0 || nb == 0.0) return 180.0;
+  double c = (ax * bx + ay * by) / (na * nb);
+  if (c > 1.0) c = 1.0;
+  if (c < -1.0) c = -1.0;
+  return acos(c) * (180.0 / ORACLE_PI);
+}
+
+/* Per token: the uncapped elbow index e (argmax of D over all N ranks) and
+ * the elbow angle in degrees (rounded to fp32). Returns 0, or -1 on
+ * unsupported arguments (as oracle_route). */
+int oracle_elbow_angle(const float* logits, int64_t T, int N, float eps, int32_t* elbow_out,
+                       float* theta_out) {
+  if (N < 2 || N > ORACLE_MAX_N || (N & (N - 1)) != 0 || T < 0) return -1;
+#pragma omp parallel for schedule(static)
+  for (int64_t t = 0; t < T; ++t) {
+    int32_t id1, e;
+    float g1, pn;
+    route_one(logits + t * N, N, 1, eps, 0, 0, &id1, &g1, NULL, &e, &pn);
+    elbow_out[t] = e;
+    theta_out[t] = (float)oracle_angle_deg(e, N, pn);
   }
   return 0;
 }
@@ -320,7 +367,7 @@ int oracle_layer_rows(const uint16_t* x, const uint16_t* w_router, const uint16_
       for (int c = 0; c < d; ++c) acc += xd[c] * bf16_to_double(w_router[(int64_t)j * d + c]);
       l[j] = (float)acc;
     }
-    int k = route_one(l, N, K, eps, mode, renorm, ids, gates, NULL, NULL);
+    int k = route_one(l, N, K, eps, mode, renorm, ids, gates, NULL, NULL, NULL);
     double* yr = y + r * d;
     for (int c = 0; c < d; ++c) yr[c] = 0.0;
     for (int s = 0; s < k; ++s) {

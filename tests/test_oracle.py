@@ -242,6 +242,72 @@ def test_theorem1_and_corollaries():
         np.testing.assert_allclose(lb["L_elb"].sum(), r["k"].mean())
 
 
+def test_load_balance_hand_example():
+    """Two tokens, N = 4, K = 2: token 0 keeps expert 0 of (0, 1), token 1 keeps
+    both of (0, 2). By hand: q_top = (1/2, 1/4, 1/4, 0), q_elb = (2/3, 0, 1/3, 0),
+    delta = 1/4, l1 = 1/2 <= 2/3, CV^2 = 1/2 and 11/9, top-1 share change
+    (1/2 - 2/3) / (1/2) = -100/3 %, CV change (sqrt(1/2) - sqrt(11/9)) / sqrt(1/2)."""
+    lb = oracle.load_balance(np.array([1, 2]), np.array([[0, 1], [0, 2]]), 4)
+    np.testing.assert_allclose(lb["q_top"], [0.5, 0.25, 0.25, 0.0], atol=1e-15)
+    np.testing.assert_allclose(lb["q_elb"], [2 / 3, 0.0, 1 / 3, 0.0], atol=1e-15)
+    assert abs(lb["delta"] - 0.25) < 1e-15
+    assert abs(lb["l1"] - 0.5) < 1e-15 and abs(lb["l1_bound"] - 2 / 3) < 1e-15
+    assert abs(lb["cv2_change"] - (11 / 9 - 0.5)) < 1e-14
+    assert abs(lb["top1_share_change_pct"] + 100 / 3) < 1e-12
+    want = (np.sqrt(0.5) - np.sqrt(11 / 9)) / np.sqrt(0.5) * 100
+    assert abs(lb["cv_change_pct"] - want) < 1e-12
+
+
+# ------------------------------------------------------ elbow angle (Sec. 3.1)
+@pytest.mark.parametrize("N", [64, 128])
+def test_elbow_angle_step_curves(N):
+    """A step of m equal high values has its elbow at e = m with p'_e = 0, so
+    v1 = (-x, -1), v2 = (1 - x, 0) and theta = 90 deg + atan(x), x = m/(N-1)."""
+    for m in (1, 2, 3, 7, 8, 20, N // 2, N - 2):
+        lg = np.zeros((1, N), np.float32)
+        lg[0, :m] = 6.0
+        a = oracle.elbow_angle(lg)
+        assert a["elbow"][0] == m
+        x = float(np.float32(m) / np.float32(N - 1))
+        assert abs(float(a["theta"][0]) - (90.0 + np.degrees(np.arctan(x)))) < 2e-5
+
+
+def test_elbow_angle_uniform_and_range():
+    """The uniform curve: e = 0, p' = 0, v1 = (0, -1), v2 = (1, 0): 90 degrees.
+    Every angle lies in [0, 180]."""
+    a = oracle.elbow_angle(np.zeros((3, 64), np.float32))
+    assert np.all(a["elbow"] == 0) and np.all(a["theta"] == 90.0)
+    lg = synth.boosted_logits(np.random.default_rng(4), 3000, 64)
+    a = oracle.elbow_angle(lg)
+    assert np.all((a["theta"] >= 0) & (a["theta"] <= 180))
+
+
+@pytest.mark.parametrize("N", [64, 128])
+def test_elbow_angle_vs_atan2(N):
+    """Recomputed from the sorted curve with atan2 (the angle between the two
+    directions, no dot product or arccos), on random curves; the uncapped
+    elbow index agrees with the routing's."""
+    rng = np.random.default_rng(N + 5)
+    lg = synth.boosted_logits(rng, 500, N)
+    a = oracle.elbow_angle(lg)
+    r = oracle.route(lg, K=8, with_sorted=True)
+    assert np.array_equal(a["elbow"], r["elbow"])
+    assert np.array_equal(r["k"], np.minimum(a["elbow"] + 1, 8))
+    f = np.float32
+    for t in range(500):
+        sp = r["sorted_p"][t]
+        e = int(a["elbow"][t])
+        inv = f(1) / (f(sp[0] - sp[-1]) + f(1e-8))
+        pn = f(f(sp[e] - sp[-1]) * inv)
+        x = float(f(e) / f(N - 1))
+        y = 1.0 - float(pn)
+        a1 = np.arctan2(-y, -x)
+        a2 = np.arctan2(1.0 - y, 1.0 - x)
+        th = abs(np.degrees(a1 - a2))
+        th = 360.0 - th if th > 180.0 else th
+        assert abs(th - float(a["theta"][t])) < 2e-4, (t, th, a["theta"][t])
+
+
 # --------------------------------------------------------------- dispatch
 def _check_dispatch(k, ids, N):
     out = oracle.dispatch(k, ids, N)
