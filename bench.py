@@ -18,6 +18,7 @@ data-path collective); timing is max over ranks.
 from __future__ import annotations
 
 import argparse
+import ctypes
 import json
 import os
 import statistics
@@ -483,12 +484,22 @@ def route_stress(moe, args, stream, dev, pk):
         lib.moe_dispatch_counted(P(k), P(ids), T, N, K, P(off), P(perm), P(pp), P(dws),
                                  dws.numel(), s)
 
+    diag_buf = torch.empty(ctypes.sizeof(moe.RouteDiag), dtype=torch.uint8, device=dev)
+    theta = torch.empty(T, dtype=torch.float32, device=dev)
+    elbow = torch.empty(T, dtype=torch.int32, device=dev)
+
+    def diagnose():
+        lib.moe_route_diagnostics(P(lg), T, N, rp, P(elbow), P(theta), P(diag_buf), s)
+
     for _ in range(3):
         route()
         disp()
         route_counted()
         disp_counted()
+        diagnose()
     n = max(20, args.steps // 4)
+    ms_diag = time_steps(diagnose, max(5, n // 4), stream, None)
+    st, _, th = moe.route_diagnostics(lg, K=K, diag=diag_buf)
     ms_r = time_steps(route, n, stream, None)
     ms_d = time_steps(disp, n, stream, None)
     ms_rc = time_steps(route_counted, n, stream, None)
@@ -509,7 +520,15 @@ def route_stress(moe, args, stream, dev, pk):
                          "frac": (br + bd) / ((ms_rc + ms_dc) * 1e-3) / 1e9 / pk["hbm"],
                          "note": "router writes the per-chunk counts; dispatch skips counting"},
             "peak_GBps": pk["hbm"], "peak_source": pk["source"] + " HBM copy",
-            "mean_k": sum_k / T}
+            "mean_k": sum_k / T,
+            "diagnostics": {
+                "ms": ms_diag, "note": "whole sorted curve per token (uncapped elbow, angle, loads)",
+                "mean_k": st["mean_k"], "delta": st["delta"], "l1": st["l1"],
+                "l1_bound": st["l1_bound"], "top1_share_change_pct": st["top1_share_change_pct"],
+                "cv_change_pct": st["cv_change_pct"], "cv2_change": st["cv2_change"],
+                "cv2_bound": st["cv2_bound"], "sharp_elbow_frac": st["sharp_elbows"] / T,
+                "mean_theta_deg": float(th.double().mean().item()),
+                "elbow_index_hist": st["elbow_hist"][:16].tolist()}}
 
 
 def cpu_baseline(inp, K, budget_s=12.0):

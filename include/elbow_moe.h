@@ -246,6 +246,54 @@ moe_status moe_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_
                        const float* gates, const uint16_t* residual, int64_t T, int d, int K,
                        uint16_t* y, void* stream);
 
+/*
+ * moe_route_diagnostics - routing diagnostics of Sec. 3.1 (elbow angle),
+ * Sec. 4.3 and App. A.3 (expert-load changes of elbow-K against top-K).
+ *
+ * Per token, the whole sorted curve is evaluated with the fp32 steps of
+ * elbow_route; e is the UNCAPPED elbow index (first argmax of D over all N
+ * ranks, so k = min(e + 1, K)), and the elbow angle theta is the angle at the
+ * elbow point (x'_e, 1 - p'_e) between the first (0,0) and the last (1,1)
+ * point of the normalised curve, evaluated in fp64 and rounded to fp32
+ * degrees (180 when the elbow is an end point).
+ *
+ *   logits     [T, N] fp32   router logits
+ *   rp         K and eps are used; mode and renorm are ignored
+ *   elbow_out  [T] int32     e per token (may be NULL)
+ *   theta_out  [T] fp32      theta per token, degrees (may be NULL)
+ *   diag       device pointer to one moe_route_diag, overwritten (8-byte
+ *              aligned): integer histograms of the batch, and the normalised
+ *              utilisations q = L / sum(L) of both selections reduced to
+ *              delta = 1 - E[k]/K, the l1 change (bound 2 delta / (1 - delta),
+ *              Theorem 1), the change of the largest share (Corollary 1, same
+ *              bound), the change of CV^2 = N |q|^2 - 1 (bound
+ *              2 N delta / (1 - delta)^2, Corollary 2), and the percentage
+ *              changes of the top-1 share and of CV (Sec. 4.3).
+ * Integer counts make every field independent of block order. Errors as
+ * elbow_route; diag NULL or misaligned: MOE_ERR_INVALID_ARG.
+ */
+#define MOE_DIAG_MAX_N 128
+typedef struct {
+  int64_t tokens;                        /* T */
+  int64_t sharp_elbows;                  /* tokens with theta <= 135 degrees */
+  int64_t k_hist[9];                     /* tokens with k = 0..8 */
+  int64_t elbow_hist[MOE_DIAG_MAX_N];    /* tokens with uncapped elbow index e */
+  int64_t theta_hist[181];               /* tokens with floor(theta) = 0..180 */
+  int64_t load_top[MOE_DIAG_MAX_N];      /* selected pairs per expert, top-K */
+  int64_t load_elb[MOE_DIAG_MAX_N];      /* selected pairs per expert, elbow-K */
+  double mean_k;                         /* E[k] */
+  double delta;                          /* 1 - E[k] / K */
+  double l1, l1_bound;                   /* |q_elb - q_top|_1 and 2 delta / (1 - delta) */
+  double top1_change;                    /* | max q_elb - max q_top | */
+  double cv2_change, cv2_bound;          /* |CV^2 change| and 2 N delta / (1 - delta)^2 */
+  double top1_share_change_pct;          /* (max q_top - max q_elb) / max q_top * 100 */
+  double cv_change_pct;                  /* (CV_top - CV_elb) / CV_top * 100 */
+} moe_route_diag;
+
+moe_status moe_route_diagnostics(const float* logits, int64_t T, int N, const moe_route_params* rp,
+                                 int32_t* elbow_out, float* theta_out, moe_route_diag* diag,
+                                 void* stream);
+
 #ifdef __cplusplus
 }
 #endif

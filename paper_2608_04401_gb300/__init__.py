@@ -15,8 +15,10 @@ import ctypes
 import os
 import threading
 
+import numpy as np
+
 __all__ = [
-    "MODE_ELBOW", "MODE_TOPK", "MoeError", "library", "build",
+    "MODE_ELBOW", "MODE_TOPK", "MoeError", "library", "build", "route_diagnostics", "RouteDiag",
     "elbow_route", "moe_dispatch", "moe_dispatch_noalloc", "dispatch_workspace_size", "layer_workspace_size",
     "moe_layer_forward", "read_device_error", "router_logits", "gather_rows",
     "expert_gate_up", "expert_down", "combine",
@@ -43,6 +45,18 @@ class RouteParams(ctypes.Structure):
                 ("renorm", ctypes.c_int)]
 
 
+class RouteDiag(ctypes.Structure):
+    """Host mirror of moe_route_diag (include/elbow_moe.h)."""
+    _fields_ = [("tokens", ctypes.c_int64), ("sharp_elbows", ctypes.c_int64),
+                ("k_hist", ctypes.c_int64 * 9), ("elbow_hist", ctypes.c_int64 * 128),
+                ("theta_hist", ctypes.c_int64 * 181), ("load_top", ctypes.c_int64 * 128),
+                ("load_elb", ctypes.c_int64 * 128), ("mean_k", ctypes.c_double),
+                ("delta", ctypes.c_double), ("l1", ctypes.c_double), ("l1_bound", ctypes.c_double),
+                ("top1_change", ctypes.c_double), ("cv2_change", ctypes.c_double),
+                ("cv2_bound", ctypes.c_double), ("top1_share_change_pct", ctypes.c_double),
+                ("cv_change_pct", ctypes.c_double)]
+
+
 def build(force: bool = False) -> str:
     """Compile libelbow_moe.so in-tree (nvcc, sm_103a)."""
     from . import buildlib
@@ -65,6 +79,7 @@ def library():
             "moe_status_string": ([i32], ctypes.c_char_p),
             "elbow_route": ([P, i64, i32, RP, P, P, P, P], i32),
             "elbow_route_with_counts": ([P, i64, i32, RP, P, P, P, P, P], i32),
+            "moe_route_diagnostics": ([P, i64, i32, RP, P, P, P, P], i32),
             "moe_dispatch_workspace_size": ([i64, i32, i32], sz),
             "moe_dispatch": ([P, P, i64, i32, i32, P, P, P, P, sz, P], i32),
             "moe_dispatch_tile_offsets": ([P, i64, i32, i32], P),
@@ -156,6 +171,32 @@ def elbow_route_with_counts(logits, chunk_counts, K: int = 8, eps: float = 1e-8,
                                        _p(ids), _p(gates), _p(chunk_counts), _stream(stream)),
            "elbow_route_with_counts")
     return k, ids, gates
+
+
+def route_diagnostics(logits, K: int = 8, eps: float = 1e-8, per_token: bool = True,
+                      diag=None, stream=None):
+    """Routing diagnostics of fp32 logits [T, N] (moe_route_diagnostics).
+    Returns (stats dict, elbow [T] int32 or None, theta [T] fp32 degrees or None);
+    `diag` may be a device uint8 tensor of sizeof(RouteDiag) bytes to reuse."""
+    torch = _torch()
+    _cuda(logits, torch.float32, "logits")
+    T, N = logits.shape
+    dev = logits.device
+    if diag is None:
+        diag = torch.empty(ctypes.sizeof(RouteDiag), dtype=torch.uint8, device=dev)
+    el = torch.empty(T, dtype=torch.int32, device=dev) if per_token else None
+    th = torch.empty(T, dtype=torch.float32, device=dev) if per_token else None
+    _check(library().moe_route_diagnostics(_p(logits), T, N, _params(K, eps, MODE_ELBOW, 0),
+                                           _p(el), _p(th), _p(diag), _stream(stream)),
+           "moe_route_diagnostics")
+    host = RouteDiag.from_buffer_copy(diag.cpu().numpy().tobytes())
+    out = {}
+    for name, _ in RouteDiag._fields_:
+        v = getattr(host, name)
+        out[name] = np.array(v[:], dtype=np.int64) if hasattr(v, "__len__") else v
+    for name in ("elbow_hist", "load_top", "load_elb"):
+        out[name] = out[name][:N]
+    return out, el, th
 
 
 def dispatch_workspace_size(T: int, N: int, K: int) -> int:

@@ -36,6 +36,9 @@ cudaError_t launch_gateup_gather_gemm(const uint16_t* x, int64_t T, const int32_
                                       const uint16_t* wgu, const int32_t* offsets,
                                       const int32_t* tile_off, int64_t P, int d, int N, int I,
                                       uint16_t* h, int32_t* err, int num_sms, cudaStream_t stream);
+cudaError_t launch_route_diagnostics(const float* logits, int64_t T, int N, int K, float eps,
+                                     int32_t* elbow_out, float* theta_out, moe_route_diag* dg,
+                                     cudaStream_t stream);
 }  // namespace moe
 
 namespace {
@@ -140,6 +143,22 @@ moe_status elbow_route(const float* logits, int64_t T, int N, const moe_route_pa
   return cuda_status(moe::launch_elbow_route(logits, T, N, rp->K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
                                              rp->renorm, k_out, ids_out, gates_out, nullptr,
                                              static_cast<cudaStream_t>(stream)));
+}
+
+moe_status moe_route_diagnostics(const float* logits, int64_t T, int N, const moe_route_params* rp,
+                                 int32_t* elbow_out, float* theta_out, moe_route_diag* diag,
+                                 void* stream) {
+  if (T < 0 || T > kMaxTokens) return MOE_ERR_INVALID_ARG;
+  if (!supported_n(N)) return MOE_ERR_UNSUPPORTED;
+  moe_status st = check_route_params(rp, N);
+  if (st != MOE_OK) return st;
+  if (!diag || (reinterpret_cast<uintptr_t>(diag) & 7u)) return MOE_ERR_INVALID_ARG;
+  if (T > 0 && (!logits || !aligned16(logits))) return MOE_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(elbow_out) & 3u) || (reinterpret_cast<uintptr_t>(theta_out) & 3u))
+    return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_route_diagnostics(logits, T, N, rp->K, rp->eps, elbow_out,
+                                                   theta_out, diag,
+                                                   static_cast<cudaStream_t>(stream)));
 }
 
 moe_status elbow_route_with_counts(const float* logits, int64_t T, int N,

@@ -265,13 +265,15 @@ __global__ void __launch_bounds__(256) gather_kernel(const uint4* __restrict__ x
 
 // y_t = sum_{s<k_t} g_{t,s} * o[pair_pos[t,s]] (+ residual_t); fp32 in s order.
 // One warp per token. The token's k positions and gates are read once (lane s
-// holds pair s) and broadcast by shuffles; the row is processed in slabs of
-// 256 sixteen-byte chunks, lane l holding chunks l + 32c (c < 8) of the slab,
-// so each of the k rows is fetched with eight independent coalesced loads
-// per lane before it is accumulated.
+// holds pair s) and broadcast by shuffles. The row is processed in slabs of 64
+// sixteen-byte chunks (lane l holds chunks l and l + 32): the loads of all k
+// rows of a slab (and of the residual) are issued before any is accumulated,
+// so a warp keeps up to 9 KB in flight.
 constexpr int kCombineWarps = 4;
+constexpr int kSlab = 64;
 
-__global__ void __launch_bounds__(32 * kCombineWarps) combine_kernel(
+template <bool RES>
+__global__ void __launch_bounds__(32 * kCombineWarps, RES ? 3 : 4) combine_kernel(
     const uint4* __restrict__ o, const int32_t* __restrict__ k, const int32_t* __restrict__ pair_pos,
     const float* __restrict__ gates, const uint4* residual, int64_t T, int d8, int K, uint4* y) {
   const int lane = threadIdx.x & 31;
@@ -282,27 +284,36 @@ __global__ void __launch_bounds__(32 * kCombineWarps) combine_kernel(
     const int kt = min(k[t], K);
     const int my_pos = lane < kt ? static_cast<int>(min_of<int64_t>(max(pair_pos[t * K + lane], 0), cap - 1)) : 0;
     const float my_g = lane < kt ? gates[t * K + lane] : 0.0f;
-    for (int slab = 0; slab < d8; slab += 256) {
-      float acc[8][8];
+    for (int slab = 0; slab < d8; slab += kSlab) {
+      uint4 v[8][2];
 #pragma unroll
-      for (int c = 0; c < 8; ++c)
+      for (int s = 0; s < 8; ++s) {
+        const int p = __shfl_sync(0xffffffffu, my_pos, s);
+        const uint4* row = o + static_cast<int64_t>(p) * d8;
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          const int ci = slab + lane + 32 * c;
+          v[s][c] = (s < kt && ci < d8) ? __ldcs(row + ci) : make_uint4(0, 0, 0, 0);
+        }
+      }
+      uint4 rv[2];
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        const int ci = slab + lane + 32 * c;
+        rv[c] = (RES && ci < d8) ? __ldcs(residual + t * d8 + ci) : make_uint4(0, 0, 0, 0);
+      }
+      float acc[2][8];
+#pragma unroll
+      for (int c = 0; c < 2; ++c)
 #pragma unroll
         for (int u = 0; u < 8; ++u) acc[c][u] = 0.0f;
 #pragma unroll
       for (int s = 0; s < 8; ++s) {
-        const int p = __shfl_sync(0xffffffffu, my_pos, s);
         const float g = __shfl_sync(0xffffffffu, my_g, s);
         if (s < kt) {
-          const uint4* row = o + static_cast<int64_t>(p) * d8 + slab;
-          uint4 v[8];
 #pragma unroll
-          for (int c = 0; c < 8; ++c) {
-            const int ci = slab + lane + 32 * c;
-            v[c] = ci < d8 ? row[lane + 32 * c] : make_uint4(0, 0, 0, 0);
-          }
-#pragma unroll
-          for (int c = 0; c < 8; ++c) {
-            const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v[c]);
+          for (int c = 0; c < 2; ++c) {
+            const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v[s][c]);
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
               const float2 f = __bfloat1622float2(h[u]);
@@ -313,12 +324,11 @@ __global__ void __launch_bounds__(32 * kCombineWarps) combine_kernel(
         }
       }
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
+      for (int c = 0; c < 2; ++c) {
         const int ci = slab + lane + 32 * c;
         if (ci >= d8) continue;
-        if (residual) {
-          const uint4 v = residual[t * d8 + ci];
-          const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+        if constexpr (RES) {
+          const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&rv[c]);
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
             const float2 f = __bfloat1622float2(h[u]);
@@ -417,7 +427,8 @@ cudaError_t launch_combine(const uint16_t* o, const int32_t* k, const int32_t* p
   int64_t blocks = (T + disp::kCombineWarps - 1) / disp::kCombineWarps;
   const int64_t cap = static_cast<int64_t>(num_sms) * 16;
   if (blocks > cap) blocks = cap;
-  disp::combine_kernel<<<static_cast<unsigned>(blocks), 32 * disp::kCombineWarps, 0, stream>>>(
+  auto kern = residual ? disp::combine_kernel<true> : disp::combine_kernel<false>;
+  kern<<<static_cast<unsigned>(blocks), 32 * disp::kCombineWarps, 0, stream>>>(
       reinterpret_cast<const uint4*>(o), k, pair_pos, gates,
       reinterpret_cast<const uint4*>(residual), T, d / 8, K, reinterpret_cast<uint4*>(y));
   return cudaGetLastError();

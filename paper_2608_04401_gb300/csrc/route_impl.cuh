@@ -289,12 +289,46 @@ MOE_DEV void write_outputs(int64_t t, int K, int k, const int (&ids)[8], const f
 // Exact full path for one token, from the row of e values in shared memory
 // and r = 1/s: every probability sorted, the elbow evaluated on every rank,
 // the top-K ids from a threshold scan. Writes the token's outputs.
-template <int N, typename RC>
-__device__ __noinline__ int route_full(const float* row, float r, int K, float eps, int topk_mode,
-                                        int renorm, const RC& rc, uint64_t* keys,
-                                        int tid, int64_t t, int32_t* k_out, int32_t* ids_out,
-                                        float* gates_out) {
-  float v[N];
+// Softmax numerators of one token: e_j = EXP(l_j - m) for the N logits in
+// row, written back into the row; the smallest e_j in emin; returns r = 1/s
+// with s the balanced tree sum of the e_j.
+template <int N>
+MOE_DEV float softmax_row(float* row, float& emin) {
+  uint64_t ep[N / 2];
+  {
+    float l[N];
+#pragma unroll
+    for (int c = 0; c < N; c += 4) {
+      const float4 q = *reinterpret_cast<const float4*>(row + c);
+      l[c] = q.x; l[c + 1] = q.y; l[c + 2] = q.z; l[c + 3] = q.w;
+    }
+    // four interleaved 3-input max chains over l[4 ..), two elements per step
+    float acc[4] = {l[0], l[1], l[2], l[3]};
+#pragma unroll
+    for (int j = 4; j < N; j += 2) acc[(j / 2) % 4] = max3f(acc[(j / 2) % 4], l[j], l[j + 1]);
+    const float m = fmaxf(max3f(acc[0], acc[1], acc[2]), acc[3]);
+    const uint64_t mm = pk(m, m);
+#pragma unroll
+    for (int a = 0; a < N / 2; ++a) ep[a] = exp_spec2(sub2(pk(l[2 * a], l[2 * a + 1]), mm));
+  }
+#pragma unroll
+  for (int c = 0; c < N; c += 4)
+    *reinterpret_cast<float4*>(row + c) =
+        make_float4(lo_of(ep[c / 2]), hi_of(ep[c / 2]), lo_of(ep[c / 2 + 1]), hi_of(ep[c / 2 + 1]));
+  {
+    // four interleaved 3-input min chains over the pairs ep[2 ..)
+    float acc[4] = {lo_of(ep[0]), hi_of(ep[0]), lo_of(ep[1]), hi_of(ep[1])};
+#pragma unroll
+    for (int a = 2; a < N / 2; ++a) acc[a % 4] = min3f(acc[a % 4], lo_of(ep[a]), hi_of(ep[a]));
+    emin = fminf(min3f(acc[0], acc[1], acc[2]), acc[3]);
+  }
+  tree_sum_level2<N / 2>(ep);
+  return __frcp_rn(__fadd_rn(lo_of(ep[0]), hi_of(ep[0])));
+}
+
+// v = all N probabilities p_j = e_j * r (row holds the e_j), sorted descending.
+template <int N>
+MOE_DEV void sorted_probs(const float* row, float r, float (&v)[N]) {
 #pragma unroll
   for (int c = 0; c < N; c += 4) {
     const float4 q = *reinterpret_cast<const float4*>(row + c);
@@ -302,27 +336,16 @@ __device__ __noinline__ int route_full(const float* row, float r, int K, float e
     v[c + 2] = __fmul_rn(q.z, r); v[c + 3] = __fmul_rn(q.w, r);
   }
   sort_desc_at<N, 0>(v);
+}
 
-  int k = K;
-  if (!topk_mode) {
-    const float p_min = v[N - 1];
-    const float inv = __frcp_rn(__fadd_rn(__fsub_rn(v[0], p_min), eps));
-    float best = -__int_as_float(0x7f800000), tail = -__int_as_float(0x7f800000);
-    int e = 0;
-#pragma unroll
-    for (int i = 0; i < N; ++i) {
-      const float pn = __fmul_rn(__fsub_rn(v[i], p_min), inv);
-      const float D = __fsub_rn(__fsub_rn(1.0f, pn), rc.x[i]);
-      if (i < 7 && i < K - 1) {
-        if (D > best) { best = D; e = i; }
-      } else {
-        tail = fmaxf(tail, D);
-      }
-    }
-    k = (best >= tail) ? e + 1 : K;
-  }
-
-  // p_(K-1) as the minimum of the first K sorted values
+// ids of the K largest probabilities in sorted order (equal probabilities by
+// ascending id), from the sorted values v and a threshold scan of the row:
+// p_(K-1) is the minimum of the first K sorted values; every p above it is
+// taken, and the equal ones in ascending id until K are taken. The (p, id)
+// keys go through this thread's 8-byte slots keys[s * kTok + tid].
+template <int N>
+MOE_DEV void topk_ids(const float* row, float r, const float (&v)[N], int K, uint64_t* keys,
+                      int tid, int (&ids)[8]) {
   float thr = v[0];
 #pragma unroll
   for (int s = 1; s < 8; ++s)
@@ -354,8 +377,39 @@ __device__ __noinline__ int route_full(const float* row, float r, int K, float e
 #pragma unroll
   for (int s = 0; s < 8; ++s) key[s] = (s < K) ? keys[s * kTok + tid] : 0ull;
   sort8_desc(key);
+#pragma unroll
+  for (int s = 0; s < 8; ++s) ids[s] = ~static_cast<int>(key[s]);
+}
+
+template <int N, typename RC>
+__device__ __noinline__ int route_full(const float* row, float r, int K, float eps, int topk_mode,
+                                        int renorm, const RC& rc, uint64_t* keys,
+                                        int tid, int64_t t, int32_t* k_out, int32_t* ids_out,
+                                        float* gates_out) {
+  float v[N];
+  sorted_probs<N>(row, r, v);
+
+  int k = K;
+  if (!topk_mode) {
+    const float p_min = v[N - 1];
+    const float inv = __frcp_rn(__fadd_rn(__fsub_rn(v[0], p_min), eps));
+    float best = -__int_as_float(0x7f800000), tail = -__int_as_float(0x7f800000);
+    int e = 0;
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+      const float pn = __fmul_rn(__fsub_rn(v[i], p_min), inv);
+      const float D = __fsub_rn(__fsub_rn(1.0f, pn), rc.x[i]);
+      if (i < 7 && i < K - 1) {
+        if (D > best) { best = D; e = i; }
+      } else {
+        tail = fmaxf(tail, D);
+      }
+    }
+    k = (best >= tail) ? e + 1 : K;
+  }
 
   int ids[8];
+  topk_ids<N>(row, r, v, K, keys, tid, ids);
   float g[8];
   float S = 0.0f;
 #pragma unroll
@@ -363,7 +417,6 @@ __device__ __noinline__ int route_full(const float* row, float r, int K, float e
     if (s < k) S = __fadd_rn(S, v[s]);
 #pragma unroll
   for (int s = 0; s < 8; ++s) {
-    ids[s] = ~static_cast<int>(key[s]);
     const float p = renorm ? __fdiv_rn(v[s], S) : v[s];
     g[s] = (s < k) ? p : 0.0f;
   }
@@ -386,37 +439,8 @@ MOE_DEV int route_token(float* row, int64_t t, int tid, int K, float eps, int to
   constexpr uint32_t kIdMask = N - 1;
 
   // ---- e_j = EXP(l_j - m), stored back into the row; e_min; s; r = 1/s
-  uint64_t ep[N / 2];
   float emin;
-  {
-    float l[N];
-#pragma unroll
-    for (int c = 0; c < N; c += 4) {
-      const float4 q = *reinterpret_cast<const float4*>(row + c);
-      l[c] = q.x; l[c + 1] = q.y; l[c + 2] = q.z; l[c + 3] = q.w;
-    }
-    // four interleaved 3-input max chains over l[4 ..), two elements per step
-    float acc[4] = {l[0], l[1], l[2], l[3]};
-#pragma unroll
-    for (int j = 4; j < N; j += 2) acc[(j / 2) % 4] = max3f(acc[(j / 2) % 4], l[j], l[j + 1]);
-    const float m = fmaxf(max3f(acc[0], acc[1], acc[2]), acc[3]);
-    const uint64_t mm = pk(m, m);
-#pragma unroll
-    for (int a = 0; a < N / 2; ++a) ep[a] = exp_spec2(sub2(pk(l[2 * a], l[2 * a + 1]), mm));
-  }
-#pragma unroll
-  for (int c = 0; c < N; c += 4)
-    *reinterpret_cast<float4*>(row + c) =
-        make_float4(lo_of(ep[c / 2]), hi_of(ep[c / 2]), lo_of(ep[c / 2 + 1]), hi_of(ep[c / 2 + 1]));
-  {
-    // four interleaved 3-input min chains over the pairs ep[2 ..)
-    float acc[4] = {lo_of(ep[0]), hi_of(ep[0]), lo_of(ep[1]), hi_of(ep[1])};
-#pragma unroll
-    for (int a = 2; a < N / 2; ++a) acc[a % 4] = min3f(acc[a % 4], lo_of(ep[a]), hi_of(ep[a]));
-    emin = fminf(min3f(acc[0], acc[1], acc[2]), acc[3]);
-  }
-  tree_sum_level2<N / 2>(ep);
-  const float r = __frcp_rn(__fadd_rn(lo_of(ep[0]), hi_of(ep[0])));
+  const float r = softmax_row<N>(row, emin);
 
   // ---- the kTop largest e, each key = truncated value | (N-1 - id)
   uint32_t key[N];

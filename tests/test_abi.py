@@ -88,3 +88,12 @@ def test_layer_validation(lib):
     assert lib.moe_layer_forward(*args(wsb=ws - 1)) == 3
     assert lib.moe_layer_forward(*args(rp=_rp(renorm=2))) == 1
     assert lib.moe_layer_workspace_size(64, 2048, 63, 1024, 8) == 0
+
+
+def test_diagnostics_validation(lib):
+    fake = ctypes.c_void_p(256)
+    assert lib.moe_route_diagnostics(fake, 10, 64, _rp(), None, None, None, None) == 1
+    assert lib.moe_route_diagnostics(fake, 10, 64, _rp(), None, None, ctypes.c_void_p(260), None) == 1
+    assert lib.moe_route_diagnostics(fake, 10, 96, _rp(), None, None, fake, None) == 2
+    assert ctypes.sizeof(moe.RouteDiag) == 8 * (2 + 9 + 128 + 181 + 128 + 128) + 8 * 9
+
