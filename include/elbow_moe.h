@@ -247,8 +247,8 @@ moe_status moe_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_
                        uint16_t* y, void* stream);
 
 /*
- * moe_route_diagnostics - routing diagnostics of Sec. 3.1 (elbow angle),
- * Sec. 4.3 and App. A.3 (expert-load changes of elbow-K against top-K).
+ * moe_route_diagnostics - routing diagnostics of Sec. 2.3 (elbow angle),
+ * Sec. 2.4 and App. A.3 (expert-load changes of elbow-K against top-K).
  *
  * Per token, the whole sorted curve is evaluated with the fp32 steps of
  * elbow_route; e is the UNCAPPED elbow index (first argmax of D over all N
@@ -268,7 +268,7 @@ moe_status moe_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_
  *              Theorem 1), the change of the largest share (Corollary 1, same
  *              bound), the change of CV^2 = N |q|^2 - 1 (bound
  *              2 N delta / (1 - delta)^2, Corollary 2), and the percentage
- *              changes of the top-1 share and of CV (Sec. 4.3).
+ *              changes of the top-1 share and of CV (Sec. 2.4).
  * Integer counts make every field independent of block order. Errors as
  * elbow_route; diag NULL or misaligned: MOE_ERR_INVALID_ARG.
  */

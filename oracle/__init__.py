@@ -11,8 +11,9 @@ Functions and the passages they follow:
   router_logits  l(x) = W_r x of Sec. 2, fp64 accumulation rounded to fp32
   layer_rows     the whole MoE layer forward (App. A.4) for chosen tokens, fp64
   load_balance   L_i, q_i, delta and the bounds of Theorem 1 / Corollaries 1-2
-                 (App. A.3), the percentage changes of Sec. 4.3
-  elbow_angle    the uncapped elbow index and the elbow angle of Sec. 3.1
+                 (App. A.3), the percentage changes of Sec. 2.4
+  elbow_angle    the uncapped elbow index and the elbow angle of Sec. 2.3
+  route_randomized  the tail / head randomisation experiment of Sec. 2.2
   exp / exp_max_ulp  the fp32 routing exponential and its error sweep
 The readings taken where the paper is silent or garbled are listed in the
 header of elbow_oracle.c.
@@ -63,6 +64,8 @@ def _load():
         lib.oracle_exp_max_ulp.restype = ctypes.c_double
         lib.oracle_route.argtypes = [P, i64, i32, i32, f32, i32, i32, P, P, P, P, P]
         lib.oracle_route.restype = i32
+        lib.oracle_route_randomized.argtypes = [P, i64, i32, i32, f32, i32, i32, P, P, P, P]
+        lib.oracle_route_randomized.restype = i32
         lib.oracle_elbow_angle.argtypes = [P, i64, i32, f32, P, P]
         lib.oracle_elbow_angle.restype = i32
         lib.oracle_angle_deg.argtypes = [i32, i32, f32]
@@ -182,9 +185,31 @@ def layer_rows(x_bits, w_router_bits, w_gate_up_bits, w_down_bits, rows=None, K:
     return dict(y=y, logits=lg, k=k, ids=ids, gates=gates)
 
 
+MODE_RAND_TAIL = 2
+MODE_RAND_HEAD = 3
+
+
+def route_randomized(logits, rand, K: int = 8, eps: float = 1e-8, mode: int = MODE_RAND_TAIL,
+                     renorm: int = 0):
+    """Tail (mode 2) or head (mode 3) randomisation of Sec. 2.2 with the uint32
+    random numbers rand [T, K]. Returns dict(k, ids, gates)."""
+    lib = _load()
+    lg = _c(logits, np.float32)
+    rnd = _c(rand, np.uint32)
+    T, N = lg.shape
+    assert rnd.shape == (T, K)
+    k = np.empty(T, np.int32)
+    ids = np.empty((T, K), np.int32)
+    gates = np.empty((T, K), np.float32)
+    if lib.oracle_route_randomized(_ptr(lg), T, N, K, eps, mode, renorm, _ptr(rnd), _ptr(k),
+                                   _ptr(ids), _ptr(gates)) != 0:
+        raise ValueError("oracle_route_randomized: unsupported arguments")
+    return dict(k=k, ids=ids, gates=gates)
+
+
 def elbow_angle(logits, eps: float = 1e-8):
     """Per token of fp32 logits [T, N]: the uncapped elbow index (argmax of D
-    over all ranks) and the elbow angle in degrees (Sec. 3.1, reading R11)."""
+    over all ranks) and the elbow angle in degrees (Sec. 2.3, reading R11)."""
     lib = _load()
     lg = _c(logits, np.float32)
     T, N = lg.shape
@@ -230,7 +255,7 @@ def load_balance(k_elb, ids, N: int):
         max_change=abs(q_elb.max() - q_top.max()),
         cv2_change=abs(cv2(q_elb) - cv2(q_top)),
         cv2_bound=2 * N * delta / (1 - delta) ** 2,
-        # the percentages of Sec. 4.3
+        # the percentages of Sec. 2.4
         top1_share_change_pct=(q_top.max() - q_elb.max()) / q_top.max() * 100.0,
         cv_change_pct=(cv_top - cv_elb) / cv_top * 100.0 if cv_top > 0 else 0.0,
     )

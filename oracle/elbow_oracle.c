@@ -41,11 +41,15 @@
  *         D_i = (1 - p'_i) - x'_i.
  *   R7  Expert MLP: SwiGLU, y_e = W_down (silu(W_gate x) * (W_up x)),
  *       silu(z) = z / (1 + exp(-z)), evaluated in fp64 on the bf16 inputs.
- *
- *   R11 Elbow angle (Sec. 3.1): the printed points (0,0), (x'_e, p'_e), (1,1)
+ *   R11 Elbow angle (Sec. 2.3): the printed points (0,0), (x'_e, p'_e), (1,1)
  *       are read on the curve y' = 1 - p' that R1's chord uses (p' itself
  *       runs from (0,1) to (1,0)); theta is evaluated in fp64 from the fp32
  *       x'_e and p'_e, and is 180 degrees when the elbow is an end point.
+ *   R12 Tail randomisation (Sec. 2.2): "experts of rank >= k" are drawn
+ *       without replacement from the remaining experts in ascending id order,
+ *       with caller-supplied uint32 random numbers; the head variant draws
+ *       from ranks >= K so that the K slots stay distinct (see
+ *       oracle_route_randomized).
  *
  * EXP, the routing exponential (written for this project from Cody & Waite's
  * argument reduction, 1980, and the Taylor series of exp):
@@ -135,7 +139,7 @@ double oracle_exp_max_ulp(float lo, float hi, float* worst_z) {
 /* Algorithm 1 plus capped selection for one token. Returns k. */
 static int route_one(const float* l, int N, int K, float eps, int mode, int renorm,
                      int32_t* ids, float* gates, float* sorted_p, int32_t* elbow_e,
-                     float* elbow_pn) {
+                     float* elbow_pn, float* p_out) {
   float e[ORACLE_MAX_N], p[ORACLE_MAX_N], v[ORACLE_MAX_N];
   int idx[ORACLE_MAX_N];
 
@@ -149,6 +153,8 @@ static int route_one(const float* l, int N, int K, float eps, int mode, int reno
     for (int i = 0; i < h; ++i) v[i] = v[i] + v[i + h];
   float r = 1.0f / v[0];
   for (int j = 0; j < N; ++j) p[j] = e[j] * r;
+  if (p_out)
+    for (int j = 0; j < N; ++j) p_out[j] = p[j];
 
   /* p <- sort_desc(p): stable insertion sort of expert ids (R3) */
   for (int j = 0; j < N; ++j) idx[j] = j;
@@ -209,12 +215,12 @@ int oracle_route(const float* logits, int64_t T, int N, int K, float eps, int mo
   for (int64_t t = 0; t < T; ++t) {
     k_out[t] = route_one(logits + t * N, N, K, eps, mode, renorm, ids_out + t * K,
                          gates_out + t * K, sorted_p_out ? sorted_p_out + t * N : NULL,
-                         elbow_out ? elbow_out + t : NULL, NULL);
+                         elbow_out ? elbow_out + t : NULL, NULL, NULL);
   }
   return 0;
 }
 
-/* Elbow angle (Sec. 3.1): the angle at the elbow point between the first and
+/* Elbow angle (Sec. 2.3): the angle at the elbow point between the first and
  * the last point of the normalised curve. With the deviation read as below
  * the chord (R1), the normalised curve is (x'_i, y'_i) = (i/(N-1), 1 - p'_i),
  * from (0,0) to (1,1); at the elbow e, v1 = (0,0) - (x'_e, y'_e) and
@@ -246,9 +252,65 @@ int oracle_elbow_angle(const float* logits, int64_t T, int N, float eps, int32_t
   for (int64_t t = 0; t < T; ++t) {
     int32_t id1, e;
     float g1, pn;
-    route_one(logits + t * N, N, 1, eps, 0, 0, &id1, &g1, NULL, &e, &pn);
+    route_one(logits + t * N, N, 1, eps, 0, 0, &id1, &g1, NULL, &e, &pn, NULL);
     elbow_out[t] = e;
     theta_out[t] = (float)oracle_angle_deg(e, N, pn);
+  }
+  return 0;
+}
+
+/* Tail randomisation (Sec. 2.2): the experiment that keeps K experts
+ * but replaces part of the elbow-K selection by random experts.
+ *   mode 2 (tail): slots s < k keep ranks 0..k-1; each slot s in [k, K) gets
+ *     an expert drawn without replacement from those outside ranks 0..k-1
+ *     (i.e. of rank >= k);
+ *   mode 3 (head): slots s in [k, K) keep ranks k..K-1; each slot s < k gets
+ *     an expert drawn without replacement from those of rank >= K (outside the
+ *     top-K, so that the K experts stay distinct).
+ * Draw (R12): the candidates are the remaining experts in ascending id order;
+ * slot s takes the one at index rand[s] mod (number remaining), which is then
+ * removed. rand [T, K] uint32 is an input. k_out = K (all K slots are used);
+ * gates[s] = p of the expert in slot s, or with renorm its share of the sum
+ * over the K slots, left to right. */
+int oracle_route_randomized(const float* logits, int64_t T, int N, int K, float eps, int mode,
+                            int renorm, const uint32_t* rand, int32_t* k_out, int32_t* ids_out,
+                            float* gates_out) {
+  if (N < 2 || N > ORACLE_MAX_N || (N & (N - 1)) != 0 || K < 1 || K > N || T < 0) return -1;
+  if (mode != 2 && mode != 3) return -1;
+  if (N - K < K) return -1; /* mode 3 needs k <= N - K candidates */
+#pragma omp parallel for schedule(static)
+  for (int64_t t = 0; t < T; ++t) {
+    int32_t ids[ORACLE_MAX_N];
+    float gates[ORACLE_MAX_N], p[ORACLE_MAX_N];
+    int taken[ORACLE_MAX_N];
+    int k = route_one(logits + t * N, N, K, eps, 0, 0, ids, gates, NULL, NULL, NULL, p);
+    for (int j = 0; j < N; ++j) taken[j] = 0;
+    int lo = (mode == 2) ? k : 0, hi = (mode == 2) ? K : k;
+    int excl = (mode == 2) ? k : K; /* ranks 0..excl-1 are not candidates */
+    for (int s = 0; s < excl; ++s) taken[ids[s]] = 1;
+    int remaining = N - excl;
+    for (int s = lo; s < hi; ++s) {
+      uint32_t idx = rand[t * K + s] % (uint32_t)remaining;
+      int pick = -1;
+      for (int j = 0, c = 0; j < N; ++j) {
+        if (taken[j]) continue;
+        if ((uint32_t)c == idx) {
+          pick = j;
+          break;
+        }
+        ++c;
+      }
+      taken[pick] = 1;
+      ids[s] = pick;
+      --remaining;
+    }
+    float S = 0.0f;
+    for (int s = 0; s < K; ++s) S = S + p[ids[s]];
+    k_out[t] = K;
+    for (int s = 0; s < K; ++s) {
+      ids_out[t * K + s] = ids[s];
+      gates_out[t * K + s] = renorm ? p[ids[s]] / S : p[ids[s]];
+    }
   }
   return 0;
 }
@@ -367,7 +429,7 @@ int oracle_layer_rows(const uint16_t* x, const uint16_t* w_router, const uint16_
       for (int c = 0; c < d; ++c) acc += xd[c] * bf16_to_double(w_router[(int64_t)j * d + c]);
       l[j] = (float)acc;
     }
-    int k = route_one(l, N, K, eps, mode, renorm, ids, gates, NULL, NULL, NULL);
+    int k = route_one(l, N, K, eps, mode, renorm, ids, gates, NULL, NULL, NULL, NULL);
     double* yr = y + r * d;
     for (int c = 0; c < d; ++c) yr[c] = 0.0;
     for (int s = 0; s < k; ++s) {

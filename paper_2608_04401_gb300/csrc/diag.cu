@@ -1,4 +1,4 @@
-// Routing diagnostics (Sec. 3.1 elbow angle; Sec. 4.3 and App. A.3 load
+// Routing diagnostics (Sec. 2.3 elbow angle; Sec. 2.4 and App. A.3 load
 // metrics): one thread per token evaluates the whole sorted curve exactly (the
 // same fp32 steps as the routing), finds the uncapped elbow index e (first
 // argmax of D over all N ranks) and the elbow angle, and counts into integer

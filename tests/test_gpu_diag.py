@@ -1,8 +1,8 @@
 """GPU parity of the routing diagnostics (moe_route_diagnostics) against the
-oracle: the uncapped elbow index bit-exact, the elbow angle of Sec. 3.1
+oracle: the uncapped elbow index bit-exact, the elbow angle of Sec. 2.3
 within 1e-4 degrees (fp64 arccos on both sides, rounded to fp32), the
 histograms and per-expert loads exact, and the load-change quantities of
-Sec. 4.3 / App. A.3 within 1e-12."""
+Sec. 2.4 / App. A.3 within 1e-12."""
 import numpy as np
 import pytest
 

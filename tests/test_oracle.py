@@ -258,7 +258,7 @@ def test_load_balance_hand_example():
     assert abs(lb["cv_change_pct"] - want) < 1e-12
 
 
-# ------------------------------------------------------ elbow angle (Sec. 3.1)
+# ------------------------------------------------------ elbow angle (Sec. 2.3)
 @pytest.mark.parametrize("N", [64, 128])
 def test_elbow_angle_step_curves(N):
     """A step of m equal high values has its elbow at e = m with p'_e = 0, so
@@ -430,3 +430,87 @@ def test_synthetic_tokens_have_elbows():
     lg = oracle.router_logits(inp["x"], inp["w_router"])
     r = oracle.route(lg, K=8)
     assert 3.0 < r["k"].mean() < 8.0
+
+
+# ------------------------------------------- tail randomisation (Sec. 2.2)
+def _p_by_id(lg):
+    """Every expert's probability, read off a full top-N routing (N slots)."""
+    T, N = lg.shape
+    r = oracle.route(lg, K=N, mode=oracle.MODE_TOPK)
+    p = np.empty((T, N), np.float32)
+    np.put_along_axis(p, r["ids"], r["gates"], axis=1)
+    return p
+
+
+@pytest.mark.parametrize("N", [64, 128])
+def test_randomized_tail_invariants(N):
+    rng = np.random.default_rng(N + 21)
+    T, K = 3000, 8
+    lg = synth.boosted_logits(rng, T, N)
+    rnd = rng.integers(0, 2**32, size=(T, K), dtype=np.uint32)
+    base = oracle.route(lg, K=K)
+    p = _p_by_id(lg)
+    for mode in (oracle.MODE_RAND_TAIL, oracle.MODE_RAND_HEAD):
+        r = oracle.route_randomized(lg, rnd, K=K, mode=mode)
+        assert np.all(r["k"] == K)
+        for t in range(T):
+            k, ids, top = base["k"][t], r["ids"][t], base["ids"][t]
+            assert len(set(ids.tolist())) == K
+            if mode == oracle.MODE_RAND_TAIL:
+                assert np.array_equal(ids[:k], top[:k])          # the head is kept
+                assert not set(ids[k:]) & set(top[:k])           # tail picks have rank >= k
+            else:
+                assert np.array_equal(ids[k:], top[k:])          # ranks k..K-1 are kept
+                assert not set(ids[:k]) & set(top)               # head picks have rank >= K
+            assert np.array_equal(r["gates"][t], p[t, ids])      # gate = the expert's own p
+
+
+def test_randomized_zero_draws_take_smallest_ids():
+    """rand = 0 selects, slot after slot, the smallest remaining id."""
+    N, K = 64, 8
+    lg = np.zeros((1, N), np.float32)
+    lg[0, [40, 50, 60]] = 6.0                     # head of 3: ranks 0..2 = 40, 50, 60; k = 4
+    base = oracle.route(lg, K=K)
+    k = int(base["k"][0])
+    assert k == 4
+    r = oracle.route_randomized(lg, np.zeros((1, K), np.uint32), K=K, mode=oracle.MODE_RAND_TAIL)
+    # rank 3 is expert 0 (ties by ascending id); the tail draws the smallest ids outside the head
+    assert r["ids"][0].tolist() == base["ids"][0, :k].tolist() + [1, 2, 3, 4]
+    r = oracle.route_randomized(lg, np.zeros((1, K), np.uint32), K=K, mode=oracle.MODE_RAND_HEAD)
+    top = set(base["ids"][0].tolist())
+    first = [j for j in range(N) if j not in top][:k]
+    assert r["ids"][0, :k].tolist() == first and r["ids"][0, k:].tolist() == base["ids"][0, k:].tolist()
+
+
+def test_randomized_draw_is_uniform():
+    """One token repeated: the first tail draw is uniform over the N - k experts
+    of rank >= k (chi-square, 60 cells, far inside the 1e-6 tail)."""
+    N, K, T = 64, 8, 60000
+    row = np.zeros(N, np.float32)
+    row[[5, 9, 33]] = 6.0
+    lg = np.tile(row, (T, 1))
+    rnd = np.random.default_rng(7).integers(0, 2**32, size=(T, K), dtype=np.uint32)
+    r = oracle.route_randomized(lg, rnd, K=K, mode=oracle.MODE_RAND_TAIL)
+    k = int(oracle.route(lg[:1], K=K)["k"][0])
+    first = r["ids"][:, k]
+    cnt = np.bincount(first, minlength=N)
+    head = oracle.route(lg[:1], K=K)["ids"][0, :k]
+    assert np.all(cnt[head] == 0)
+    cells = np.delete(cnt, head)
+    exp_c = T / (N - k)
+    chi2 = float(((cells - exp_c) ** 2 / exp_c).sum())
+    assert chi2 < 130.0, chi2      # dof = N - k - 1 = 59; P(chi2 > 130) < 1e-6
+
+
+def test_randomized_renorm_and_full_head():
+    rng = np.random.default_rng(3)
+    lg = synth.boosted_logits(rng, 500, 64)
+    rnd = rng.integers(0, 2**32, size=(500, 8), dtype=np.uint32)
+    r = oracle.route_randomized(lg, rnd, mode=oracle.MODE_RAND_TAIL, renorm=1)
+    np.testing.assert_allclose(r["gates"].astype(np.float64).sum(1), 1.0, atol=1e-6)
+    base = oracle.route(lg, K=8, mode=oracle.MODE_TOPK)
+    k = oracle.route(lg, K=8)["k"]
+    full = k == 8                              # no tail: nothing to randomise
+    r0 = oracle.route_randomized(lg, rnd, mode=oracle.MODE_RAND_TAIL)
+    assert np.array_equal(r0["ids"][full], base["ids"][full])
+    assert np.array_equal(r0["gates"][full], base["gates"][full])
