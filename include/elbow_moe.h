@@ -45,7 +45,12 @@ typedef enum {
   MOE_ERR_DEVICE_TIMEOUT = 5  /* a kernel gave up a bounded wait (see moe_read_device_error) */
 } moe_status;
 
-typedef enum { MOE_ROUTE_ELBOW = 0, MOE_ROUTE_TOPK = 1 } moe_route_mode;
+typedef enum {
+  MOE_ROUTE_ELBOW = 0,
+  MOE_ROUTE_TOPK = 1,
+  MOE_ROUTE_RAND_TAIL = 2,  /* elbow_route_randomized only */
+  MOE_ROUTE_RAND_HEAD = 3   /* elbow_route_randomized only */
+} moe_route_mode;
 
 /* Routing parameters. K: the cap (top-K of the base router, Sec. 2.1).
  * eps: the epsilon of Alg. 1's normalisation (the paper leaves it unstated;
@@ -245,6 +250,31 @@ moe_status moe_gather_rows(const uint16_t* x, const int32_t* perm, const int32_t
 moe_status moe_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_pos,
                        const float* gates, const uint16_t* residual, int64_t T, int d, int K,
                        uint16_t* y, void* stream);
+
+/*
+ * elbow_route_randomized - the tail-randomisation experiment of Sec. 2.2,
+ * which keeps K experts per token but replaces part of the elbow-K selection
+ * by random experts:
+ *   rp->mode MOE_ROUTE_RAND_TAIL: slots s < k keep ranks 0..k-1 (k the elbow
+ *     count of elbow_route); each slot s in [k, K) gets an expert drawn
+ *     without replacement from those of rank >= k;
+ *   rp->mode MOE_ROUTE_RAND_HEAD: slots s in [k, K) keep ranks k..K-1; each
+ *     slot s < k gets an expert drawn without replacement from those of
+ *     rank >= K.
+ *   rand      [T, K] uint32   caller's random numbers; slot s of token t takes,
+ *                             among the remaining experts in ascending id
+ *                             order, the one at index rand[t, s] mod (number
+ *                             remaining); slots that keep their rank ignore it
+ *   k_out     [T]             K (every slot is used)
+ *   ids_out, gates_out [T, K] the K experts and their own probabilities p
+ *                             (renorm: divided by the sum over the K slots)
+ * Routing arithmetic as elbow_route. Errors as elbow_route; rand NULL or a
+ * mode other than the two above: MOE_ERR_INVALID_ARG. Pointers 4-byte
+ * aligned (logits 16-byte).
+ */
+moe_status elbow_route_randomized(const float* logits, int64_t T, int N, const moe_route_params* rp,
+                                  const uint32_t* rand, int32_t* k_out, int32_t* ids_out,
+                                  float* gates_out, void* stream);
 
 /*
  * moe_route_diagnostics - routing diagnostics of Sec. 2.3 (elbow angle),

@@ -19,6 +19,7 @@ import numpy as np
 
 __all__ = [
     "MODE_ELBOW", "MODE_TOPK", "MoeError", "library", "build", "route_diagnostics", "RouteDiag",
+    "elbow_route_randomized", "MODE_RAND_TAIL", "MODE_RAND_HEAD",
     "elbow_route", "moe_dispatch", "moe_dispatch_noalloc", "dispatch_workspace_size", "layer_workspace_size",
     "moe_layer_forward", "read_device_error", "router_logits", "gather_rows",
     "expert_gate_up", "expert_down", "combine",
@@ -80,6 +81,7 @@ def library():
             "elbow_route": ([P, i64, i32, RP, P, P, P, P], i32),
             "elbow_route_with_counts": ([P, i64, i32, RP, P, P, P, P, P], i32),
             "moe_route_diagnostics": ([P, i64, i32, RP, P, P, P, P], i32),
+            "elbow_route_randomized": ([P, i64, i32, RP, P, P, P, P, P], i32),
             "moe_dispatch_workspace_size": ([i64, i32, i32], sz),
             "moe_dispatch": ([P, P, i64, i32, i32, P, P, P, P, sz, P], i32),
             "moe_dispatch_tile_offsets": ([P, i64, i32, i32], P),
@@ -170,6 +172,30 @@ def elbow_route_with_counts(logits, chunk_counts, K: int = 8, eps: float = 1e-8,
     _check(lib.elbow_route_with_counts(_p(logits), T, N, _params(K, eps, mode, renorm), _p(k),
                                        _p(ids), _p(gates), _p(chunk_counts), _stream(stream)),
            "elbow_route_with_counts")
+    return k, ids, gates
+
+
+MODE_RAND_TAIL = 2
+MODE_RAND_HEAD = 3
+
+
+def elbow_route_randomized(logits, rand, K: int = 8, eps: float = 1e-8, mode: int = MODE_RAND_TAIL,
+                           renorm: int = 0, stream=None):
+    """Tail (MODE_RAND_TAIL) or head (MODE_RAND_HEAD) randomisation with the
+    uint32 random numbers rand [T, K] (an int32 tensor holding the bits is
+    accepted too). Returns (k, ids, gates)."""
+    torch = _torch()
+    _cuda(logits, torch.float32, "logits")
+    T, N = logits.shape
+    if rand.dtype not in (torch.int32, getattr(torch, "uint32", torch.int32)) or \
+            tuple(rand.shape) != (T, K) or not rand.is_contiguous() or rand.device != logits.device:
+        raise ValueError(f"rand must be a contiguous [{T}, {K}] 32-bit tensor on {logits.device}")
+    k = torch.empty(T, dtype=torch.int32, device=logits.device)
+    ids = torch.empty(T, K, dtype=torch.int32, device=logits.device)
+    gates = torch.empty(T, K, dtype=torch.float32, device=logits.device)
+    _check(library().elbow_route_randomized(_p(logits), T, N, _params(K, eps, mode, renorm),
+                                            _p(rand), _p(k), _p(ids), _p(gates), _stream(stream)),
+           "elbow_route_randomized")
     return k, ids, gates
 
 

@@ -8,7 +8,8 @@
 namespace moe {
 cudaError_t launch_elbow_route(const float* logits, int64_t T, int N, int K, float eps,
                                int topk_mode, int renorm, int32_t* k_out, int32_t* ids_out,
-                               float* gates_out, int32_t* blk_cnt, cudaStream_t stream);
+                               float* gates_out, int32_t* blk_cnt, const uint32_t* rand,
+                               int rand_mode, cudaStream_t stream);
 size_t dispatch_ws_bytes(int64_t T, int N);
 int32_t* dispatch_tile_off(void* ws, int64_t T, int N);
 int32_t* dispatch_counts(void* ws);
@@ -142,6 +143,28 @@ moe_status elbow_route(const float* logits, int64_t T, int N, const moe_route_pa
     return MOE_ERR_INVALID_ARG;
   return cuda_status(moe::launch_elbow_route(logits, T, N, rp->K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
                                              rp->renorm, k_out, ids_out, gates_out, nullptr,
+                                             nullptr, 0, static_cast<cudaStream_t>(stream)));
+}
+
+moe_status elbow_route_randomized(const float* logits, int64_t T, int N, const moe_route_params* rp,
+                                  const uint32_t* rand, int32_t* k_out, int32_t* ids_out,
+                                  float* gates_out, void* stream) {
+  if (T < 0 || T > kMaxTokens) return MOE_ERR_INVALID_ARG;
+  if (!supported_n(N)) return MOE_ERR_UNSUPPORTED;
+  if (!rp || (rp->mode != MOE_ROUTE_RAND_TAIL && rp->mode != MOE_ROUTE_RAND_HEAD))
+    return MOE_ERR_INVALID_ARG;
+  moe_route_params base = *rp;
+  base.mode = MOE_ROUTE_ELBOW;
+  moe_status st = check_route_params(&base, N);
+  if (st != MOE_OK) return st;
+  if (T == 0) return MOE_OK;
+  if (!logits || !rand || !k_out || !ids_out || !gates_out) return MOE_ERR_INVALID_ARG;
+  if (!aligned16(logits) || (reinterpret_cast<uintptr_t>(rand) & 3u) ||
+      (reinterpret_cast<uintptr_t>(k_out) & 3u) || (reinterpret_cast<uintptr_t>(ids_out) & 3u) ||
+      (reinterpret_cast<uintptr_t>(gates_out) & 3u))
+    return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_elbow_route(logits, T, N, rp->K, rp->eps, 0, rp->renorm, k_out,
+                                             ids_out, gates_out, nullptr, rand, rp->mode,
                                              static_cast<cudaStream_t>(stream)));
 }
 
@@ -175,7 +198,7 @@ moe_status elbow_route_with_counts(const float* logits, int64_t T, int N,
     return MOE_ERR_INVALID_ARG;
   return cuda_status(moe::launch_elbow_route(logits, T, N, rp->K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
                                              rp->renorm, k_out, ids_out, gates_out, chunk_counts,
-                                             static_cast<cudaStream_t>(stream)));
+                                             nullptr, 0, static_cast<cudaStream_t>(stream)));
 }
 
 size_t moe_dispatch_workspace_size(int64_t T, int N, int K) {

@@ -273,7 +273,7 @@ constexpr int kCombineWarps = 4;
 constexpr int kSlab = 64;
 
 template <bool RES>
-__global__ void __launch_bounds__(32 * kCombineWarps, RES ? 3 : 4) combine_kernel(
+__global__ void __launch_bounds__(32 * kCombineWarps, 4) combine_kernel(
     const uint4* __restrict__ o, const int32_t* __restrict__ k, const int32_t* __restrict__ pair_pos,
     const float* __restrict__ gates, const uint4* residual, int64_t T, int d8, int K, uint4* y) {
   const int lane = threadIdx.x & 31;
@@ -284,27 +284,28 @@ __global__ void __launch_bounds__(32 * kCombineWarps, RES ? 3 : 4) combine_kerne
     const int kt = min(k[t], K);
     const int my_pos = lane < kt ? static_cast<int>(min_of<int64_t>(max(pair_pos[t * K + lane], 0), cap - 1)) : 0;
     const float my_g = lane < kt ? gates[t * K + lane] : 0.0f;
-    for (int slab = 0; slab < d8; slab += kSlab) {
-      uint4 v[8][2];
+    constexpr int CH = RES ? 1 : 2;
+    for (int slab = 0; slab < d8; slab += 32 * CH) {
+      uint4 v[8][CH];
 #pragma unroll
       for (int s = 0; s < 8; ++s) {
         const int p = __shfl_sync(0xffffffffu, my_pos, s);
         const uint4* row = o + static_cast<int64_t>(p) * d8;
 #pragma unroll
-        for (int c = 0; c < 2; ++c) {
+        for (int c = 0; c < CH; ++c) {
           const int ci = slab + lane + 32 * c;
           v[s][c] = (s < kt && ci < d8) ? __ldcs(row + ci) : make_uint4(0, 0, 0, 0);
         }
       }
-      uint4 rv[2];
+      uint4 rv[CH];
 #pragma unroll
-      for (int c = 0; c < 2; ++c) {
+      for (int c = 0; c < CH; ++c) {
         const int ci = slab + lane + 32 * c;
         rv[c] = (RES && ci < d8) ? __ldcs(residual + t * d8 + ci) : make_uint4(0, 0, 0, 0);
       }
-      float acc[2][8];
+      float acc[CH][8];
 #pragma unroll
-      for (int c = 0; c < 2; ++c)
+      for (int c = 0; c < CH; ++c)
 #pragma unroll
         for (int u = 0; u < 8; ++u) acc[c][u] = 0.0f;
 #pragma unroll
@@ -312,7 +313,7 @@ __global__ void __launch_bounds__(32 * kCombineWarps, RES ? 3 : 4) combine_kerne
         const float g = __shfl_sync(0xffffffffu, my_g, s);
         if (s < kt) {
 #pragma unroll
-          for (int c = 0; c < 2; ++c) {
+          for (int c = 0; c < CH; ++c) {
             const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v[s][c]);
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
@@ -324,7 +325,7 @@ __global__ void __launch_bounds__(32 * kCombineWarps, RES ? 3 : 4) combine_kerne
         }
       }
 #pragma unroll
-      for (int c = 0; c < 2; ++c) {
+      for (int c = 0; c < CH; ++c) {
         const int ci = slab + lane + 32 * c;
         if (ci >= d8) continue;
         if constexpr (RES) {

@@ -5,15 +5,76 @@
 namespace moe {
 namespace route {
 
+// Tail / head randomisation (Sec. 2.2) of one routed token, in place of its
+// outputs: top[] holds the ids of ranks 0..K-1 and k the elbow count. mode 2
+// keeps ranks 0..k-1 and fills slots k..K-1 with experts of rank >= k; mode 3
+// keeps ranks k..K-1 and fills slots 0..k-1 with experts of rank >= K. Each
+// draw takes, among the remaining experts in ascending id order, the one at
+// index rand[t, s] mod (number remaining). Gates are the experts' own p (the
+// row holds their e, and 1/s is recomputed with the routing's tree order).
+template <int N>
+__device__ __noinline__ void randomize_token(const float* row, int64_t t, int K, int mode,
+                                             int renorm, int k, const int* top,
+                                             const uint32_t* __restrict__ rand,
+                                             int32_t* __restrict__ k_out,
+                                             int32_t* __restrict__ ids_out,
+                                             float* __restrict__ gates_out) {
+  float v[N];
+#pragma unroll
+  for (int j = 0; j < N; ++j) v[j] = row[j];
+#pragma unroll
+  for (int h = N / 2; h >= 1; h /= 2)
+#pragma unroll
+    for (int i = 0; i < h; ++i) v[i] = __fadd_rn(v[i], v[i + h]);
+  const float r = __frcp_rn(v[0]);
+  uint32_t taken[N / 32];
+#pragma unroll
+  for (int w = 0; w < N / 32; ++w) taken[w] = 0u;
+  int ids[8];
+  const int excl = mode == 2 ? k : K;
+  for (int s = 0; s < K; ++s) {
+    ids[s] = top[s];
+    if (s < excl) taken[top[s] / 32] |= 1u << (top[s] % 32);
+  }
+  const int lo = mode == 2 ? k : 0, hi = mode == 2 ? K : k;
+  int remaining = N - excl;
+  for (int s = lo; s < hi; ++s) {
+    uint32_t idx = rand[t * K + s] % static_cast<uint32_t>(remaining);
+    int pick = 0;
+    for (int w = 0; w < N / 32; ++w) {
+      const uint32_t freew = ~taken[w];
+      const uint32_t c = static_cast<uint32_t>(__popc(freew));
+      if (idx < c) {
+        uint32_t f = freew;
+        for (uint32_t i = 0; i < idx; ++i) f &= f - 1u;  // drop the idx lowest free bits
+        pick = w * 32 + __ffs(static_cast<int>(f)) - 1;
+        break;
+      }
+      idx -= c;
+    }
+    taken[pick / 32] |= 1u << (pick % 32);
+    ids[s] = pick;
+    --remaining;
+  }
+  float S = 0.0f;
+  for (int s = 0; s < K; ++s) S = __fadd_rn(S, __fmul_rn(row[ids[s]], r));
+  k_out[t] = K;
+  for (int s = 0; s < K; ++s) {
+    const float p = __fmul_rn(row[ids[s]], r);
+    ids_out[t * K + s] = ids[s];
+    gates_out[t * K + s] = renorm ? __fdiv_rn(p, S) : p;
+  }
+}
+
 // One thread per token; optionally (blk_cnt != nullptr) also the block's
 // per-expert pair counts, written to blk_cnt[e * nblk + blockIdx.x] (the
 // first pass of the dispatch, fused here so that the ids are not re-read).
-template <int N>
+template <int N, bool RAND>
 __global__ void __launch_bounds__(kTok) elbow_route_kernel(
     const float* __restrict__ logits, int64_t T, int K, float eps, int topk_mode, int renorm,
     const __grid_constant__ RouteConsts<N> rc, int32_t* __restrict__ k_out,
     int32_t* __restrict__ ids_out, float* __restrict__ gates_out, int32_t* __restrict__ blk_cnt,
-    int nblk) {
+    int nblk, const uint32_t* __restrict__ rand, int rand_mode) {
   constexpr int kPitch = N + 4;
   extern __shared__ float4 smem4[];
   __shared__ int hist[N];
@@ -38,9 +99,18 @@ __global__ void __launch_bounds__(kTok) elbow_route_kernel(
   __syncthreads();
   int ids_sel[8];
   int k_sel = 0;
-  if (tid < ntok)
+  if (tid < ntok) {
     k_sel = route_token<N, RouteConsts<N>>(tile + tid * kPitch, t0 + tid, tid, K, eps, topk_mode,
                                            renorm, rc, keys64, k_out, ids_out, gates_out, ids_sel);
+    if constexpr (RAND) {
+      randomize_token<N>(tile + tid * kPitch, t0 + tid, K, rand_mode, renorm, k_sel, ids_sel, rand,
+                         k_out, ids_out, gates_out);
+      k_sel = K;
+#pragma unroll
+      for (int s = 0; s < 8; ++s)
+        if (s < K) ids_sel[s] = ids_out[(t0 + tid) * K + s];
+    }
+  }
   if (blk_cnt != nullptr) {
 #pragma unroll
     for (int s = 0; s < 8; ++s)
@@ -53,38 +123,43 @@ __global__ void __launch_bounds__(kTok) elbow_route_kernel(
 template <int N>
 cudaError_t launch(const float* logits, int64_t T, int K, float eps, int topk_mode, int renorm,
                    int32_t* k_out, int32_t* ids_out, float* gates_out, int32_t* blk_cnt,
-                   cudaStream_t stream) {
+                   const uint32_t* rand, int rand_mode, cudaStream_t stream) {
   RouteConsts<N> rc;
   fill_route_consts(rc, N);
   constexpr size_t smem = smem_bytes<N>();
+  auto kern = rand_mode ? elbow_route_kernel<N, true> : elbow_route_kernel<N, false>;
   static int attr_dev = -1;
   int dev = 0;
   cudaGetDevice(&dev);
   if (attr_dev != dev) {
-    cudaError_t e = cudaFuncSetAttribute(elbow_route_kernel<N>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
+    for (auto f : {elbow_route_kernel<N, true>, elbow_route_kernel<N, false>}) {
+      cudaError_t e =
+          cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e != cudaSuccess) return e;
+    }
     attr_dev = dev;
   }
   const int64_t blocks = (T + kTok - 1) / kTok;
-  elbow_route_kernel<N><<<static_cast<unsigned>(blocks), kTok, smem, stream>>>(
+  kern<<<static_cast<unsigned>(blocks), kTok, smem, stream>>>(
       logits, T, K, eps, topk_mode, renorm, rc, k_out, ids_out, gates_out, blk_cnt,
-      static_cast<int>(blocks));
+      static_cast<int>(blocks), rand, rand_mode);
   return cudaGetLastError();
 }
 
 }  // namespace route
 
 // blk_cnt (nullable): per-128-token-chunk expert counts, [N][ceil(T/128)].
+// rand (nullable) and rand_mode (0, or 2 / 3 for the tail / head randomisation).
 cudaError_t launch_elbow_route(const float* logits, int64_t T, int N, int K, float eps,
                                int topk_mode, int renorm, int32_t* k_out, int32_t* ids_out,
-                               float* gates_out, int32_t* blk_cnt, cudaStream_t stream) {
+                               float* gates_out, int32_t* blk_cnt, const uint32_t* rand,
+                               int rand_mode, cudaStream_t stream) {
   if (T == 0) return cudaSuccess;
   if (N == 64)
     return route::launch<64>(logits, T, K, eps, topk_mode, renorm, k_out, ids_out, gates_out,
-                             blk_cnt, stream);
+                             blk_cnt, rand, rand_mode, stream);
   return route::launch<128>(logits, T, K, eps, topk_mode, renorm, k_out, ids_out, gates_out,
-                            blk_cnt, stream);
+                            blk_cnt, rand, rand_mode, stream);
 }
 
 }  // namespace moe

@@ -97,3 +97,13 @@ def test_diagnostics_validation(lib):
     assert lib.moe_route_diagnostics(fake, 10, 96, _rp(), None, None, fake, None) == 2
     assert ctypes.sizeof(moe.RouteDiag) == 8 * (2 + 9 + 128 + 181 + 128 + 128) + 8 * 9
 
+
+def test_randomized_validation(lib):
+    fake = ctypes.c_void_p(256)
+    # modes other than 2 / 3, missing rand
+    assert lib.elbow_route_randomized(fake, 10, 64, _rp(mode=0), fake, fake, fake, fake, None) == 1
+    assert lib.elbow_route_randomized(fake, 10, 64, _rp(mode=2), None, fake, fake, fake, None) == 1
+    assert lib.elbow_route_randomized(fake, 10, 64, _rp(mode=3, K=9), fake, fake, fake, fake, None) == 2
+    # elbow_route itself rejects the randomisation modes
+    assert lib.elbow_route(fake, 10, 64, _rp(mode=2), fake, fake, fake, None) == 1
+
