@@ -265,12 +265,12 @@ __global__ void __launch_bounds__(256) gather_kernel(const uint4* __restrict__ x
 
 // y_t = sum_{s<k_t} g_{t,s} * o[pair_pos[t,s]] (+ residual_t); fp32 in s order.
 // One warp per token. The token's k positions and gates are read once (lane s
-// holds pair s) and broadcast by shuffles. The row is processed in slabs of 64
-// sixteen-byte chunks (lane l holds chunks l and l + 32): the loads of all k
-// rows of a slab (and of the residual) are issued before any is accumulated,
-// so a warp keeps up to 9 KB in flight.
+// holds pair s) and broadcast by shuffles. The row is processed in slabs of
+// 32 * CH sixteen-byte chunks (lane l holds chunks l + 32c, c < CH; CH = 2
+// without a residual, 1 with one, which keeps both variants at four blocks
+// per SM): the loads of all k rows of a slab (and of the residual) are issued
+// before any is accumulated, so a warp keeps up to 8 KB in flight.
 constexpr int kCombineWarps = 4;
-constexpr int kSlab = 64;
 
 template <bool RES>
 __global__ void __launch_bounds__(32 * kCombineWarps, 4) combine_kernel(
