@@ -99,6 +99,8 @@ def library():
             "moe_combine": ([P, P, P, P, P, i64, i32, i32, P, P], i32),
             "moe_router_route": ([P, P, i64, i32, i32, RP, P, P, P, P, P, P, P], i32),
             "moe_expert_gate_up_gathered": ([P, i64, P, P, P, P, i64, i32, i32, i32, P, P, P], i32),
+            "moe_expert_gate_up_decode": ([P, P, P, i64, i64, i32, i32, i32, P, P, P], i32),
+            "moe_expert_down_decode": ([P, P, P, i64, i64, i32, i32, i32, P, P, P], i32),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -391,6 +393,29 @@ def expert_gate_up_gathered(x, perm, w_gate_up, offsets, tile_off, P: int, err=N
                                                  _p(tile_off), P, d, N, I2 // 2, _p(h), _p(err),
                                                  _stream(stream)), "moe_expert_gate_up_gathered")
     return h
+
+
+def expert_gate_up_decode(xs, w_gate_up, offsets, T: int, err=None, stream=None):
+    """Decode-shaped gate/up GEMM (T <= 64): h [P, I] from the dispatched rows xs [P, d]."""
+    torch = _torch()
+    P, d = xs.shape
+    N, I2, _ = w_gate_up.shape
+    h = torch.empty(max(P, 1), I2 // 2, dtype=torch.bfloat16, device=xs.device)
+    _check(library().moe_expert_gate_up_decode(_p(xs), _p(w_gate_up), _p(offsets), T, P, d, N,
+                                               I2 // 2, _p(h), _p(err), _stream(stream)),
+           "moe_expert_gate_up_decode")
+    return h
+
+
+def expert_down_decode(h, w_down, offsets, T: int, err=None, stream=None):
+    """Decode-shaped down GEMM (T <= 64): o [P, d] from h [P, I]."""
+    torch = _torch()
+    P, I = h.shape
+    N, d, _ = w_down.shape
+    o = torch.empty(max(P, 1), d, dtype=torch.bfloat16, device=h.device)
+    _check(library().moe_expert_down_decode(_p(h), _p(w_down), _p(offsets), T, P, d, N, I, _p(o),
+                                            _p(err), _stream(stream)), "moe_expert_down_decode")
+    return o
 
 
 def gather_rows(x, perm, offsets, P: int, stream=None):

@@ -37,6 +37,12 @@ cudaError_t launch_gateup_gather_gemm(const uint16_t* x, int64_t T, const int32_
                                       const uint16_t* wgu, const int32_t* offsets,
                                       const int32_t* tile_off, int64_t P, int d, int N, int I,
                                       uint16_t* h, int32_t* err, int num_sms, cudaStream_t stream);
+cudaError_t launch_gateup_decode_gemm(const uint16_t* xs, const uint16_t* wgu,
+                                      const int32_t* offsets, int64_t P, int d, int N, int I,
+                                      uint16_t* h, int32_t* err, int num_sms, cudaStream_t stream);
+cudaError_t launch_down_decode_gemm(const uint16_t* h, const uint16_t* wd, const int32_t* offsets,
+                                    int64_t P, int d, int N, int I, uint16_t* o, int32_t* err,
+                                    int num_sms, cudaStream_t stream);
 cudaError_t launch_route_diagnostics(const float* logits, int64_t T, int N, int K, float eps,
                                      int32_t* elbow_out, float* theta_out, moe_route_diag* dg,
                                      cudaStream_t stream);
@@ -46,6 +52,9 @@ namespace {
 
 constexpr int64_t kMaxTokens = int64_t(1) << 28;  // keeps T * K * 8 row counts in int32
 constexpr int kMaxDim = 16384;
+// Batches of at most this many tokens take the decode-shaped expert GEMMs
+// (weights as the M operand; every expert then has at most 64 rows).
+constexpr int64_t kDecodeMaxTokens = 64;
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -299,13 +308,24 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   e = moe::launch_dispatch(kk, ids, T, N, K, w.offsets, w.perm, w.pair_pos, w.disp, offsets_out,
                            true, s);
   if (e != cudaSuccess) return MOE_ERR_CUDA;
-  const int32_t* tile_off = moe::dispatch_tile_off(w.disp, T, N);
-  // gate/up GEMM gathers its token rows itself (no dispatched copy of x)
-  e = moe::launch_gateup_gather_gemm(x, T, w.perm, w_gate_up, w.offsets, tile_off, P, d, N, I, w.h,
-                                     w.err, nsm, s);
-  if (e != cudaSuccess) return MOE_ERR_CUDA;
-  e = moe::launch_down_gemm(w.h, w_down, w.offsets, tile_off, P, d, N, I, w.o, w.err, nsm, s);
-  if (e != cudaSuccess) return MOE_ERR_CUDA;
+  if (T <= kDecodeMaxTokens) {
+    // decode-sized: gather the few token rows (into o, which the down GEMM
+    // overwrites afterwards) and stream the weights as the M operand
+    e = moe::launch_gather(x, w.perm, w.offsets, N, P, d, w.o, nsm, s);
+    if (e != cudaSuccess) return MOE_ERR_CUDA;
+    e = moe::launch_gateup_decode_gemm(w.o, w_gate_up, w.offsets, P, d, N, I, w.h, w.err, nsm, s);
+    if (e != cudaSuccess) return MOE_ERR_CUDA;
+    e = moe::launch_down_decode_gemm(w.h, w_down, w.offsets, P, d, N, I, w.o, w.err, nsm, s);
+    if (e != cudaSuccess) return MOE_ERR_CUDA;
+  } else {
+    const int32_t* tile_off = moe::dispatch_tile_off(w.disp, T, N);
+    // gate/up GEMM gathers its token rows itself (no dispatched copy of x)
+    e = moe::launch_gateup_gather_gemm(x, T, w.perm, w_gate_up, w.offsets, tile_off, P, d, N, I,
+                                       w.h, w.err, nsm, s);
+    if (e != cudaSuccess) return MOE_ERR_CUDA;
+    e = moe::launch_down_gemm(w.h, w_down, w.offsets, tile_off, P, d, N, I, w.o, w.err, nsm, s);
+    if (e != cudaSuccess) return MOE_ERR_CUDA;
+  }
   e = moe::launch_combine(w.o, kk, w.pair_pos, gates, residual, T, d, K, y, nsm, s);
   if (e != cudaSuccess) return MOE_ERR_CUDA;
   return MOE_OK;
@@ -359,6 +379,37 @@ moe_status moe_expert_down(const uint16_t* h, const uint16_t* w_down, const int3
     return MOE_ERR_INVALID_ARG;
   return cuda_status(moe::launch_down_gemm(h, w_down, offsets, tile_off, P, d, N, I, o, err_word,
                                            sm_count(), static_cast<cudaStream_t>(stream)));
+}
+
+moe_status moe_expert_gate_up_decode(const uint16_t* xs, const uint16_t* w_gate_up,
+                                     const int32_t* offsets, int64_t T, int64_t P, int d, int N,
+                                     int I, uint16_t* h, int32_t* err_word, void* stream) {
+  if (T < 0 || P < 0 || P > kMaxTokens * 8) return MOE_ERR_INVALID_ARG;
+  if (T > kDecodeMaxTokens) return MOE_ERR_UNSUPPORTED;
+  if (!supported_n(N) || d <= 0 || d > kMaxDim || d % 64 != 0 || I <= 0 || I > kMaxDim ||
+      I % 64 != 0)
+    return MOE_ERR_UNSUPPORTED;
+  if (P == 0 || T == 0) return MOE_OK;
+  if (!xs || !w_gate_up || !offsets || !h || !aligned16(xs) || !aligned16(w_gate_up) ||
+      !aligned16(h))
+    return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_gateup_decode_gemm(xs, w_gate_up, offsets, P, d, N, I, h, err_word,
+                                                    sm_count(), static_cast<cudaStream_t>(stream)));
+}
+
+moe_status moe_expert_down_decode(const uint16_t* h, const uint16_t* w_down, const int32_t* offsets,
+                                  int64_t T, int64_t P, int d, int N, int I, uint16_t* o,
+                                  int32_t* err_word, void* stream) {
+  if (T < 0 || P < 0 || P > kMaxTokens * 8) return MOE_ERR_INVALID_ARG;
+  if (T > kDecodeMaxTokens) return MOE_ERR_UNSUPPORTED;
+  if (!supported_n(N) || d <= 0 || d > kMaxDim || d % 128 != 0 || I <= 0 || I > kMaxDim ||
+      I % 64 != 0)
+    return MOE_ERR_UNSUPPORTED;
+  if (P == 0 || T == 0) return MOE_OK;
+  if (!h || !w_down || !offsets || !o || !aligned16(h) || !aligned16(w_down) || !aligned16(o))
+    return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_down_decode_gemm(h, w_down, offsets, P, d, N, I, o, err_word,
+                                                  sm_count(), static_cast<cudaStream_t>(stream)));
 }
 
 moe_status moe_gather_rows(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int64_t T,

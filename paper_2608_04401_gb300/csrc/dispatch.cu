@@ -149,7 +149,9 @@ MOE_DEV int block_exclusive_scan_small(int v, int* warp_tmp, int& total) {
   return before + x - v;
 }
 
-template <int N>
+// SINGLE: the batch is one chunk (T <= 128); its own counts are the expert
+// totals and its scan the expert offsets, so no count or scan pass runs.
+template <int N, bool SINGLE>
 __global__ void __launch_bounds__(kChunk) scatter_kernel(
     const int32_t* __restrict__ k, const int32_t* __restrict__ ids, int64_t T, int K, int nblk,
     const int32_t* __restrict__ base, const int32_t* __restrict__ totals,
@@ -165,12 +167,8 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int tid = threadIdx.x;
 
-  // expert offsets from the totals (every chunk recomputes them)
-  const int tot = tid < N ? totals[tid] : 0;
-  int total_pairs;
-  const int off = block_exclusive_scan_small<N>(tot, warp_tmp, total_pairs);
-  if (tid < N) exp_off[tid] = off;
-  if (blockIdx.x == 0) {
+  // expert offsets [N + 1] and m-tile prefix sums [N + 1], written by block 0
+  auto write_offsets = [&](int tot, int off, int total_pairs) {
     int total_tiles;
     const int toff = block_exclusive_scan_small<N>(tid < N ? (tot + 127) / 128 : 0, warp_tmp,
                                                    total_tiles);
@@ -184,6 +182,14 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
       tile_off[N] = total_tiles;
       if (offsets_copy) offsets_copy[N] = total_pairs;
     }
+  };
+  if constexpr (!SINGLE) {
+    // expert offsets from the totals (every chunk recomputes them)
+    const int tot = tid < N ? totals[tid] : 0;
+    int total_pairs;
+    const int off = block_exclusive_scan_small<N>(tot, warp_tmp, total_pairs);
+    if (tid < N) exp_off[tid] = off;
+    if (blockIdx.x == 0) write_offsets(tot, off, total_pairs);
   }
 
   const int64_t t = static_cast<int64_t>(blockIdx.x) * kChunk + tid;
@@ -205,8 +211,9 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
   }
   int chunk_pairs;
   const int chunk_off = block_exclusive_scan_small<N>(c_e, warp_tmp, chunk_pairs);
+  if constexpr (SINGLE) write_offsets(c_e, chunk_off, chunk_pairs);
   if (tid < N) {
-    int acc = exp_off[tid] + base[static_cast<int64_t>(tid) * nblk + blockIdx.x];
+    int acc = SINGLE ? chunk_off : exp_off[tid] + base[static_cast<int64_t>(tid) * nblk + blockIdx.x];
     int lacc = chunk_off;
 #pragma unroll
     for (int w = 0; w < kWarps; ++w) {
@@ -264,28 +271,35 @@ __global__ void __launch_bounds__(256) gather_kernel(const uint4* __restrict__ x
 }
 
 // y_t = sum_{s<k_t} g_{t,s} * o[pair_pos[t,s]] (+ residual_t); fp32 in s order.
-// One warp per token. The token's k positions and gates are read once (lane s
-// holds pair s) and broadcast by shuffles. The row is processed in slabs of
-// 32 * CH sixteen-byte chunks (lane l holds chunks l + 32c, c < CH; CH = 2
-// without a residual, 1 with one, which keeps both variants at four blocks
-// per SM): the loads of all k rows of a slab (and of the residual) are issued
-// before any is accumulated, so a warp keeps up to 8 KB in flight.
+// One warp per unit: a whole token, or for small batches one slab of a token
+// so that they still spread over many warps. The token's k positions and
+// gates are read per unit (lane s holds pair s) and broadcast by shuffles. A slab is 32 * CH sixteen-byte
+// chunks (lane l holds chunks l + 32c, c < CH; CH = 2 without a residual, 1
+// with one, which keeps both variants at four blocks per SM): the loads of
+// all k rows of a slab (and of the residual) are issued before any is
+// accumulated, so a warp keeps up to 8 KB in flight.
 constexpr int kCombineWarps = 4;
 
-template <bool RES>
+template <bool RES, bool SPLIT>
 __global__ void __launch_bounds__(32 * kCombineWarps, 4) combine_kernel(
     const uint4* __restrict__ o, const int32_t* __restrict__ k, const int32_t* __restrict__ pair_pos,
     const float* __restrict__ gates, const uint4* residual, int64_t T, int d8, int K, uint4* y) {
   const int lane = threadIdx.x & 31;
   const int64_t nwarps = static_cast<int64_t>(gridDim.x) * kCombineWarps;
   const int64_t cap = T * K;
-  for (int64_t t = static_cast<int64_t>(blockIdx.x) * kCombineWarps + threadIdx.x / 32; t < T;
-       t += nwarps) {
+  constexpr int CH = RES ? 1 : 2;
+  constexpr int kSlabChunks = 32 * CH;
+  // unit = a whole token, or (SPLIT, small batches) one slab of a token
+  const int nslab = (d8 + kSlabChunks - 1) / kSlabChunks;
+  for (int64_t u = static_cast<int64_t>(blockIdx.x) * kCombineWarps + threadIdx.x / 32;
+       u < (SPLIT ? T * nslab : T); u += nwarps) {
+    const int64_t t = SPLIT ? u / nslab : u;
     const int kt = min(k[t], K);
     const int my_pos = lane < kt ? static_cast<int>(min_of<int64_t>(max(pair_pos[t * K + lane], 0), cap - 1)) : 0;
     const float my_g = lane < kt ? gates[t * K + lane] : 0.0f;
-    constexpr int CH = RES ? 1 : 2;
-    for (int slab = 0; slab < d8; slab += 32 * CH) {
+    const int s0 = SPLIT ? static_cast<int>(u % nslab) * kSlabChunks : 0;
+    const int s1 = SPLIT ? s0 + kSlabChunks : d8;
+    for (int slab = s0; slab < s1; slab += kSlabChunks) {
       uint4 v[8][CH];
 #pragma unroll
       for (int s = 0; s < 8; ++s) {
@@ -380,6 +394,15 @@ static cudaError_t run_dispatch(const int32_t* k, const int32_t* ids, int64_t T,
                                 int32_t* totals, int32_t* tile_off, int32_t* offsets_copy,
                                 bool counts_ready, cudaStream_t stream) {
   const int nblk = num_chunks(T);
+  if (nblk == 1) {
+    if (N == 64)
+      disp::scatter_kernel<64, true><<<1, disp::kChunk, 0, stream>>>(
+          k, ids, T, K, nblk, cnt, totals, perm, pair_pos, offsets, tile_off, offsets_copy);
+    else
+      disp::scatter_kernel<128, true><<<1, disp::kChunk, 0, stream>>>(
+          k, ids, T, K, nblk, cnt, totals, perm, pair_pos, offsets, tile_off, offsets_copy);
+    return cudaGetLastError();
+  }
   if (nblk > 0 && !counts_ready) {
     if (N == 64) disp::count_kernel<64><<<nblk, disp::kChunk, 0, stream>>>(k, ids, T, K, nblk, cnt);
     else disp::count_kernel<128><<<nblk, disp::kChunk, 0, stream>>>(k, ids, T, K, nblk, cnt);
@@ -392,11 +415,11 @@ static cudaError_t run_dispatch(const int32_t* k, const int32_t* ids, int64_t T,
   }
   const int grid = nblk > 0 ? nblk : 1;
   if (N == 64)
-    disp::scatter_kernel<64><<<grid, disp::kChunk, 0, stream>>>(k, ids, T, K, nblk, cnt, totals, perm,
+    disp::scatter_kernel<64, false><<<grid, disp::kChunk, 0, stream>>>(k, ids, T, K, nblk, cnt, totals, perm,
                                                                 pair_pos, offsets, tile_off,
                                                                 offsets_copy);
   else
-    disp::scatter_kernel<128><<<grid, disp::kChunk, 0, stream>>>(k, ids, T, K, nblk, cnt, totals,
+    disp::scatter_kernel<128, false><<<grid, disp::kChunk, 0, stream>>>(k, ids, T, K, nblk, cnt, totals,
                                                                  perm, pair_pos, offsets, tile_off,
                                                                  offsets_copy);
   return cudaGetLastError();
@@ -425,10 +448,16 @@ cudaError_t launch_combine(const uint16_t* o, const int32_t* k, const int32_t* p
                            const float* gates, const uint16_t* residual, int64_t T, int d, int K,
                            uint16_t* y, int num_sms, cudaStream_t stream) {
   if (T == 0) return cudaSuccess;
-  int64_t blocks = (T + disp::kCombineWarps - 1) / disp::kCombineWarps;
+  const int ch = residual ? 32 : 64;  // sixteen-byte chunks per slab
+  const int nslab = (d / 8 + ch - 1) / ch;
+  // whole tokens per warp once the batch alone fills the GPU; slabs otherwise
+  const bool split = T < static_cast<int64_t>(num_sms) * 16;
+  const int64_t units = split ? T * nslab : T;
+  int64_t blocks = (units + disp::kCombineWarps - 1) / disp::kCombineWarps;
   const int64_t cap = static_cast<int64_t>(num_sms) * 16;
   if (blocks > cap) blocks = cap;
-  auto kern = residual ? disp::combine_kernel<true> : disp::combine_kernel<false>;
+  auto kern = residual ? (split ? disp::combine_kernel<true, true> : disp::combine_kernel<true, false>)
+                       : (split ? disp::combine_kernel<false, true> : disp::combine_kernel<false, false>);
   kern<<<static_cast<unsigned>(blocks), 32 * disp::kCombineWarps, 0, stream>>>(
       reinterpret_cast<const uint4*>(o), k, pair_pos, gates,
       reinterpret_cast<const uint4*>(residual), T, d / 8, K, reinterpret_cast<uint4*>(y));

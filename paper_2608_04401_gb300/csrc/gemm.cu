@@ -12,6 +12,13 @@
 //                   dispatch permutation (cp.async into the swizzled layout),
 //                   so the dispatched copy of x is never materialised
 //   kDown         : o[P, d] = h W_down[e]^T, per expert                 (bf16 out)
+//   kDecGateUp, kDecDown : the same two expert contractions for decode-sized
+//                   batches (every expert has at most 64 rows), with the roles
+//                   of the operands swapped: A = 128 weight rows (M), B = the
+//                   expert's <= 64 token rows (N = 64), so a tile streams
+//                   weights instead of padding 128-row token tiles. For
+//                   kDecGateUp the A tile is 64 gate rows and the matching 64
+//                   up rows; the epilogue pairs them through shared memory.
 //
 // Both operands are K-major bf16 tiles of 64 columns (128 bytes) moved by TMA
 // with 128-byte swizzle; the MMA is tcgen05.mma.cta_group::1.kind::f16 with
@@ -50,12 +57,22 @@ struct Roles {
   static constexpr int kEpiWarp0 = kProdWarps + 1;
   static constexpr int kThreads = 32 * (kProdWarps + 5);
 };
-enum Mode { kRouter = 0, kGateUp = 1, kDown = 2, kGateUpGather = 3, kRouterFused = 4 };
+enum Mode {
+  kRouter = 0,
+  kGateUp = 1,
+  kDown = 2,
+  kGateUpGather = 3,
+  kRouterFused = 4,
+  kDecGateUp = 5,
+  kDecDown = 6
+};
 
 template <int MODE>
 __host__ __device__ constexpr bool is_router() { return MODE == kRouter || MODE == kRouterFused; }
 template <int MODE>
 __host__ __device__ constexpr bool is_gateup() { return MODE == kGateUp || MODE == kGateUpGather; }
+template <int MODE>
+__host__ __device__ constexpr bool is_decode() { return MODE == kDecGateUp || MODE == kDecDown; }
 
 // Routing constants for the fused router epilogue (x'_i for i < N, and the
 // fast-path bound), in the layout route_token expects.
@@ -73,8 +90,10 @@ struct Cfg {
   static constexpr int kRouteTileBytes = 128 * (BN + 4) * 4;
   static constexpr int kRouteBytes =
       MODE == kRouterFused ? kRouteTileBytes + 8 * 128 * 8 + BN * 4 : 0;
-  // kDown: per epilogue warp two 32 x 32 bf16 staging tiles for TMA stores
-  static constexpr int kEpiBytes = MODE == kDown ? 4 * 2 * 32 * 64 : 0;
+  // kDown: per epilogue warp two 32 x 32 bf16 staging tiles for TMA stores;
+  // kDecGateUp: the up half of the accumulator, [64 rows][65] fp32
+  static constexpr int kEpiBytes =
+      MODE == kDown ? 4 * 2 * 32 * 64 : (MODE == kDecGateUp ? 64 * 65 * 4 : 0);
   static constexpr int kStages = (208 * 1024 - kRouteBytes - kEpiBytes) / kStageBytes;
   static constexpr int kTmemCols = (2 * BN <= 64) ? 64 : (2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512));
   static constexpr int kBarOff = kStages * kStageBytes;
@@ -126,6 +145,15 @@ MOE_DEV Tile decode(int tile, const Args& a, const int* s_off, const int* s_toff
     t.nb = 0;
     t.row0 = tile * BM;
     t.rows = static_cast<int>(min_of<int64_t>(BM, a.m_rows - t.row0));
+    return t;
+  }
+  if (is_decode<MODE>()) {
+    // tile = expert * n_tiles + weight-row block; the expert's rows are its
+    // B columns (an expert without rows has nothing to compute)
+    t.g = tile / a.n_tiles;
+    t.nb = tile % a.n_tiles;
+    t.row0 = s_off[t.g];
+    t.rows = s_off[t.g + 1] - t.row0;
     return t;
   }
   int lo = 0, hi = a.groups;  // s_toff[lo] * n_tiles <= tile < s_toff[hi] * n_tiles
@@ -238,7 +266,9 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
   if (!is_router<MODE>()) {  // grouped schedule tables (router modes have none)
     for (int i = threadIdx.x; i <= args.groups; i += kThreads) {
       s_off[i] = args.offsets[i];
-      s_toff[i] = args.tile_off[i];
+      // the decode modes schedule by expert and need no m-tile prefix sums
+      // (their tile_off is null)
+      s_toff[i] = is_decode<MODE>() ? 0 : args.tile_off[i];
     }
   }
   if (warp == 0 && lane == 0) {
@@ -255,8 +285,9 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  const int total = is_router<MODE>() ? static_cast<int>((args.m_rows + BM - 1) / BM)
-                                       : s_toff[args.groups] * args.n_tiles;
+  const int total = is_router<MODE>()   ? static_cast<int>((args.m_rows + BM - 1) / BM)
+                    : is_decode<MODE>() ? args.groups * args.n_tiles
+                                        : s_toff[args.groups] * args.n_tiles;
 
   if (MODE == kGateUpGather && warp < R::kProdWarps) {
     // --------------------------------------- producers, gathered A rows
@@ -321,13 +352,27 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
       int issued = 0;
       for (int tile = blockIdx.x; tile < total && !*abort_flag; tile += gridDim.x) {
         const Tile t = decode<MODE>(tile, args, s_off, s_toff);
+        if (is_decode<MODE>() && t.rows <= 0) continue;
         for (int kb = 0; kb < args.k_blocks; ++kb) {
           if (!mbar_wait_bounded(empty_bar(stage), phase ^ 1u, abort_flag)) break;
           const uint32_t a_dst = sbase + stage * C::kStageBytes;
           const uint32_t b_dst = a_dst + C::kABytes;
           mbar_arrive_expect_tx(full_bar(stage), C::kStageBytes);
-          tma_load_2d(a_dst, &tmA, full_bar(stage), kb * BK, t.row0);
-          if (is_gateup<MODE>()) {
+          if (MODE == kDecGateUp) {
+            // 64 gate rows, then the matching 64 up rows, of the expert's W_gate/up
+            const int arow = t.g * args.b_rows + t.nb * 64;
+            tma_load_2d(a_dst, &tmA, full_bar(stage), kb * BK, arow);
+            tma_load_2d(a_dst + 64 * BK * 2, &tmA, full_bar(stage), kb * BK, arow + args.b_half);
+          } else if (MODE == kDecDown) {
+            tma_load_2d(a_dst, &tmA, full_bar(stage), kb * BK, t.g * args.b_rows + t.nb * BM);
+          } else {
+            tma_load_2d(a_dst, &tmA, full_bar(stage), kb * BK, t.row0);
+          }
+          if (is_decode<MODE>()) {
+            // the expert's token rows (rows past them belong to other experts
+            // or lie past the end: their columns are never stored)
+            tma_load_2d(b_dst, &tmB, full_bar(stage), kb * BK, t.row0);
+          } else if (is_gateup<MODE>()) {
             const int brow = t.g * args.b_rows + t.nb * 128;
             tma_load_2d(b_dst, &tmB, full_bar(stage), kb * BK, brow);
             tma_load_2d(b_dst + 128 * BK * 2, &tmB, full_bar(stage), kb * BK, brow + args.b_half);
@@ -362,6 +407,10 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
       int local = 0;
       bool issued_any = false;
       for (int tile = blockIdx.x; tile < total && !*abort_flag; tile += gridDim.x, ++local) {
+        if (is_decode<MODE>() && decode<MODE>(tile, args, s_off, s_toff).rows <= 0) {
+          --local;  // an empty expert uses no accumulator (the loop step adds it back)
+          continue;
+        }
         const int acc = local & 1;
         const uint32_t acc_phase = (local >> 1) & 1;
         if (!mbar_wait_bounded(tempty_bar(acc), acc_phase ^ 1u, abort_flag)) break;
@@ -407,10 +456,14 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
     int local = 0;
     for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++local) {
       const Tile t = decode<MODE>(tile, args, s_off, s_toff);
+      if (is_decode<MODE>() && t.rows <= 0) {
+        --local;  // as in the MMA loop
+        continue;
+      }
       const int acc = local & 1;
       const uint32_t acc_phase = (local >> 1) & 1;
       const bool ok = mbar_wait_bounded(tfull_bar(acc), acc_phase, abort_flag);
-      if (MODE == kRouterFused) {
+      if (MODE == kRouterFused || MODE == kDecGateUp) {
         // all four epilogue warps take the same decision (they meet at named
         // barriers below), and each warp reconverges
         if (!epilogue_all(ok)) break;
@@ -480,6 +533,50 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
           for (int e = r; e < BN; e += 128)
             args.blk_cnt[static_cast<int64_t>(e) * args.nblk + tile] = hist[e];
           epilogue_sync();
+        }
+        continue;
+      } else if (is_decode<MODE>()) {
+        // TMEM lane r = weight row of the tile, column c = the expert's c-th row
+        uint32_t v0[32], v1[32];
+        tmem_ld_32x32b_x32(taddr, v0);
+        tmem_ld_32x32b_x32(taddr + 32, v1);
+        tmem_ld_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(tempty_bar(acc));
+        const int ncols = min(t.rows, BN);
+        __nv_bfloat16* out = static_cast<__nv_bfloat16*>(args.out) +
+                             static_cast<int64_t>(t.row0) * args.ldo;
+        if (MODE == kDecGateUp) {
+          // rows 64..127 hold up(i0 + r - 64): hand them to the warps holding gate(i0 + r)
+          float* xch = reinterpret_cast<float*>(smem + C::kEpiOff);
+          if (q >= 2) {
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+              xch[(r - 64) * 65 + c] = __uint_as_float(v0[c]);
+              xch[(r - 64) * 65 + 32 + c] = __uint_as_float(v1[c]);
+            }
+          }
+          epilogue_sync();
+          if (q < 2) {
+            __nv_bfloat16* o = out + t.nb * 64 + r;
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+              if (c < ncols)
+                o[c * args.ldo] = __float2bfloat16_rn(silu(__uint_as_float(v0[c])) * xch[r * 65 + c]);
+              if (32 + c < ncols)
+                o[(32 + c) * args.ldo] =
+                    __float2bfloat16_rn(silu(__uint_as_float(v1[c])) * xch[r * 65 + 32 + c]);
+            }
+          }
+          epilogue_sync();  // the exchange buffer is reused by the next tile
+        } else {
+          __nv_bfloat16* o = out + t.nb * BM + r;
+#pragma unroll
+          for (int c = 0; c < 32; ++c) {
+            if (c < ncols) o[c * args.ldo] = __float2bfloat16_rn(__uint_as_float(v0[c]));
+            if (32 + c < ncols) o[(32 + c) * args.ldo] = __float2bfloat16_rn(__uint_as_float(v1[c]));
+          }
         }
         continue;
       } else if (is_gateup<MODE>()) {
@@ -762,6 +859,52 @@ cudaError_t launch_down_gemm(const uint16_t* h, const uint16_t* wd, const int32_
   CUtensorMap mc;  // o [P, d], boxes of 32 x 32, no swizzle (TMA stores)
   if (!make_map_plain(&mc, o, d, P, 32, 32)) return cudaErrorInvalidValue;
   return launch_mode<kDown, 256>(ma, mb, mc, a, num_sms, stream);
+}
+
+// Decode-sized batches (every expert has at most 64 rows):
+// h[P, I] = silu(xs W_g^T) * (xs W_u^T) per expert, weights as the M operand
+cudaError_t launch_gateup_decode_gemm(const uint16_t* xs, const uint16_t* wgu,
+                                      const int32_t* offsets, int64_t P, int d, int N, int I,
+                                      uint16_t* h, int32_t* err, int num_sms, cudaStream_t stream) {
+  using namespace gemm;
+  if (P == 0) return cudaSuccess;
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, wgu, d, static_cast<uint64_t>(N) * 2 * I, 64) || !make_map(&mb, xs, d, P, 64))
+    return cudaErrorInvalidValue;
+  Args a{};
+  a.offsets = offsets;
+  a.groups = N;
+  a.n_tiles = I / 64;
+  a.k_blocks = d / BK;
+  a.b_rows = 2 * I;
+  a.b_half = I;
+  a.out = h;
+  a.ldo = I;
+  a.err = err;
+  const int tiles = N * a.n_tiles;
+  return launch_mode<kDecGateUp, 64>(ma, mb, ma, a, tiles < num_sms ? tiles : num_sms, stream);
+}
+
+// o[P, d] = h W_d[e]^T per expert, weights as the M operand
+cudaError_t launch_down_decode_gemm(const uint16_t* h, const uint16_t* wd, const int32_t* offsets,
+                                    int64_t P, int d, int N, int I, uint16_t* o, int32_t* err,
+                                    int num_sms, cudaStream_t stream) {
+  using namespace gemm;
+  if (P == 0) return cudaSuccess;
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, wd, I, static_cast<uint64_t>(N) * d, BM) || !make_map(&mb, h, I, P, 64))
+    return cudaErrorInvalidValue;
+  Args a{};
+  a.offsets = offsets;
+  a.groups = N;
+  a.n_tiles = d / BM;
+  a.k_blocks = I / BK;
+  a.b_rows = d;
+  a.out = o;
+  a.ldo = d;
+  a.err = err;
+  const int tiles = N * a.n_tiles;
+  return launch_mode<kDecDown, 64>(ma, mb, ma, a, tiles < num_sms ? tiles : num_sms, stream);
 }
 
 }  // namespace moe
