@@ -156,6 +156,28 @@ def bf16_dev(bits, dev):
     return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
 
 
+def max_over_ranks(value, pg):
+    """The largest value over all ranks (the slowest rank sets the job's time).
+    NCCL reduces a CUDA tensor, gloo a CPU one."""
+    if pg is None:
+        return float(value)
+    import torch
+    dev = "cuda" if pg.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([float(value)], dtype=torch.float64, device=dev)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+def rank_seed(base: int, rank: int) -> int:
+    """Each rank routes its own batch (weak scaling): a distinct seeded input."""
+    return base + 7919 * rank
+
+
+def job_tokens_per_s(tokens_per_rank: int, world: int, ms_per_step: float) -> float:
+    """Whole-job throughput: the tokens of all ranks over the slowest rank's time."""
+    return world * tokens_per_rank / (ms_per_step * 1e-3)
+
+
 def time_steps(fn, steps, stream, pg):
     """Barrier + sync on both sides; CUDA events on the launching stream."""
     import torch
@@ -171,9 +193,7 @@ def time_steps(fn, steps, stream, pg):
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1)
     if pg is not None:
-        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        ms = float(t.item())
+        ms = max_over_ranks(ms, pg)
     return ms / steps
 
 
@@ -195,7 +215,7 @@ def run_ours(args, rank, world, local, pg):
     T, d, N, I, K = w["T"], w["d"], w["N"], w["I"], w["K"]
     if args.tokens > 0:
         T = args.tokens
-    inp = synth.layer_inputs(T=T, d=d, N=N, I=I, seed=w["seed"] + 7919 * rank)
+    inp = synth.layer_inputs(T=T, d=d, N=N, I=I, seed=rank_seed(w["seed"], rank))
     x = bf16_dev(inp["x"], dev)
     wr = bf16_dev(inp["w_router"], dev)
     wgu = bf16_dev(inp["w_gate_up"], dev)
@@ -217,7 +237,7 @@ def run_ours(args, rank, world, local, pg):
     moe.read_device_error(ws)
     clocks = clk.summary()
     if args.quick:
-        return {"metric": METRIC, "value": world * T / (ms_elbow * 1e-3), "unit": "tokens/s",
+        return {"metric": METRIC, "value": job_tokens_per_s(T, world, ms_elbow), "unit": "tokens/s",
                 "n_gpus": world, "steps": args.steps, "ms_per_step": ms_elbow,
                 "topk_ms_per_step": ms_topk, "config": {"workload": f"{WORKLOAD} T={T}"},
                 "quick": True, "clocks": clocks}
@@ -257,7 +277,7 @@ def run_ours(args, rank, world, local, pg):
         e2e_step()
     ms_e2e = time_steps(e2e_step, max(20, args.steps // 4), stream, pg)
 
-    tok_s = world * T / (ms_elbow * 1e-3)
+    tok_s = job_tokens_per_s(T, world, ms_elbow)
     out = {
         "metric": METRIC,
         "value": tok_s,
@@ -278,7 +298,7 @@ def run_ours(args, rank, world, local, pg):
             "l2": "inputs larger than L2: 805 MB of expert weights and 64 MB of tokens per step",
             "parallelism": f"replicas x{world} (independent batches, no collective)",
         },
-        "topk": {"value": world * T / (ms_topk * 1e-3), "unit": "tokens/s", "ms_per_step": ms_topk,
+        "topk": {"value": job_tokens_per_s(T, world, ms_topk), "unit": "tokens/s", "ms_per_step": ms_topk,
                  "elbow_speedup": ms_topk / ms_elbow},
         "routing": {"mean_k": sum_k / T, "k_hist": np.bincount(kk, minlength=K + 1)[1:].tolist(),
                     "expert_load_min": int(load.min()), "expert_load_max": int(load.max())},
@@ -293,7 +313,7 @@ def run_ours(args, rank, world, local, pg):
         "kernels": kern,
         "route_stress": route,
         "other_configs": others,
-        "e2e": {"value": world * T / (ms_e2e * 1e-3), "unit": "tokens/s", "ms_per_step": ms_e2e,
+        "e2e": {"value": job_tokens_per_s(T, world, ms_e2e), "unit": "tokens/s", "ms_per_step": ms_e2e,
                 "h2d_bytes_per_step": T * d * 2, "d2h_bytes_per_step": T * d * 2},
         "gpu_launches": KERNELS_PER_STEP * args.steps * 2,
         "clocks": clocks,
