@@ -292,6 +292,14 @@ moe_status elbow_route_randomized(const float* logits, int64_t T, int N, const m
                                   const uint32_t* rand, int32_t* k_out, int32_t* ids_out,
                                   float* gates_out, void* stream);
 
+/* Exercises the bounded wait that every GEMM pipeline uses, on an mbarrier
+ * that nothing arrives on: the kernel gives up after `seconds` (0 < seconds
+ * <= 10) and writes the timeout code into err_word (device, 4-byte aligned;
+ * cleared first), exactly as a GEMM whose producer never delivered would.
+ * moe_read_device_error(err_word, stream) then returns MOE_ERR_DEVICE_TIMEOUT
+ * and the context stays usable. */
+moe_status moe_check_bounded_wait(int32_t* err_word, double seconds, void* stream);
+
 /*
  * moe_route_diagnostics - routing diagnostics of Sec. 2.3 (elbow angle),
  * Sec. 2.4 and App. A.3 (expert-load changes of elbow-K against top-K).

@@ -18,7 +18,7 @@ import threading
 import numpy as np
 
 __all__ = [
-    "MODE_ELBOW", "MODE_TOPK", "MoeError", "library", "build", "route_diagnostics", "RouteDiag",
+    "MODE_ELBOW", "MODE_TOPK", "MoeError", "library", "build", "route_diagnostics", "RouteDiag", "check_bounded_wait",
     "elbow_route_randomized", "MODE_RAND_TAIL", "MODE_RAND_HEAD",
     "elbow_route", "moe_dispatch", "moe_dispatch_noalloc", "dispatch_workspace_size", "layer_workspace_size",
     "moe_layer_forward", "read_device_error", "router_logits", "gather_rows",
@@ -92,6 +92,7 @@ def library():
             "moe_layer_forward": ([P, P, P, P, i64, i32, i32, i32, RP, P, P, P, P, P, P, P, P, sz, P],
                                   i32),
             "moe_read_device_error": ([P, P], i32),
+            "moe_check_bounded_wait": ([P, ctypes.c_double, P], i32),
             "moe_router_logits": ([P, P, i64, i32, i32, P, P, P], i32),
             "moe_expert_gate_up": ([P, P, P, P, i64, i32, i32, i32, P, P, P], i32),
             "moe_expert_down": ([P, P, P, P, i64, i32, i32, i32, P, P, P], i32),
@@ -199,6 +200,15 @@ def elbow_route_randomized(logits, rand, K: int = 8, eps: float = 1e-8, mode: in
                                             _p(rand), _p(k), _p(ids), _p(gates), _stream(stream)),
            "elbow_route_randomized")
     return k, ids, gates
+
+
+def check_bounded_wait(err, seconds: float = 0.2, stream=None) -> int:
+    """Run the GEMMs' bounded wait on a barrier nothing arrives on; returns the
+    status moe_read_device_error reports afterwards (MOE_ERR_DEVICE_TIMEOUT = 5)."""
+    lib = library()
+    _check(lib.moe_check_bounded_wait(_p(err), float(seconds), _stream(stream)),
+           "moe_check_bounded_wait")
+    return int(lib.moe_read_device_error(_p(err), _stream(stream)))
 
 
 def route_diagnostics(logits, K: int = 8, eps: float = 1e-8, per_token: bool = True,

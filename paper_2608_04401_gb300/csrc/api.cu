@@ -50,6 +50,22 @@ cudaError_t launch_route_diagnostics(const float* logits, int64_t T, int N, int 
 
 namespace {
 
+// The bounded wait of the GEMM pipelines on an mbarrier that nothing arrives
+// on: thread 0 gives up after limit_ns and writes the timeout code into *err.
+__global__ void bounded_wait_check_kernel(int32_t* err, uint64_t limit_ns) {
+  __shared__ alignas(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    moe::mbar_init(moe::smem_u32(&bar), 1);
+    abort_flag = 0;
+    moe::fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 &&
+      !moe::mbar_wait_bounded(moe::smem_u32(&bar), 0u, &abort_flag, limit_ns))
+    atomicExch(err, moe::kDevErrTimeout);
+}
+
 constexpr int64_t kMaxTokens = int64_t(1) << 28;  // keeps T * K * 8 row counts in int32
 constexpr int kMaxDim = 16384;
 // Batches of at most this many tokens take the decode-shaped expert GEMMs
@@ -329,6 +345,15 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   e = moe::launch_combine(w.o, kk, w.pair_pos, gates, residual, T, d, K, y, nsm, s);
   if (e != cudaSuccess) return MOE_ERR_CUDA;
   return MOE_OK;
+}
+
+moe_status moe_check_bounded_wait(int32_t* err_word, double seconds, void* stream) {
+  if (!err_word || (reinterpret_cast<uintptr_t>(err_word) & 3u)) return MOE_ERR_INVALID_ARG;
+  if (!(seconds > 0.0) || seconds > 10.0) return MOE_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(err_word, 0, sizeof(int32_t), s) != cudaSuccess) return MOE_ERR_CUDA;
+  bounded_wait_check_kernel<<<1, 32, 0, s>>>(err_word, static_cast<uint64_t>(seconds * 1e9));
+  return cuda_status(cudaGetLastError());
 }
 
 moe_status moe_read_device_error(const void* ws, void* stream) {

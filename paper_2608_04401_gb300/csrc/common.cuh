@@ -74,7 +74,8 @@ MOE_DEV bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 // Waits until the phase with the given parity has completed. Gives up after
 // kWaitLimitNs, or at once when *abort is set by another thread; returns false
 // then (and raises *abort).
-MOE_DEV bool mbar_wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort) {
+MOE_DEV bool mbar_wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort,
+                               uint64_t limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_timer_ns();
   uint32_t spins = 0;
@@ -82,7 +83,7 @@ MOE_DEV bool mbar_wait_bounded(uint32_t bar, uint32_t parity, volatile int* abor
     if (mbar_try_wait(bar, parity)) return true;
     if (++spins % 64u == 0u) {
       if (*abort) return false;
-      if (global_timer_ns() - t0 > kWaitLimitNs) {
+      if (global_timer_ns() - t0 > limit_ns) {
         *abort = 1;
         return false;
       }

@@ -107,3 +107,10 @@ def test_randomized_validation(lib):
     # elbow_route itself rejects the randomisation modes
     assert lib.elbow_route(fake, 10, 64, _rp(mode=2), fake, fake, fake, None) == 1
 
+
+def test_bounded_wait_check_validation(lib):
+    assert lib.moe_check_bounded_wait(None, 0.1, None) == 1
+    assert lib.moe_check_bounded_wait(ctypes.c_void_p(258), 0.1, None) == 1
+    assert lib.moe_check_bounded_wait(ctypes.c_void_p(256), 0.0, None) == 1
+    assert lib.moe_check_bounded_wait(ctypes.c_void_p(256), 11.0, None) == 1
+
