@@ -2,15 +2,15 @@
 // plus the row gather and the gate-weighted combine.
 //
 // Dispatch is a deterministic counting sort over chunks of 128 tokens:
-//   count   : per chunk, per-expert pair counts (warp ballots), stored
+//   count   : per chunk, per-expert pair counts (bit-transposed warp masks), stored
 //             expert-major: cnt[e][chunk]. The elbow router can write these
 //             itself, in which case this pass is skipped.
 //   scan    : one block per expert: exclusive prefix over the chunks, in
 //             place, and the expert's total.
 //   scatter : each chunk recomputes the expert offsets from the totals, then
 //             places its pairs: position = offsets[e] + chunk base + earlier
-//             warps of the chunk (ballots in smem) + earlier lanes of the warp
-//             (popc of the ballot). Chunk 0 also writes offsets [N+1] and the
+//             warps of the chunk (per-expert warp masks in smem) + earlier lanes
+//             of the warp (popc of the mask). Chunk 0 also writes offsets [N+1] and the
 //             m-tile prefix sums ceil(count_e / 128) [N+1].
 #include <mutex>
 
@@ -48,9 +48,30 @@ MOE_DEV void load_selection(const int32_t* __restrict__ k, const int32_t* __rest
   }
 }
 
-template <int N>
-MOE_DEV bool has_expert(int e, uint64_t m0, uint64_t m1) {
-  return ((e < 64 ? (m0 >> e) : (m1 >> (e - 64))) & 1ull) != 0;
+// 32 x 32 bit-matrix transpose across a warp: lane i holds row i in x; lane j
+// gets column j (bit i of the result = bit j of lane i's x). Five stages swap
+// the off-diagonal blocks of width 16, 8, 4, 2, 1 with the partner lane
+// (Warren, Hacker's Delight, sec. 7-3, with lanes as rows). Applied to the
+// lanes' expert masks it gives lane e the ballot of expert e for the warp's 32
+// tokens, in five shuffles instead of 32 ballots.
+MOE_DEV uint32_t transpose32(uint32_t x, int lane) {
+#pragma unroll
+  for (int s = 16; s >= 1; s >>= 1) {
+    const uint32_t m = s == 16 ? 0x0000FFFFu
+                     : s == 8  ? 0x00FF00FFu
+                     : s == 4  ? 0x0F0F0F0Fu
+                     : s == 2  ? 0x33333333u
+                               : 0x55555555u;
+    const uint32_t y = __shfl_xor_sync(0xffffffffu, x, s);
+    x = (lane & s) ? ((x & ~m) | ((y & ~m) >> s)) : ((x & m) | ((y & m) << s));
+  }
+  return x;
+}
+
+// The expert masks as 32-bit words: experts 32q .. 32q + 31 in word q.
+MOE_DEV uint32_t mask_word(int q, uint64_t m0, uint64_t m1) {
+  const uint64_t m = q < 2 ? m0 : m1;
+  return static_cast<uint32_t>((q & 1) ? (m >> 32) : m);
 }
 
 template <int N>
@@ -64,10 +85,8 @@ __global__ void __launch_bounds__(kChunk) count_kernel(const int32_t* __restrict
   uint64_t m0, m1;
   load_selection(k, ids, t, t < T, K, kt, my, m0, m1);
 #pragma unroll
-  for (int e = 0; e < N; ++e) {
-    const int c = __popc(__ballot_sync(0xffffffffu, has_expert<N>(e, m0, m1)));
-    if (lane == (e & 31)) wcnt[warp][e] = c;
-  }
+  for (int q = 0; q < N / 32; ++q)
+    wcnt[warp][32 * q + lane] = __popc(transpose32(mask_word(q, m0, m1), lane));
   __syncthreads();
   for (int e = threadIdx.x; e < N; e += kChunk) {
     int c = 0;
@@ -198,10 +217,7 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
   uint64_t m0, m1;
   load_selection(k, ids, t, valid, K, kt, my, m0, m1);
 #pragma unroll
-  for (int e = 0; e < N; ++e) {
-    const uint32_t b = __ballot_sync(0xffffffffu, has_expert<N>(e, m0, m1));
-    if (lane == (e & 31)) bal[warp][e] = b;
-  }
+  for (int q = 0; q < N / 32; ++q) bal[warp][32 * q + lane] = transpose32(mask_word(q, m0, m1), lane);
   __syncthreads();
   // this chunk's count per expert, and its exclusive scan over the experts
   int c_e = 0;
