@@ -377,6 +377,25 @@ def dev_experts(N, d, I, seed, dev):
     return wgu, wd
 
 
+def graph_ms(step, steps, stream, pg):
+    """ms per replay of a CUDA graph that captured one call of `step` (the
+    library launches on the current stream and allocates nothing, so a whole
+    layer, or stack of layers, is one graph)."""
+    import torch
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for _ in range(2):
+            step()
+    torch.cuda.current_stream().wait_stream(side)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        step()
+    for _ in range(3):
+        g.replay()
+    return time_steps(g.replay, steps, stream, pg)
+
+
 def time_layer_modes(moe, x, wr, wgu, wd, K, steps, stream, pg, residual=None):
     """ms per moe_layer_forward in elbow and in top-K mode; sum k of the elbow batch."""
     import torch
@@ -392,6 +411,7 @@ def time_layer_modes(moe, x, wr, wgu, wd, K, steps, stream, pg, residual=None):
         for _ in range(3):
             step()
         out[name] = time_steps(step, steps, stream, pg)
+        out[name + "_graph"] = graph_ms(step, steps, stream, pg)
     moe.read_device_error(ws)
     _, it = moe.moe_layer_forward(x, wr, wgu, wd, K=K, y=y, ws=ws, return_intermediates=True)
     out["sum_k"] = int(it["k"].sum().item())
@@ -422,11 +442,25 @@ def other_configs(moe, args, stream, dev, pk, pg):
             "workload": f"T={T}, d_model={d}, N={N}, I={I}, K={K}"
                         + (f", {int(100 * w['flat_frac'])}% flat tokens" if "flat_frac" in w else ""),
             "elbow_ms": r["elbow"], "topk_ms": r["topk"], "elbow_speedup": r["topk"] / r["elbow"],
+            "elbow_graph_ms": r["elbow_graph"], "topk_graph_ms": r["topk_graph"],
             "tokens_per_s": T / (r["elbow"] * 1e-3), "mean_k": r["sum_k"] / T,
             "experts_touched": r["touched"],
             "tflops": flops / (r["elbow"] * 1e-3) / 1e12,
             "weight_hbm_frac": wbytes / (r["elbow"] * 1e-3) / 1e9 / pk["hbm"],
         }
+        if name == "layer_t64":
+            # single-token and 8-token decode steps on the same weights: the
+            # elbow's k decides how many experts' weights are streamed at all
+            dec = {}
+            for Td in (1, 8):
+                rd = time_layer_modes(moe, x[:Td].contiguous(), wr, wgu, wd, K, steps, stream, pg)
+                wb = rd["touched"] * 3 * d * I * 2
+                dec[f"T={Td}"] = {"elbow_ms": rd["elbow"], "topk_ms": rd["topk"],
+                                  "elbow_graph_ms": rd["elbow_graph"],
+                                  "topk_graph_ms": rd["topk_graph"],
+                                  "experts_touched": rd["touched"], "mean_k": rd["sum_k"] / Td,
+                                  "weight_hbm_frac_graph": wb / (rd["elbow_graph"] * 1e-3) / 1e9 / pk["hbm"]}
+            res[name]["decode"] = dec
         del wgu, wd
         torch.cuda.empty_cache()
     # 16-layer stack with the residual add between layers
@@ -449,6 +483,7 @@ def other_configs(moe, args, stream, dev, pk, pg):
         for _ in range(2):
             stack()
         out[name] = time_steps(stack, max(5, steps // 4), stream, pg)
+        out[name + "_graph"] = graph_ms(stack, max(5, steps // 4), stream, pg)
     moe.read_device_error(ws)
     mean_k = []
     cur = x0
@@ -461,6 +496,7 @@ def other_configs(moe, args, stream, dev, pk, pg):
     res["stack16_t4k"] = {
         "workload": f"{L} layers, T={T}, d_model={d}, N={N}, I={I}, K={K}, residual add",
         "elbow_ms": out["elbow"], "topk_ms": out["topk"], "elbow_speedup": out["topk"] / out["elbow"],
+        "elbow_graph_ms": out["elbow_graph"], "topk_graph_ms": out["topk_graph"],
         "tokens_per_s": T / (out["elbow"] * 1e-3), "mean_k_per_layer": mean_k,
     }
     del layers
