@@ -90,6 +90,16 @@ const char* moe_status_string(moe_status s);
 moe_status elbow_route(const float* logits, int64_t T, int N, const moe_route_params* rp,
                        int32_t* k_out, int32_t* ids_out, float* gates_out, void* stream);
 
+/* elbow_route with one warp (instead of one thread) per token: lane l holds
+ * experts l + 32c, the N (p, id) keys are sorted by a bitonic network of warp
+ * shuffles and the argmax is a warp reduction. Same specification, same bits
+ * as elbow_route; a much shorter critical path per token, at about three
+ * times the instructions per token, so elbow_route uses it by itself for
+ * T <= 16 (and moe_layer_forward's router for T <= 16). Arguments and errors
+ * as elbow_route (ids_out and gates_out need only 4-byte alignment). */
+moe_status elbow_route_warp(const float* logits, int64_t T, int N, const moe_route_params* rp,
+                            int32_t* k_out, int32_t* ids_out, float* gates_out, void* stream);
+
 /* elbow_route that also counts, for the dispatch, the selected pairs of each
  * expert in each chunk of 128 tokens: chunk_counts [N][ceil(T/128)] int32
  * (pass moe_dispatch_chunk_counts(ws) and follow with moe_dispatch_counted,

@@ -18,7 +18,7 @@ import threading
 import numpy as np
 
 __all__ = [
-    "MODE_ELBOW", "MODE_TOPK", "MoeError", "library", "build", "route_diagnostics", "RouteDiag", "check_bounded_wait",
+    "MODE_ELBOW", "MODE_TOPK", "MoeError", "library", "build", "route_diagnostics", "RouteDiag", "check_bounded_wait", "elbow_route_warp",
     "elbow_route_randomized", "MODE_RAND_TAIL", "MODE_RAND_HEAD",
     "elbow_route", "moe_dispatch", "moe_dispatch_noalloc", "dispatch_workspace_size", "layer_workspace_size",
     "moe_layer_forward", "read_device_error", "router_logits", "gather_rows",
@@ -80,6 +80,7 @@ def library():
             "moe_status_string": ([i32], ctypes.c_char_p),
             "elbow_route": ([P, i64, i32, RP, P, P, P, P], i32),
             "elbow_route_with_counts": ([P, i64, i32, RP, P, P, P, P, P], i32),
+            "elbow_route_warp": ([P, i64, i32, RP, P, P, P, P], i32),
             "moe_route_diagnostics": ([P, i64, i32, RP, P, P, P, P], i32),
             "elbow_route_randomized": ([P, i64, i32, RP, P, P, P, P, P], i32),
             "moe_dispatch_workspace_size": ([i64, i32, i32], sz),
@@ -158,6 +159,20 @@ def elbow_route(logits, K: int = 8, eps: float = 1e-8, mode: int = MODE_ELBOW, r
     gates = torch.empty(T, K, dtype=torch.float32, device=logits.device)
     _check(lib.elbow_route(_p(logits), T, N, _params(K, eps, mode, renorm), _p(k), _p(ids),
                            _p(gates), _stream(stream)), "elbow_route")
+    return k, ids, gates
+
+
+def elbow_route_warp(logits, K: int = 8, eps: float = 1e-8, mode: int = MODE_ELBOW, renorm: int = 0,
+                     stream=None):
+    """elbow_route with one warp per token (same results; the small-batch kernel)."""
+    torch = _torch()
+    _cuda(logits, torch.float32, "logits")
+    T, N = logits.shape
+    k = torch.empty(T, dtype=torch.int32, device=logits.device)
+    ids = torch.empty(T, K, dtype=torch.int32, device=logits.device)
+    gates = torch.empty(T, K, dtype=torch.float32, device=logits.device)
+    _check(library().elbow_route_warp(_p(logits), T, N, _params(K, eps, mode, renorm), _p(k),
+                                      _p(ids), _p(gates), _stream(stream)), "elbow_route_warp")
     return k, ids, gates
 
 

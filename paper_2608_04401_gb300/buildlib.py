@@ -16,7 +16,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(OUT_DIR, "libelbow_moe.so")
-SOURCES = ["api.cu", "route.cu", "dispatch.cu", "gemm.cu", "diag.cu"]
+SOURCES = ["api.cu", "route.cu", "route_warp.cu", "dispatch.cu", "gemm.cu", "diag.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

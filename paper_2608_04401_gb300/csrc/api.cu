@@ -43,6 +43,11 @@ cudaError_t launch_gateup_decode_gemm(const uint16_t* xs, const uint16_t* wgu,
 cudaError_t launch_down_decode_gemm(const uint16_t* h, const uint16_t* wd, const int32_t* offsets,
                                     int64_t P, int d, int N, int I, uint16_t* o, int32_t* err,
                                     int num_sms, cudaStream_t stream);
+cudaError_t launch_route_warp(const float* src, int nslice, int64_t T, int N, int K, float eps,
+                              int topk_mode, int renorm, float* logits_out, int32_t* k_out,
+                              int32_t* ids_out, float* gates_out, cudaStream_t stream);
+cudaError_t launch_router_small(const uint16_t* x, const uint16_t* w_router, int T, int d, int N,
+                                float* partial, cudaStream_t stream);
 cudaError_t launch_route_diagnostics(const float* logits, int64_t T, int N, int K, float eps,
                                      int32_t* elbow_out, float* theta_out, moe_route_diag* dg,
                                      cudaStream_t stream);
@@ -71,6 +76,10 @@ constexpr int kMaxDim = 16384;
 // Batches of at most this many tokens take the decode-shaped expert GEMMs
 // (weights as the M operand; every expert then has at most 64 rows).
 constexpr int64_t kDecodeMaxTokens = 64;
+// Batches of at most this many tokens route with one warp per token, after a
+// router GEMM split over d (below it the fused router's one-thread-per-token
+// routing chain dominates; above it the fused router is faster).
+constexpr int64_t kWarpRouteMaxTokens = 16;
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -112,6 +121,7 @@ struct LayerWs {
   int32_t* pair_pos;
   uint16_t* h;
   uint16_t* o;
+  float* partial;  // decode-sized batches: router partial sums [d/64][T][N]
   size_t bytes;
 };
 
@@ -135,6 +145,8 @@ LayerWs layer_ws(void* base, int64_t T, int d, int N, int I, int K) {
   w.pair_pos = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * (P > 0 ? P : 1)));
   w.h = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * P * I));
   w.o = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * P * d));
+  w.partial = reinterpret_cast<float*>(
+      take(T <= kWarpRouteMaxTokens ? sizeof(float) * static_cast<size_t>(d / 64) * T * N : 0));
   w.bytes = off;
   return w;
 }
@@ -166,9 +178,30 @@ moe_status elbow_route(const float* logits, int64_t T, int N, const moe_route_pa
   if (!aligned16(logits) || !aligned16(ids_out) || !aligned16(gates_out) ||
       (reinterpret_cast<uintptr_t>(k_out) & 3u))
     return MOE_ERR_INVALID_ARG;
+  if (T <= kWarpRouteMaxTokens)  // a few tokens: one warp each has the shorter critical path
+    return cuda_status(moe::launch_route_warp(logits, 1, T, N, rp->K, rp->eps,
+                                              rp->mode == MOE_ROUTE_TOPK, rp->renorm, nullptr,
+                                              k_out, ids_out, gates_out,
+                                              static_cast<cudaStream_t>(stream)));
   return cuda_status(moe::launch_elbow_route(logits, T, N, rp->K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
                                              rp->renorm, k_out, ids_out, gates_out, nullptr,
                                              nullptr, 0, static_cast<cudaStream_t>(stream)));
+}
+
+moe_status elbow_route_warp(const float* logits, int64_t T, int N, const moe_route_params* rp,
+                            int32_t* k_out, int32_t* ids_out, float* gates_out, void* stream) {
+  if (T < 0 || T > kMaxTokens) return MOE_ERR_INVALID_ARG;
+  if (!supported_n(N)) return MOE_ERR_UNSUPPORTED;
+  moe_status st = check_route_params(rp, N);
+  if (st != MOE_OK) return st;
+  if (T == 0) return MOE_OK;
+  if (!logits || !k_out || !ids_out || !gates_out) return MOE_ERR_INVALID_ARG;
+  if (!aligned16(logits) || (reinterpret_cast<uintptr_t>(ids_out) & 3u) ||
+      (reinterpret_cast<uintptr_t>(gates_out) & 3u) || (reinterpret_cast<uintptr_t>(k_out) & 3u))
+    return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_route_warp(logits, 1, T, N, rp->K, rp->eps,
+                                            rp->mode == MOE_ROUTE_TOPK, rp->renorm, nullptr, k_out,
+                                            ids_out, gates_out, static_cast<cudaStream_t>(stream)));
 }
 
 moe_status elbow_route_randomized(const float* logits, int64_t T, int N, const moe_route_params* rp,
@@ -315,11 +348,20 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   const int nsm = sm_count();
 
   cudaError_t e;
-  // router GEMM with the elbow routing in its epilogue; it also leaves the
-  // per-chunk expert counts of the dispatch
-  e = moe::launch_router_route(x, w_router, T, d, N, K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
-                               rp->renorm, logits_out, kk, ids, gates, moe::dispatch_counts(w.disp),
-                               w.err, nsm, s);
+  if (T <= kWarpRouteMaxTokens) {
+    // a few tokens: the router GEMM split over d on every SM, then one warp per
+    // token routes (the single-chunk dispatch counts the pairs itself)
+    e = moe::launch_router_small(x, w_router, static_cast<int>(T), d, N, w.partial, s);
+    if (e != cudaSuccess) return MOE_ERR_CUDA;
+    e = moe::launch_route_warp(w.partial, d / 64, T, N, K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
+                               rp->renorm, logits_out, kk, ids, gates, s);
+  } else {
+    // router GEMM with the elbow routing in its epilogue; it also leaves the
+    // per-chunk expert counts of the dispatch
+    e = moe::launch_router_route(x, w_router, T, d, N, K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
+                                 rp->renorm, logits_out, kk, ids, gates,
+                                 moe::dispatch_counts(w.disp), w.err, nsm, s);
+  }
   if (e != cudaSuccess) return MOE_ERR_CUDA;
   e = moe::launch_dispatch(kk, ids, T, N, K, w.offsets, w.perm, w.pair_pos, w.disp, offsets_out,
                            true, s);

@@ -191,3 +191,46 @@ def test_route_with_counts_then_counted_dispatch(moe, N, T):
     n = int(d["offsets"][-1])
     assert np.array_equal(perm.cpu().numpy()[:n], d["perm"])
     assert np.array_equal(pp.cpu().numpy(), d["pair_pos"])
+
+
+# ------------------------------------------- one warp per token (small batches)
+def _route_warp_both(moe, lg, K=8, mode=0, renorm=0, eps=1e-8):
+    k, ids, gates = moe.elbow_route_warp(to_dev(lg), K=K, eps=eps, mode=mode, renorm=renorm)
+    ref = oracle.route(lg, K=K, eps=eps, mode=mode, renorm=renorm)
+    return (k.cpu().numpy(), ids.cpu().numpy(), gates.cpu().numpy()), ref
+
+
+@pytest.mark.parametrize("N", [64, 128])
+@pytest.mark.parametrize("K,mode,renorm", [(8, 0, 0), (8, 1, 0), (8, 0, 1), (1, 0, 0), (3, 0, 1)])
+def test_route_warp_bitexact(moe, N, K, mode, renorm):
+    rng = np.random.default_rng(N * 3 + K + 7 * mode + renorm)
+    lg = synth.boosted_logits(rng, 3001, N)
+    _assert_route_equal(*_route_warp_both(moe, lg, K=K, mode=mode, renorm=renorm))
+
+
+@pytest.mark.parametrize("N", [64, 128])
+def test_route_warp_edge_cases(moe, N):
+    """The curves that stress the thread kernel's shortcuts, through the warp
+    kernel: near ties, exact ties, flat and linear curves, wide heads, tails
+    that underflow, uniform rows, step curves."""
+    rng = np.random.default_rng(N + 5)
+    rows = [np.zeros(N), np.full(N, 2.5)]
+    for m in (1, 2, 7, 8, 9, N // 2, N - 2, N - 1):
+        r = np.zeros(N); r[:m] = 6.0; rows.append(r)
+    r = np.full(N, -500.0); r[3] = 0.0; rows.append(r)
+    r = np.linspace(-60, 30, N); rows.append(r)
+    lg = rng.standard_normal((1024, N)).astype(np.float32)
+    lg[0:256] = (2.0 + rng.integers(-3, 4, (256, N)) * np.float32(2.0 ** -22)).astype(np.float32)
+    lg[256:512] = np.round(rng.uniform(-1, 1, (256, N)) * 4) / 4
+    lg[512:768] = rng.uniform(-200, -60, (256, N)); lg[512:768, 0] = 0.0
+    lg = np.concatenate([np.array(rows, np.float32), lg]).astype(np.float32)
+    for K, mode in ((8, 0), (8, 1), (2, 0)):
+        _assert_route_equal(*_route_warp_both(moe, lg, K=K, mode=mode))
+
+
+def test_route_warp_full_stress(moe):
+    """The 1,048,576-token stress through the warp kernel, token by token."""
+    w = synth.WORKLOADS["route_t1m"]
+    rng = np.random.Generator(np.random.PCG64(w["seed"] + 2))
+    lg = synth.boosted_logits(rng, w["T"], w["N"])
+    _assert_route_equal(*_route_warp_both(moe, lg, K=w["K"]))
