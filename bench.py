@@ -262,20 +262,9 @@ def run_ours(args, rank, world, local, pg):
     route = route_stress(moe, args, stream, dev, pk)
     others = other_configs(moe, args, stream, dev, pk, pg)
 
-    # end to end through the public API with host buffers
-    xh = torch.empty(T, d, dtype=torch.bfloat16, pin_memory=True)
-    xh.copy_(x.cpu())
-    yh = torch.empty(T, d, dtype=torch.bfloat16, pin_memory=True)
-    xd = torch.empty_like(x)
-
-    def e2e_step():
-        xd.copy_(xh, non_blocking=True)
-        moe.moe_layer_forward(xd, wr, wgu, wd, K=K, y=y, ws=ws)
-        yh.copy_(y, non_blocking=True)
-
-    for _ in range(3):
-        e2e_step()
-    ms_e2e = time_steps(e2e_step, max(20, args.steps // 4), stream, pg)
+    # end to end through the public API with host buffers: every step copies
+    # its tokens in from pinned host memory and its outputs back out
+    ms_e2e_serial, ms_e2e = e2e_ms(moe, x, wr, wgu, wd, K, ws, max(20, args.steps // 4), stream, pg)
 
     tok_s = job_tokens_per_s(T, world, ms_elbow)
     out = {
@@ -314,7 +303,10 @@ def run_ours(args, rank, world, local, pg):
         "route_stress": route,
         "other_configs": others,
         "e2e": {"value": job_tokens_per_s(T, world, ms_e2e), "unit": "tokens/s", "ms_per_step": ms_e2e,
-                "h2d_bytes_per_step": T * d * 2, "d2h_bytes_per_step": T * d * 2},
+                "h2d_bytes_per_step": T * d * 2, "d2h_bytes_per_step": T * d * 2,
+                "pipelined": "copy-in and copy-out streams, two device x/y buffers: step i's "
+                             "copy-out and step i+1's copy-in overlap step i's layer",
+                "serial_ms_per_step": ms_e2e_serial},
         "gpu_launches": KERNELS_PER_STEP * args.steps * 2,
         "clocks": clocks,
     }
@@ -362,6 +354,71 @@ def kernel_breakdown(moe, x, wr, wgu, wd, T, d, N, I, K, args, stream, dev):
     assert int(err.item()) == 0, "device timeout in a GEMM"
     tot = sum(acc.values())
     return {n: {"ms": acc[n] / steps, "share": acc[n] / tot} for n in names}
+
+
+def e2e_ms(moe, x, wr, wgu, wd, K, ws, steps, stream, pg):
+    """ms per step end to end (pinned host x in, host y out, through
+    moe_layer_forward): (serial on one stream, pipelined over two copy streams
+    with double-buffered device x and y). The pipelined form keeps every
+    step's own copies; it overlaps them with the neighbouring steps' layers."""
+    import torch
+    T, d = x.shape
+    xh = torch.empty(T, d, dtype=torch.bfloat16, pin_memory=True)
+    xh.copy_(x.cpu())
+    yh = [torch.empty(T, d, dtype=torch.bfloat16, pin_memory=True) for _ in range(2)]
+    xd = [torch.empty_like(x) for _ in range(2)]
+    yd = [torch.empty_like(x) for _ in range(2)]
+
+    def serial_step():
+        xd[0].copy_(xh, non_blocking=True)
+        moe.moe_layer_forward(xd[0], wr, wgu, wd, K=K, y=yd[0], ws=ws)
+        yh[0].copy_(yd[0], non_blocking=True)
+
+    for _ in range(3):
+        serial_step()
+    ms_serial = time_steps(serial_step, steps, stream, pg)
+
+    comp = torch.cuda.current_stream()
+    cin, cout = torch.cuda.Stream(), torch.cuda.Stream()
+    in_done = [torch.cuda.Event() for _ in range(2)]
+    comp_done = [torch.cuda.Event() for _ in range(2)]
+    out_done = [torch.cuda.Event() for _ in range(2)]
+    for b in range(2):  # buffers start free
+        comp_done[b].record(comp)
+        out_done[b].record(comp)
+    state = {"i": 0}
+
+    def pipelined_step():
+        b = state["i"] % 2
+        state["i"] += 1
+        cin.wait_event(comp_done[b])          # the layer that read xd[b] is done
+        with torch.cuda.stream(cin):
+            xd[b].copy_(xh, non_blocking=True)
+        in_done[b].record(cin)
+        comp.wait_event(in_done[b])
+        comp.wait_event(out_done[b])           # yd[b] has been copied out
+        moe.moe_layer_forward(xd[b], wr, wgu, wd, K=K, y=yd[b], ws=ws)
+        comp_done[b].record(comp)
+        cout.wait_event(comp_done[b])
+        with torch.cuda.stream(cout):
+            yh[b].copy_(yd[b], non_blocking=True)
+        out_done[b].record(cout)
+
+    for _ in range(4):
+        pipelined_step()
+    if pg is not None:
+        pg.barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(comp)
+    for _ in range(steps):
+        pipelined_step()
+    comp.wait_stream(cout)
+    e1.record(comp)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(e0.elapsed_time(e1), pg) / steps
+    return ms_serial, ms
 
 
 def dev_experts(N, d, I, seed, dev):
