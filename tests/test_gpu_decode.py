@@ -120,3 +120,28 @@ def test_layer_decode_sizes(moe, T):
     same = (ref["k"] == r["k"]) & np.all(ref["ids"] == r["ids"], axis=1)
     assert same.sum() >= max(1, int(0.9 * T))
     assert_layer_close(bf16_tensor_to_f64(y)[same], ref["y"][same])
+
+
+@pytest.mark.parametrize("T,N,d,I,K,mode", [(16, 128, 1024, 512, 8, 0), (40, 128, 1024, 512, 8, 1),
+                                            (9, 64, 512, 256, 4, 0), (64, 64, 512, 256, 2, 0)])
+def test_layer_small_batches_shapes(moe, T, N, d, I, K, mode):
+    """Small batches with 128 experts, other caps and top-K mode: the warp
+    router (T <= 16) or the fused router, the decode GEMMs, every token vs the
+    oracle."""
+    import torch
+    inp = synth.layer_inputs(T=T, d=d, N=N, I=I, seed=900 + T + N)
+    ws = torch.empty(moe.layer_workspace_size(T, d, N, I, K), dtype=torch.uint8, device="cuda")
+    y, it = moe.moe_layer_forward(to_dev_bf16(inp["x"]), to_dev_bf16(inp["w_router"]),
+                                  to_dev_bf16(inp["w_gate_up"]), to_dev_bf16(inp["w_down"]), K=K,
+                                  mode=mode, ws=ws, return_intermediates=True)
+    moe.read_device_error(ws)
+    r = oracle.route(it["logits"].cpu().numpy(), K=K, mode=mode)
+    assert np.array_equal(r["k"], it["k"].cpu().numpy())
+    assert np.array_equal(r["ids"], it["ids"].cpu().numpy())
+    assert np.array_equal(r["gates"].view(np.uint32), it["gates"].cpu().numpy().view(np.uint32))
+    rows = np.arange(T)
+    ref = oracle.layer_rows(inp["x"], inp["w_router"], inp["w_gate_up"], inp["w_down"], rows=rows,
+                            K=K, mode=mode)
+    same = (ref["k"] == r["k"]) & np.all(ref["ids"] == r["ids"], axis=1)
+    assert same.sum() >= max(1, int(0.9 * T))
+    assert_layer_close(bf16_tensor_to_f64(y)[same], ref["y"][same])
