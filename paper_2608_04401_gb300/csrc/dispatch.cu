@@ -287,94 +287,168 @@ __global__ void __launch_bounds__(256) gather_kernel(const uint4* __restrict__ x
 }
 
 // y_t = sum_{s<k_t} g_{t,s} * o[pair_pos[t,s]] (+ residual_t); fp32 in s order.
-// One warp per unit: a whole token, or for small batches one slab of a token
-// so that they still spread over many warps. The token's k positions and
-// gates are read per unit (lane s holds pair s) and broadcast by shuffles. A slab is 32 * CH sixteen-byte
-// chunks (lane l holds chunks l + 32c, c < CH; CH = 2 without a residual, 1
-// with one, which keeps both variants at four blocks per SM): the loads of
-// all k rows of a slab (and of the residual) are issued before any is
-// accumulated, so a warp keeps up to 8 KB in flight.
+// One warp per unit: a whole token, or for small batches (SPLIT) one slab of a
+// token so that they still spread over many warps. A slab is 32 * CH
+// sixteen-byte chunks (lane l owns chunks l + 32c, c < CH; CH = 2 without a
+// residual, 1 with one). The k rows of a slab (and the residual) are copied
+// with cp.async into this warp's two-stage shared-memory ring while the
+// previous slab is accumulated, so a warp keeps up to two slabs (16 KB) in
+// flight without holding them in registers. Each lane reads back only the
+// chunks it copied itself, so no barrier is needed between the lanes; the
+// next unit's k, positions and gates are read a unit ahead.
 constexpr int kCombineWarps = 4;
 
+template <bool RES>
+struct CombineCfg {
+  static constexpr int CH = RES ? 1 : 2;
+  static constexpr int kSlabChunks = 32 * CH;
+  static constexpr int kRows = 8 + (RES ? 1 : 0);                 // k rows (+ residual)
+  static constexpr int kStage = kRows * CH * 32;                  // uint4 per stage
+  static constexpr int kWarpBytes = 2 * kStage * 16;              // two stages
+  static constexpr int kBlockBytes = kCombineWarps * kWarpBytes;
+};
+
+MOE_DEV void combine_cp16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src)
+               : "memory");
+}
+
+struct CombineUnit {
+  int64_t t;
+  int s0, s1, kt, pos;
+  float g;
+  bool valid;
+};
+
 template <bool RES, bool SPLIT>
-__global__ void __launch_bounds__(32 * kCombineWarps, 4) combine_kernel(
+__global__ void __launch_bounds__(32 * kCombineWarps) combine_kernel(
     const uint4* __restrict__ o, const int32_t* __restrict__ k, const int32_t* __restrict__ pair_pos,
     const float* __restrict__ gates, const uint4* residual, int64_t T, int d8, int K, uint4* y) {
+  using C = CombineCfg<RES>;
+  constexpr int CH = C::CH;
+  extern __shared__ uint4 cmb_smem[];
   const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x / 32;
+  uint4* ring = cmb_smem + static_cast<size_t>(warp) * 2 * C::kStage;
   const int64_t nwarps = static_cast<int64_t>(gridDim.x) * kCombineWarps;
   const int64_t cap = T * K;
-  constexpr int CH = RES ? 1 : 2;
-  constexpr int kSlabChunks = 32 * CH;
-  // unit = a whole token, or (SPLIT, small batches) one slab of a token
-  const int nslab = (d8 + kSlabChunks - 1) / kSlabChunks;
-  for (int64_t u = static_cast<int64_t>(blockIdx.x) * kCombineWarps + threadIdx.x / 32;
-       u < (SPLIT ? T * nslab : T); u += nwarps) {
-    const int64_t t = SPLIT ? u / nslab : u;
-    const int kt = min(k[t], K);
-    const int my_pos = lane < kt ? static_cast<int>(min_of<int64_t>(max(pair_pos[t * K + lane], 0), cap - 1)) : 0;
-    const float my_g = lane < kt ? gates[t * K + lane] : 0.0f;
-    const int s0 = SPLIT ? static_cast<int>(u % nslab) * kSlabChunks : 0;
-    const int s1 = SPLIT ? s0 + kSlabChunks : d8;
-    for (int slab = s0; slab < s1; slab += kSlabChunks) {
-      uint4 v[8][CH];
+  const int nslab = (d8 + C::kSlabChunks - 1) / C::kSlabChunks;
+  const int64_t units = SPLIT ? T * nslab : T;
+
+  auto unit_at = [&](int64_t u) {
+    CombineUnit m;
+    m.valid = u < units;
+    if (!m.valid) {
+      m.t = 0; m.s0 = m.s1 = 0; m.kt = 0; m.pos = 0; m.g = 0.0f;
+      return m;
+    }
+    m.t = SPLIT ? u / nslab : u;
+    m.s0 = SPLIT ? static_cast<int>(u % nslab) * C::kSlabChunks : 0;
+    m.s1 = SPLIT ? m.s0 + C::kSlabChunks : d8;
+    m.kt = min(k[m.t], K);
+    m.pos = lane < m.kt ? static_cast<int>(min_of<int64_t>(max(pair_pos[m.t * K + lane], 0), cap - 1))
+                        : 0;
+    m.g = lane < m.kt ? gates[m.t * K + lane] : 0.0f;
+    return m;
+  };
+  // copies of one slab of unit m into stage st (rows s >= kt are not read back)
+  auto issue = [&](const CombineUnit& m, int slab, int st) {
+    uint4* b = ring + st * C::kStage;
 #pragma unroll
-      for (int s = 0; s < 8; ++s) {
-        const int p = __shfl_sync(0xffffffffu, my_pos, s);
-        const uint4* row = o + static_cast<int64_t>(p) * d8;
-#pragma unroll
-        for (int c = 0; c < CH; ++c) {
-          const int ci = slab + lane + 32 * c;
-          v[s][c] = (s < kt && ci < d8) ? __ldcs(row + ci) : make_uint4(0, 0, 0, 0);
-        }
-      }
-      uint4 rv[CH];
-#pragma unroll
-      for (int c = 0; c < CH; ++c) {
-        const int ci = slab + lane + 32 * c;
-        rv[c] = (RES && ci < d8) ? __ldcs(residual + t * d8 + ci) : make_uint4(0, 0, 0, 0);
-      }
-      float acc[CH][8];
-#pragma unroll
-      for (int c = 0; c < CH; ++c)
-#pragma unroll
-        for (int u = 0; u < 8; ++u) acc[c][u] = 0.0f;
-#pragma unroll
-      for (int s = 0; s < 8; ++s) {
-        const float g = __shfl_sync(0xffffffffu, my_g, s);
-        if (s < kt) {
-#pragma unroll
-          for (int c = 0; c < CH; ++c) {
-            const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v[s][c]);
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              const float2 f = __bfloat1622float2(h[u]);
-              acc[c][2 * u] = fmaf(g, f.x, acc[c][2 * u]);
-              acc[c][2 * u + 1] = fmaf(g, f.y, acc[c][2 * u + 1]);
-            }
-          }
-        }
-      }
+    for (int s = 0; s < 8; ++s) {
+      const int p = __shfl_sync(0xffffffffu, m.pos, s);
 #pragma unroll
       for (int c = 0; c < CH; ++c) {
         const int ci = slab + lane + 32 * c;
-        if (ci >= d8) continue;
-        if constexpr (RES) {
-          const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&rv[c]);
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const float2 f = __bfloat1622float2(h[u]);
-            acc[c][2 * u] += f.x;
-            acc[c][2 * u + 1] += f.y;
-          }
-        }
-        uint4 out;
-        out.x = pack_bf16x2(acc[c][0], acc[c][1]);
-        out.y = pack_bf16x2(acc[c][2], acc[c][3]);
-        out.z = pack_bf16x2(acc[c][4], acc[c][5]);
-        out.w = pack_bf16x2(acc[c][6], acc[c][7]);
-        y[t * d8 + ci] = out;
+        if (s < m.kt && ci < d8)
+          combine_cp16(b + (s * CH + c) * 32 + lane, o + static_cast<int64_t>(p) * d8 + ci);
       }
     }
+    if constexpr (RES) {
+#pragma unroll
+      for (int c = 0; c < CH; ++c) {
+        const int ci = slab + lane + 32 * c;
+        if (ci < d8) combine_cp16(b + (8 * CH + c) * 32 + lane, residual + m.t * d8 + ci);
+      }
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+
+  int64_t u = static_cast<int64_t>(blockIdx.x) * kCombineWarps + warp;
+  CombineUnit cur = unit_at(u);
+  if (!cur.valid) return;  // uniform per warp
+  CombineUnit nxt = unit_at(u + nwarps);
+  int slab = cur.s0;
+  int st = 0;
+  issue(cur, slab, 0);
+  while (true) {
+    // the next slab: the rest of this unit, else the next unit's first
+    const bool more_here = slab + C::kSlabChunks < cur.s1;
+    if (more_here) {
+      issue(cur, slab + C::kSlabChunks, st ^ 1);
+      asm volatile("cp.async.wait_group 1;" ::: "memory");
+    } else if (nxt.valid) {
+      issue(nxt, nxt.s0, st ^ 1);
+      asm volatile("cp.async.wait_group 1;" ::: "memory");
+    } else {
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
+    }
+    // accumulate this slab from the ring, in s order
+    const uint4* b = ring + st * C::kStage;
+    float acc[CH][8];
+#pragma unroll
+    for (int c = 0; c < CH; ++c)
+#pragma unroll
+      for (int q = 0; q < 8; ++q) acc[c][q] = 0.0f;
+#pragma unroll
+    for (int s = 0; s < 8; ++s) {
+      const float g = __shfl_sync(0xffffffffu, cur.g, s);
+      if (s < cur.kt) {
+#pragma unroll
+        for (int c = 0; c < CH; ++c) {
+          const uint4 v = b[(s * CH + c) * 32 + lane];
+          const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            const float2 f = __bfloat1622float2(h[q]);
+            acc[c][2 * q] = fmaf(g, f.x, acc[c][2 * q]);
+            acc[c][2 * q + 1] = fmaf(g, f.y, acc[c][2 * q + 1]);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int c = 0; c < CH; ++c) {
+      const int ci = slab + lane + 32 * c;
+      if (ci >= d8) continue;
+      if constexpr (RES) {
+        const uint4 rv = b[(8 * CH + c) * 32 + lane];
+        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&rv);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float2 f = __bfloat1622float2(h[q]);
+          acc[c][2 * q] += f.x;
+          acc[c][2 * q + 1] += f.y;
+        }
+      }
+      uint4 out;
+      out.x = pack_bf16x2(acc[c][0], acc[c][1]);
+      out.y = pack_bf16x2(acc[c][2], acc[c][3]);
+      out.z = pack_bf16x2(acc[c][4], acc[c][5]);
+      out.w = pack_bf16x2(acc[c][6], acc[c][7]);
+      y[cur.t * d8 + ci] = out;
+    }
+    // advance
+    if (more_here) {
+      slab += C::kSlabChunks;
+    } else {
+      if (!nxt.valid) break;
+      cur = nxt;
+      slab = cur.s0;
+      u += nwarps;
+      nxt = unit_at(u + nwarps);
+    }
+    st ^= 1;
   }
 }
 
@@ -469,12 +543,30 @@ cudaError_t launch_combine(const uint16_t* o, const int32_t* k, const int32_t* p
   // whole tokens per warp once the batch alone fills the GPU; slabs otherwise
   const bool split = T < static_cast<int64_t>(num_sms) * 16;
   const int64_t units = split ? T * nslab : T;
-  int64_t blocks = (units + disp::kCombineWarps - 1) / disp::kCombineWarps;
-  const int64_t cap = static_cast<int64_t>(num_sms) * 16;
-  if (blocks > cap) blocks = cap;
+  const int smem = residual ? disp::CombineCfg<true>::kBlockBytes : disp::CombineCfg<false>::kBlockBytes;
   auto kern = residual ? (split ? disp::combine_kernel<true, true> : disp::combine_kernel<true, false>)
                        : (split ? disp::combine_kernel<false, true> : disp::combine_kernel<false, false>);
-  kern<<<static_cast<unsigned>(blocks), 32 * disp::kCombineWarps, 0, stream>>>(
+  static int attr_dev = -1;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (attr_dev != dev) {
+    for (auto f : {disp::combine_kernel<true, true>, disp::combine_kernel<true, false>,
+                   disp::combine_kernel<false, true>, disp::combine_kernel<false, false>}) {
+      cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           disp::CombineCfg<false>::kBlockBytes);
+      if (e != cudaSuccess) return e;
+    }
+    attr_dev = dev;
+  }
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 32 * disp::kCombineWarps, smem) !=
+          cudaSuccess ||
+      per_sm < 1)
+    per_sm = 1;
+  int64_t blocks = (units + disp::kCombineWarps - 1) / disp::kCombineWarps;
+  const int64_t cap = static_cast<int64_t>(num_sms) * per_sm;
+  if (blocks > cap) blocks = cap;
+  kern<<<static_cast<unsigned>(blocks), 32 * disp::kCombineWarps, smem, stream>>>(
       reinterpret_cast<const uint4*>(o), k, pair_pos, gates,
       reinterpret_cast<const uint4*>(residual), T, d / 8, K, reinterpret_cast<uint4*>(y));
   return cudaGetLastError();
