@@ -46,8 +46,10 @@ cudaError_t launch_down_decode_gemm(const uint16_t* h, const uint16_t* wd, const
 cudaError_t launch_route_warp(const float* src, int nslice, int64_t T, int N, int K, float eps,
                               int topk_mode, int renorm, float* logits_out, int32_t* k_out,
                               int32_t* ids_out, float* gates_out, cudaStream_t stream);
-cudaError_t launch_router_small(const uint16_t* x, const uint16_t* w_router, int T, int d, int N,
-                                float* partial, cudaStream_t stream);
+cudaError_t launch_router_small_route(const uint16_t* x, const uint16_t* w_router, int T, int d,
+                                      int N, float* partial, unsigned int* ticket, int K, float eps,
+                                      int topk_mode, int renorm, float* logits_out, int32_t* k_out,
+                                      int32_t* ids_out, float* gates_out, cudaStream_t stream);
 cudaError_t launch_route_diagnostics(const float* logits, int64_t T, int N, int K, float eps,
                                      int32_t* elbow_out, float* theta_out, moe_route_diag* dg,
                                      cudaStream_t stream);
@@ -328,8 +330,9 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   LayerWs w = layer_ws(ws, T, d, N, I, K);
   if (ws_bytes < w.bytes) return MOE_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  // clear the device error word first, so that a no-op call reads clean
-  if (cudaMemsetAsync(w.err, 0, sizeof(int32_t), s) != cudaSuccess) return MOE_ERR_CUDA;
+  // clear the device error word (and the small-batch router's ticket counter
+  // beside it) first, so that a no-op call reads clean
+  if (cudaMemsetAsync(w.err, 0, 2 * sizeof(int32_t), s) != cudaSuccess) return MOE_ERR_CUDA;
   if (T == 0) return MOE_OK;
   const void* need[] = {x, w_router, w_gate_up, w_down, y};
   for (const void* p : need)
@@ -351,10 +354,10 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   if (T <= kWarpRouteMaxTokens) {
     // a few tokens: the router GEMM split over d on every SM, then one warp per
     // token routes (the single-chunk dispatch counts the pairs itself)
-    e = moe::launch_router_small(x, w_router, static_cast<int>(T), d, N, w.partial, s);
-    if (e != cudaSuccess) return MOE_ERR_CUDA;
-    e = moe::launch_route_warp(w.partial, d / 64, T, N, K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
-                               rp->renorm, logits_out, kk, ids, gates, s);
+    e = moe::launch_router_small_route(x, w_router, static_cast<int>(T), d, N, w.partial,
+                                       reinterpret_cast<unsigned int*>(w.err + 1), K, rp->eps,
+                                       rp->mode == MOE_ROUTE_TOPK, rp->renorm, logits_out, kk, ids,
+                                       gates, s);
   } else {
     // router GEMM with the elbow routing in its epilogue; it also leaves the
     // per-chunk expert counts of the dispatch

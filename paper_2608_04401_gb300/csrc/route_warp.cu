@@ -14,10 +14,11 @@
 // The logits may arrive as `nslice` partial sums (the small-batch router GEMM
 // splits d); they are added in slice order.
 //
-// router_small_kernel: the router GEMM for T <= 64 tokens on CUDA cores, split
-// over d in slices of 64 columns (one block per slice) so that every SM
-// streams a slice of x and W_r instead of one SM streaming them all:
-// partial[s][t][e] = sum_{k in slice s} x[t][k] w[e][k], fp32 fma in k order.
+// router_small_route_kernel: the router GEMM for T <= 64 tokens on CUDA cores,
+// split over d in slices of 64 columns (one block per slice) so that many SMs
+// stream a slice of x and W_r instead of one SM streaming them all:
+// partial[s][t][e] = sum_{k in slice s} x[t][k] w[e][k], fp32 fma in k order;
+// the block that finishes last routes every token (slices added in order).
 #include "route_impl.cuh"
 
 namespace moe {
@@ -31,10 +32,8 @@ constexpr int kSmallT = 64;      // largest batch of the small router GEMM
 constexpr int kPitch2 = kSlice / 2 + 1;  // row pitch in bf16 pairs (odd: no bank conflicts)
 
 template <int N>
-__global__ void __launch_bounds__(256) router_small_kernel(const uint32_t* __restrict__ x,
-                                                            const uint32_t* __restrict__ w,
-                                                            int T, int d,
-                                                            float* __restrict__ partial) {
+MOE_DEV void router_small_body(const uint32_t* __restrict__ x, const uint32_t* __restrict__ w, int T,
+                               int d, float* __restrict__ partial) {
   __shared__ uint32_t xs[kSmallT][kPitch2];  // bf16 pairs
   __shared__ uint32_t wsm[N][kPitch2];
   const int s = blockIdx.x;
@@ -73,16 +72,18 @@ __global__ void __launch_bounds__(256) router_small_kernel(const uint32_t* __res
   }
 }
 
-template <int N>
-__global__ void __launch_bounds__(32 * kWarps) route_warp_kernel(
-    const float* __restrict__ src, int64_t T, int nslice, int K, float eps, int topk_mode,
-    int renorm, float* __restrict__ logits_out, int32_t* __restrict__ k_out,
-    int32_t* __restrict__ ids_out, float* __restrict__ gates_out) {
+// Routes token t with the calling (whole, converged) warp. src holds the
+// logits as nslice partial sums [nslice][T][N] (nslice = 1: the logits); with
+// L2_ONLY they are read past L1 (written by other blocks of the same launch).
+template <int N, bool L2_ONLY>
+MOE_DEV void route_one_warp(const float* __restrict__ src, int64_t t, int64_t T, int nslice, int K,
+                            float eps, int topk_mode, int renorm, float* __restrict__ logits_out,
+                            int32_t* __restrict__ k_out, int32_t* __restrict__ ids_out,
+                            float* __restrict__ gates_out) {
   constexpr int C = N / 32;
   const unsigned full = 0xffffffffu;
   const int lane = threadIdx.x & 31;
-  const int64_t t = static_cast<int64_t>(blockIdx.x) * kWarps + threadIdx.x / 32;
-  if (t >= T) return;  // uniform per warp
+  auto ld = [&](int64_t i) { return L2_ONLY ? __ldcg(src + i) : src[i]; };
 
   // logits, slices added in order
   float l[C];
@@ -90,17 +91,17 @@ __global__ void __launch_bounds__(32 * kWarps) route_warp_kernel(
   for (int c = 0; c < C; ++c) {
     const int64_t off = t * N + 32 * c + lane;
     const int64_t stride = T * N;
-    float a = src[off];
+    float a = ld(off);
     int s = 1;
     // eight slices' loads in flight at a time; the sum stays in slice order
     for (; s + 8 <= nslice; s += 8) {
       float q[8];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) q[u] = src[(s + u) * stride + off];
+      for (int u = 0; u < 8; ++u) q[u] = ld((s + u) * stride + off);
 #pragma unroll
       for (int u = 0; u < 8; ++u) a = __fadd_rn(a, q[u]);
     }
-    for (; s < nslice; ++s) a = __fadd_rn(a, src[s * stride + off]);
+    for (; s < nslice; ++s) a = __fadd_rn(a, ld(s * stride + off));
     l[c] = a;
     if (logits_out) logits_out[off] = a;
   }
@@ -214,6 +215,41 @@ __global__ void __launch_bounds__(32 * kWarps) route_warp_kernel(
   if (lane == 0) k_out[t] = k;
 }
 
+template <int N>
+__global__ void __launch_bounds__(32 * kWarps) route_warp_kernel(
+    const float* __restrict__ src, int64_t T, int nslice, int K, float eps, int topk_mode,
+    int renorm, float* __restrict__ logits_out, int32_t* __restrict__ k_out,
+    int32_t* __restrict__ ids_out, float* __restrict__ gates_out) {
+  const int64_t t = static_cast<int64_t>(blockIdx.x) * kWarps + threadIdx.x / 32;
+  if (t >= T) return;  // uniform per warp
+  route_one_warp<N, false>(src, t, T, nslice, K, eps, topk_mode, renorm, logits_out, k_out,
+                           ids_out, gates_out);
+}
+
+// The small-batch router in one launch: every block writes its slice's
+// partial sums; the block that finishes last (a ticket counter, after a
+// memory fence: no block waits for another) routes all T tokens with its
+// eight warps, reading the partials from L2, and resets the counter.
+template <int N>
+__global__ void __launch_bounds__(256) router_small_route_kernel(
+    const uint32_t* __restrict__ x, const uint32_t* __restrict__ w, int T, int d,
+    float* __restrict__ partial, unsigned int* __restrict__ ticket, int K, float eps, int topk_mode,
+    int renorm, float* __restrict__ logits_out, int32_t* __restrict__ k_out,
+    int32_t* __restrict__ ids_out, float* __restrict__ gates_out) {
+  router_small_body<N>(x, w, T, d, partial);
+  __threadfence();
+  __syncthreads();
+  __shared__ bool last;
+  if (threadIdx.x == 0) last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  for (int t = threadIdx.x / 32; t < T; t += 8)
+    route_one_warp<N, true>(partial, t, T, static_cast<int>(gridDim.x), K, eps, topk_mode, renorm,
+                            logits_out, k_out, ids_out, gates_out);
+  if (threadIdx.x == 0) *ticket = 0u;
+}
+
 }  // namespace rwarp
 
 // Warp-per-token routing of fp32 logits [T, N] (or of `nslice` partial sums
@@ -232,19 +268,24 @@ cudaError_t launch_route_warp(const float* src, int nslice, int64_t T, int N, in
   return cudaGetLastError();
 }
 
-// Router logits of T <= 64 tokens as d / 64 partial sums: partial [d/64][T][N].
-cudaError_t launch_router_small(const uint16_t* x, const uint16_t* w_router, int T, int d, int N,
-                                float* partial, cudaStream_t stream) {
+// Router logits of T <= 64 tokens (as d / 64 partial sums, partial [d/64][T][N])
+// and their routing, in one launch; ticket: a zeroed device counter, left zero.
+cudaError_t launch_router_small_route(const uint16_t* x, const uint16_t* w_router, int T, int d,
+                                      int N, float* partial, unsigned int* ticket, int K, float eps,
+                                      int topk_mode, int renorm, float* logits_out, int32_t* k_out,
+                                      int32_t* ids_out, float* gates_out, cudaStream_t stream) {
   if (T == 0) return cudaSuccess;
   const unsigned slices = static_cast<unsigned>(d / rwarp::kSlice);
+  auto xx = reinterpret_cast<const uint32_t*>(x);
+  auto ww = reinterpret_cast<const uint32_t*>(w_router);
   if (N == 64)
-    rwarp::router_small_kernel<64><<<slices, 256, 0, stream>>>(
-        reinterpret_cast<const uint32_t*>(x), reinterpret_cast<const uint32_t*>(w_router), T, d,
-        partial);
+    rwarp::router_small_route_kernel<64><<<slices, 256, 0, stream>>>(
+        xx, ww, T, d, partial, ticket, K, eps, topk_mode, renorm, logits_out, k_out, ids_out,
+        gates_out);
   else
-    rwarp::router_small_kernel<128><<<slices, 256, 0, stream>>>(
-        reinterpret_cast<const uint32_t*>(x), reinterpret_cast<const uint32_t*>(w_router), T, d,
-        partial);
+    rwarp::router_small_route_kernel<128><<<slices, 256, 0, stream>>>(
+        xx, ww, T, d, partial, ticket, K, eps, topk_mode, renorm, logits_out, k_out, ids_out,
+        gates_out);
   return cudaGetLastError();
 }
 
