@@ -95,8 +95,9 @@ moe_status elbow_route(const float* logits, int64_t T, int N, const moe_route_pa
  * shuffles and the argmax is a warp reduction. Same specification, same bits
  * as elbow_route; a much shorter critical path per token, at about three
  * times the instructions per token, so elbow_route uses it by itself for
- * T <= 16 (and moe_layer_forward's router for T <= 16). Arguments and errors
- * as elbow_route (ids_out and gates_out need only 4-byte alignment). */
+ * T <= 16 (and moe_layer_forward's router, after a router GEMM split over d
+ * and 16-token groups, for T <= 64). Arguments and errors as elbow_route
+ * (ids_out and gates_out need only 4-byte alignment). */
 moe_status elbow_route_warp(const float* logits, int64_t T, int N, const moe_route_params* rp,
                             int32_t* k_out, int32_t* ids_out, float* gates_out, void* stream);
 

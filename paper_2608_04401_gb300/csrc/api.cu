@@ -43,9 +43,9 @@ cudaError_t launch_gateup_decode_gemm(const uint16_t* xs, const uint16_t* wgu,
 cudaError_t launch_down_decode_gemm(const uint16_t* h, const uint16_t* wd, const int32_t* offsets,
                                     int64_t P, int d, int N, int I, uint16_t* o, int32_t* err,
                                     int num_sms, cudaStream_t stream);
-cudaError_t launch_route_warp(const float* src, int nslice, int64_t T, int N, int K, float eps,
-                              int topk_mode, int renorm, float* logits_out, int32_t* k_out,
-                              int32_t* ids_out, float* gates_out, cudaStream_t stream);
+cudaError_t launch_route_warp(const float* logits, int64_t T, int N, int K, float eps,
+                              int topk_mode, int renorm, int32_t* k_out, int32_t* ids_out,
+                              float* gates_out, cudaStream_t stream);
 cudaError_t launch_router_small_route(const uint16_t* x, const uint16_t* w_router, int T, int d,
                                       int N, float* partial, unsigned int* ticket, int K, float eps,
                                       int topk_mode, int renorm, float* logits_out, int32_t* k_out,
@@ -82,6 +82,13 @@ constexpr int64_t kDecodeMaxTokens = 64;
 // router GEMM split over d (below it the fused router's one-thread-per-token
 // routing chain dominates; above it the fused router is faster).
 constexpr int64_t kWarpRouteMaxTokens = 16;
+// Layer batches of at most this many tokens take the router GEMM split over d
+// and over 16-token groups (each block a 64-column slice of one group; the
+// last block of a group routes it, one warp per token) instead of the
+// tensor-core router, whose single 128-row tile would stream all of x and W_r
+// through one SM.
+constexpr int64_t kSmallRouterMaxTokens = 64;
+constexpr int kSmallRouterSlice = 64;
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -148,7 +155,9 @@ LayerWs layer_ws(void* base, int64_t T, int d, int N, int I, int K) {
   w.h = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * P * I));
   w.o = reinterpret_cast<uint16_t*>(take(sizeof(uint16_t) * P * d));
   w.partial = reinterpret_cast<float*>(
-      take(T <= kWarpRouteMaxTokens ? sizeof(float) * static_cast<size_t>(d / 64) * T * N : 0));
+      take(T <= kSmallRouterMaxTokens
+               ? sizeof(float) * static_cast<size_t>(d / kSmallRouterSlice) * T * N
+               : 0));
   w.bytes = off;
   return w;
 }
@@ -181,9 +190,9 @@ moe_status elbow_route(const float* logits, int64_t T, int N, const moe_route_pa
       (reinterpret_cast<uintptr_t>(k_out) & 3u))
     return MOE_ERR_INVALID_ARG;
   if (T <= kWarpRouteMaxTokens)  // a few tokens: one warp each has the shorter critical path
-    return cuda_status(moe::launch_route_warp(logits, 1, T, N, rp->K, rp->eps,
-                                              rp->mode == MOE_ROUTE_TOPK, rp->renorm, nullptr,
-                                              k_out, ids_out, gates_out,
+    return cuda_status(moe::launch_route_warp(logits, T, N, rp->K, rp->eps,
+                                              rp->mode == MOE_ROUTE_TOPK, rp->renorm, k_out,
+                                              ids_out, gates_out,
                                               static_cast<cudaStream_t>(stream)));
   return cuda_status(moe::launch_elbow_route(logits, T, N, rp->K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
                                              rp->renorm, k_out, ids_out, gates_out, nullptr,
@@ -201,9 +210,9 @@ moe_status elbow_route_warp(const float* logits, int64_t T, int N, const moe_rou
   if (!aligned16(logits) || (reinterpret_cast<uintptr_t>(ids_out) & 3u) ||
       (reinterpret_cast<uintptr_t>(gates_out) & 3u) || (reinterpret_cast<uintptr_t>(k_out) & 3u))
     return MOE_ERR_INVALID_ARG;
-  return cuda_status(moe::launch_route_warp(logits, 1, T, N, rp->K, rp->eps,
-                                            rp->mode == MOE_ROUTE_TOPK, rp->renorm, nullptr, k_out,
-                                            ids_out, gates_out, static_cast<cudaStream_t>(stream)));
+  return cuda_status(moe::launch_route_warp(logits, T, N, rp->K, rp->eps,
+                                            rp->mode == MOE_ROUTE_TOPK, rp->renorm, k_out, ids_out,
+                                            gates_out, static_cast<cudaStream_t>(stream)));
 }
 
 moe_status elbow_route_randomized(const float* logits, int64_t T, int N, const moe_route_params* rp,
@@ -330,9 +339,9 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   LayerWs w = layer_ws(ws, T, d, N, I, K);
   if (ws_bytes < w.bytes) return MOE_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  // clear the device error word (and the small-batch router's ticket counter
-  // beside it) first, so that a no-op call reads clean
-  if (cudaMemsetAsync(w.err, 0, 2 * sizeof(int32_t), s) != cudaSuccess) return MOE_ERR_CUDA;
+  // clear the device error word (and the small-batch router's four group
+  // tickets beside it) first, so that a no-op call reads clean
+  if (cudaMemsetAsync(w.err, 0, 8 * sizeof(int32_t), s) != cudaSuccess) return MOE_ERR_CUDA;
   if (T == 0) return MOE_OK;
   const void* need[] = {x, w_router, w_gate_up, w_down, y};
   for (const void* p : need)
@@ -351,8 +360,8 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   const int nsm = sm_count();
 
   cudaError_t e;
-  if (T <= kWarpRouteMaxTokens) {
-    // a few tokens: the router GEMM split over d on every SM, then one warp per
+  if (T <= kSmallRouterMaxTokens) {
+    // a few tokens: the router GEMM split over d on many SMs, then one warp per
     // token routes (the single-chunk dispatch counts the pairs itself)
     e = moe::launch_router_small_route(x, w_router, static_cast<int>(T), d, N, w.partial,
                                        reinterpret_cast<unsigned int*>(w.err + 1), K, rp->eps,

@@ -11,12 +11,11 @@
 //   shuffles), which orders by p descending and ascending id on ties;
 //   p'_i, D_i on each rank, the first argmax by a (max D, min index) warp
 //   reduction, k = min(e + 1, K).
-// The logits may arrive as `nslice` partial sums (the small-batch router GEMM
-// splits d); they are added in slice order.
 //
 // router_small_route_kernel: the router GEMM for T <= 64 tokens on CUDA cores,
-// split over d in slices of 64 columns (one block per slice) so that many SMs
-// stream a slice of x and W_r instead of one SM streaming them all:
+// split over d in slices of 64 columns and over tokens in groups of 16 (one
+// block per slice and group) so that many SMs share the work instead of one
+// SM streaming all of x and W_r:
 // partial[s][t][e] = sum_{k in slice s} x[t][k] w[e][k], fp32 fma in k order;
 // the block that finishes last routes every token (slices added in order).
 #include "route_impl.cuh"
@@ -24,87 +23,97 @@
 namespace moe {
 namespace rwarp {
 
-using route::RouteConsts;
-
-constexpr int kWarps = 4;        // tokens per block of the routing kernel
-constexpr int kSlice = 64;       // d columns per block of the small router GEMM
-constexpr int kSmallT = 64;      // largest batch of the small router GEMM
+constexpr int kWarps = 4;            // tokens per block of the routing kernel
+constexpr int kSlice = 64;           // d columns per block of the small router GEMM
+constexpr int kGroupT = 16;          // tokens per block of the small router GEMM
+constexpr int kSmallT = 64;          // largest batch of the small router
+constexpr int kSmallThreads = 512;   // threads per block of the small router (16 warps)
 constexpr int kPitch2 = kSlice / 2 + 1;  // row pitch in bf16 pairs (odd: no bank conflicts)
 
-template <int N>
-MOE_DEV void router_small_body(const uint32_t* __restrict__ x, const uint32_t* __restrict__ w, int T,
-                               int d, float* __restrict__ partial) {
-  __shared__ uint32_t xs[kSmallT][kPitch2];  // bf16 pairs
-  __shared__ uint32_t wsm[N][kPitch2];
-  const int s = blockIdx.x;
-  const int d2 = d / 2;
-  const int c0 = s * (kSlice / 2);
-  for (int i = threadIdx.x; i < kSmallT * (kSlice / 2); i += 256) {
-    const int r = i / (kSlice / 2), c = i % (kSlice / 2);
-    xs[r][c] = r < T ? x[static_cast<int64_t>(r) * d2 + c0 + c] : 0u;
-  }
-  for (int i = threadIdx.x; i < N * (kSlice / 2); i += 256) {
-    const int r = i / (kSlice / 2), c = i % (kSlice / 2);
-    wsm[r][c] = w[static_cast<int64_t>(r) * d2 + c0 + c];
-  }
-  __syncthreads();
-  constexpr int kGroups = 256 / N;             // token groups
-  constexpr int kTpg = kSmallT / kGroups;      // tokens per group
-  const int e = threadIdx.x % N, g = threadIdx.x / N;
-  float acc[kTpg];
+// acc[i] = sum over the slice's columns of x[t_i] w[e], t_i = g + G * i, fp32
+// fma in column order (xs, wrow: bf16 pairs in shared memory).
+template <int NT, int G>
+MOE_DEV void slice_dots(const uint32_t (*xs)[kPitch2], const uint32_t* wrow, int g,
+                        float (&acc)[NT]) {
 #pragma unroll
-  for (int i = 0; i < kTpg; ++i) acc[i] = 0.0f;
-#pragma unroll 4
+  for (int i = 0; i < NT; ++i) acc[i] = 0.0f;
+#pragma unroll 8
   for (int c = 0; c < kSlice / 2; ++c) {
-    const float2 wv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&wsm[e][c]));
+    const float2 wv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&wrow[c]));
 #pragma unroll
-    for (int i = 0; i < kTpg; ++i) {
+    for (int i = 0; i < NT; ++i) {
       const float2 xv =
-          __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xs[g * kTpg + i][c]));
+          __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&xs[g + G * i][c]));
       acc[i] = fmaf(xv.x, wv.x, acc[i]);
       acc[i] = fmaf(xv.y, wv.y, acc[i]);
     }
   }
+}
+
+// Thread (e, g) of G = kSmallThreads / N groups: the partial sums of its NT
+// tokens g, g + G, ... of the block's token group (NT is the thread's token
+// count as a compile-time constant, so that no accumulator idles).
+template <int N, int NT>
+MOE_DEV void slice_tokens(const uint32_t (*xs)[kPitch2], const uint32_t* wrow, int g, int e,
+                          float* __restrict__ out) {
+  constexpr int G = kSmallThreads / N;
+  float acc[NT];
+  slice_dots<NT, G>(xs, wrow, g, acc);
 #pragma unroll
-  for (int i = 0; i < kTpg; ++i) {
-    const int t = g * kTpg + i;
-    if (t < T) partial[(static_cast<int64_t>(s) * T + t) * N + e] = acc[i];
+  for (int i = 0; i < NT; ++i) out[(g + G * i) * N + e] = acc[i];
+}
+
+// Block (s, j): the partial sums of tokens t0 = 16 j .. t0 + nj - 1 over the
+// d columns [64 s, 64 s + 64): partial[s][t0 + r][e].
+template <int N>
+MOE_DEV void router_small_body(const uint32_t* __restrict__ x, const uint32_t* __restrict__ w, int T,
+                               int d, int t0, int nj, float* __restrict__ partial) {
+  __shared__ uint32_t xs[kGroupT][kPitch2];  // bf16 pairs
+  __shared__ uint32_t wsm[N][kPitch2];
+  const int s = blockIdx.x;
+  const int d2 = d / 2;
+  const int c0 = s * (kSlice / 2);
+  // 16-byte loads (four bf16 pairs), stored as single pairs into the odd pitch
+  constexpr int kVec = kSlice / 8;  // uint4 per row slice
+  for (int i = threadIdx.x; i < (nj + N) * kVec; i += kSmallThreads) {
+    const int r = i / kVec, c = (i % kVec) * 4;
+    const bool is_x = r < nj;
+    const uint32_t* src = is_x ? x + static_cast<int64_t>(t0 + r) * d2
+                               : w + static_cast<int64_t>(r - nj) * d2;
+    const uint4 v = *reinterpret_cast<const uint4*>(src + c0 + c);
+    uint32_t* dst = is_x ? &xs[r][c] : &wsm[r - nj][c];
+    dst[0] = v.x; dst[1] = v.y; dst[2] = v.z; dst[3] = v.w;
+  }
+  __syncthreads();
+  constexpr int G = kSmallThreads / N;
+  const int e = threadIdx.x % N, g = threadIdx.x / N;
+  if (g >= nj) return;  // whole warps (N >= 64)
+  const int nt = (nj - g + G - 1) / G;  // 1 .. kGroupT / G
+  float* out = partial + (static_cast<int64_t>(s) * T + t0) * N;
+  switch (nt) {
+    case 1: slice_tokens<N, 1>(xs, wsm[e], g, e, out); break;
+    case 2: slice_tokens<N, 2>(xs, wsm[e], g, e, out); break;
+    default:
+      if constexpr (kGroupT / G > 2) {
+        if (nt == 3) slice_tokens<N, 3>(xs, wsm[e], g, e, out);
+        else slice_tokens<N, 4>(xs, wsm[e], g, e, out);
+      }
   }
 }
 
-// Routes token t with the calling (whole, converged) warp. src holds the
-// logits as nslice partial sums [nslice][T][N] (nslice = 1: the logits); with
-// L2_ONLY they are read past L1 (written by other blocks of the same launch).
-template <int N, bool L2_ONLY>
-MOE_DEV void route_one_warp(const float* __restrict__ src, int64_t t, int64_t T, int nslice, int K,
-                            float eps, int topk_mode, int renorm, float* __restrict__ logits_out,
-                            int32_t* __restrict__ k_out, int32_t* __restrict__ ids_out,
-                            float* __restrict__ gates_out) {
+// Routes token t with the calling (whole, converged) warp from its logits
+// row[0 .. N) (global or shared memory).
+template <int N>
+MOE_DEV void route_one_warp(const float* __restrict__ row, int64_t t, int K, float eps,
+                            int topk_mode, int renorm, int32_t* __restrict__ k_out,
+                            int32_t* __restrict__ ids_out, float* __restrict__ gates_out) {
   constexpr int C = N / 32;
   const unsigned full = 0xffffffffu;
   const int lane = threadIdx.x & 31;
-  auto ld = [&](int64_t i) { return L2_ONLY ? __ldcg(src + i) : src[i]; };
 
-  // logits, slices added in order
   float l[C];
 #pragma unroll
-  for (int c = 0; c < C; ++c) {
-    const int64_t off = t * N + 32 * c + lane;
-    const int64_t stride = T * N;
-    float a = ld(off);
-    int s = 1;
-    // eight slices' loads in flight at a time; the sum stays in slice order
-    for (; s + 8 <= nslice; s += 8) {
-      float q[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) q[u] = ld((s + u) * stride + off);
-#pragma unroll
-      for (int u = 0; u < 8; ++u) a = __fadd_rn(a, q[u]);
-    }
-    for (; s < nslice; ++s) a = __fadd_rn(a, ld(s * stride + off));
-    l[c] = a;
-    if (logits_out) logits_out[off] = a;
-  }
+  for (int c = 0; c < C; ++c) l[c] = row[32 * c + lane];
   float m = l[0];
 #pragma unroll
   for (int c = 1; c < C; ++c) m = fmaxf(m, l[c]);
@@ -217,75 +226,110 @@ MOE_DEV void route_one_warp(const float* __restrict__ src, int64_t t, int64_t T,
 
 template <int N>
 __global__ void __launch_bounds__(32 * kWarps) route_warp_kernel(
-    const float* __restrict__ src, int64_t T, int nslice, int K, float eps, int topk_mode,
-    int renorm, float* __restrict__ logits_out, int32_t* __restrict__ k_out,
-    int32_t* __restrict__ ids_out, float* __restrict__ gates_out) {
+    const float* __restrict__ logits, int64_t T, int K, float eps, int topk_mode, int renorm,
+    int32_t* __restrict__ k_out, int32_t* __restrict__ ids_out, float* __restrict__ gates_out) {
   const int64_t t = static_cast<int64_t>(blockIdx.x) * kWarps + threadIdx.x / 32;
   if (t >= T) return;  // uniform per warp
-  route_one_warp<N, false>(src, t, T, nslice, K, eps, topk_mode, renorm, logits_out, k_out,
-                           ids_out, gates_out);
+  route_one_warp<N>(logits + t * N, t, K, eps, topk_mode, renorm, k_out, ids_out, gates_out);
 }
 
-// The small-batch router in one launch: every block writes its slice's
-// partial sums; the block that finishes last (a ticket counter, after a
-// memory fence: no block waits for another) routes all T tokens with its
-// eight warps, reading the partials from L2, and resets the counter.
+// The small-batch router in one launch: block (s, j) writes the partial sums
+// of slice s for token group j; the block of group j that finishes last (a
+// ticket counter per group, after a memory fence: no block waits for
+// another) adds them up in slice order with all its threads (two pairs'
+// loads in flight per thread), keeps the group's logits in shared memory,
+// routes its tokens with one warp each and resets the counter.
 template <int N>
-__global__ void __launch_bounds__(256) router_small_route_kernel(
+__global__ void __launch_bounds__(kSmallThreads) router_small_route_kernel(
     const uint32_t* __restrict__ x, const uint32_t* __restrict__ w, int T, int d,
     float* __restrict__ partial, unsigned int* __restrict__ ticket, int K, float eps, int topk_mode,
     int renorm, float* __restrict__ logits_out, int32_t* __restrict__ k_out,
     int32_t* __restrict__ ids_out, float* __restrict__ gates_out) {
-  router_small_body<N>(x, w, T, d, partial);
+  __shared__ float lg[kGroupT * N];
+  __shared__ bool last;
+  const int t0 = blockIdx.y * kGroupT;
+  const int nj = min(kGroupT, T - t0);
+  router_small_body<N>(x, w, T, d, t0, nj, partial);
   __threadfence();
   __syncthreads();
-  __shared__ bool last;
-  if (threadIdx.x == 0) last = atomicAdd(ticket, 1u) == gridDim.x - 1;
+  if (threadIdx.x == 0) last = atomicAdd(ticket + blockIdx.y, 1u) == gridDim.x - 1;
   __syncthreads();
   if (!last) return;
   __threadfence();
-  for (int t = threadIdx.x / 32; t < T; t += 8)
-    route_one_warp<N, true>(partial, t, T, static_cast<int>(gridDim.x), K, eps, topk_mode, renorm,
-                            logits_out, k_out, ids_out, gates_out);
-  if (threadIdx.x == 0) *ticket = 0u;
+  const int nslice = static_cast<int>(gridDim.x);
+  const int64_t stride = static_cast<int64_t>(T) * N;
+  const float* src = partial + static_cast<int64_t>(t0) * N;
+  float* dst = logits_out ? logits_out + static_cast<int64_t>(t0) * N : nullptr;
+  const int npair = nj * N;
+  auto sum_slices = [&](int i0, int i1) {  // pairs i0 and i1 (i1 may be past the end)
+    const bool two = i1 < npair;
+    float a0 = __ldcg(src + i0), a1 = two ? __ldcg(src + i1) : 0.0f;
+    int sl = 1;
+    for (; sl + 16 <= nslice; sl += 16) {
+      float q0[16], q1[16];
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        q0[u] = __ldcg(src + (sl + u) * stride + i0);
+        q1[u] = two ? __ldcg(src + (sl + u) * stride + i1) : 0.0f;
+      }
+#pragma unroll
+      for (int u = 0; u < 16; ++u) {
+        a0 = __fadd_rn(a0, q0[u]);
+        a1 = __fadd_rn(a1, q1[u]);
+      }
+    }
+    for (; sl < nslice; ++sl) {
+      a0 = __fadd_rn(a0, __ldcg(src + sl * stride + i0));
+      if (two) a1 = __fadd_rn(a1, __ldcg(src + sl * stride + i1));
+    }
+    lg[i0] = a0;
+    if (dst) dst[i0] = a0;
+    if (two) {
+      lg[i1] = a1;
+      if (dst) dst[i1] = a1;
+    }
+  };
+  for (int i = threadIdx.x; i < npair; i += 2 * kSmallThreads) sum_slices(i, i + kSmallThreads);
+  __syncthreads();
+  const int wp = threadIdx.x / 32;
+  if (wp < nj)
+    route_one_warp<N>(lg + wp * N, t0 + wp, K, eps, topk_mode, renorm, k_out, ids_out, gates_out);
+  if (threadIdx.x == 0) ticket[blockIdx.y] = 0u;
 }
 
 }  // namespace rwarp
 
-// Warp-per-token routing of fp32 logits [T, N] (or of `nslice` partial sums
-// of them, [nslice][T][N]); logits_out (nullable) receives the summed logits.
-cudaError_t launch_route_warp(const float* src, int nslice, int64_t T, int N, int K, float eps,
-                              int topk_mode, int renorm, float* logits_out, int32_t* k_out,
-                              int32_t* ids_out, float* gates_out, cudaStream_t stream) {
+// Warp-per-token routing of fp32 logits [T, N].
+cudaError_t launch_route_warp(const float* logits, int64_t T, int N, int K, float eps,
+                              int topk_mode, int renorm, int32_t* k_out, int32_t* ids_out,
+                              float* gates_out, cudaStream_t stream) {
   if (T == 0) return cudaSuccess;
   const int64_t blocks = (T + rwarp::kWarps - 1) / rwarp::kWarps;
   if (N == 64)
     rwarp::route_warp_kernel<64><<<static_cast<unsigned>(blocks), 32 * rwarp::kWarps, 0, stream>>>(
-        src, T, nslice, K, eps, topk_mode, renorm, logits_out, k_out, ids_out, gates_out);
+        logits, T, K, eps, topk_mode, renorm, k_out, ids_out, gates_out);
   else
     rwarp::route_warp_kernel<128><<<static_cast<unsigned>(blocks), 32 * rwarp::kWarps, 0, stream>>>(
-        src, T, nslice, K, eps, topk_mode, renorm, logits_out, k_out, ids_out, gates_out);
+        logits, T, K, eps, topk_mode, renorm, k_out, ids_out, gates_out);
   return cudaGetLastError();
 }
 
 // Router logits of T <= 64 tokens (as d / 64 partial sums, partial [d/64][T][N])
-// and their routing, in one launch; ticket: a zeroed device counter, left zero.
+// and their routing, in one launch; ticket: ceil(T / 16) zeroed device
+// counters, left zero.
 cudaError_t launch_router_small_route(const uint16_t* x, const uint16_t* w_router, int T, int d,
                                       int N, float* partial, unsigned int* ticket, int K, float eps,
                                       int topk_mode, int renorm, float* logits_out, int32_t* k_out,
                                       int32_t* ids_out, float* gates_out, cudaStream_t stream) {
   if (T == 0) return cudaSuccess;
-  const unsigned slices = static_cast<unsigned>(d / rwarp::kSlice);
+  if (T > rwarp::kSmallT || d % rwarp::kSlice != 0) return cudaErrorInvalidValue;
+  const dim3 grid(static_cast<unsigned>(d / rwarp::kSlice),
+                  static_cast<unsigned>((T + rwarp::kGroupT - 1) / rwarp::kGroupT));
   auto xx = reinterpret_cast<const uint32_t*>(x);
   auto ww = reinterpret_cast<const uint32_t*>(w_router);
-  if (N == 64)
-    rwarp::router_small_route_kernel<64><<<slices, 256, 0, stream>>>(
-        xx, ww, T, d, partial, ticket, K, eps, topk_mode, renorm, logits_out, k_out, ids_out,
-        gates_out);
-  else
-    rwarp::router_small_route_kernel<128><<<slices, 256, 0, stream>>>(
-        xx, ww, T, d, partial, ticket, K, eps, topk_mode, renorm, logits_out, k_out, ids_out,
-        gates_out);
+  auto kern = N == 64 ? rwarp::router_small_route_kernel<64> : rwarp::router_small_route_kernel<128>;
+  kern<<<grid, rwarp::kSmallThreads, 0, stream>>>(xx, ww, T, d, partial, ticket, K, eps, topk_mode,
+                                                  renorm, logits_out, k_out, ids_out, gates_out);
   return cudaGetLastError();
 }
 

@@ -123,10 +123,13 @@ def test_layer_decode_sizes(moe, T):
 
 
 @pytest.mark.parametrize("T,N,d,I,K,mode", [(16, 128, 1024, 512, 8, 0), (40, 128, 1024, 512, 8, 1),
-                                            (9, 64, 512, 256, 4, 0), (64, 64, 512, 256, 2, 0)])
+                                            (9, 64, 512, 256, 4, 0), (64, 64, 512, 256, 2, 0),
+                                            (64, 128, 1024, 512, 8, 0), (24, 64, 4096, 128, 8, 0),
+                                            (33, 64, 256, 128, 8, 0)])
 def test_layer_small_batches_shapes(moe, T, N, d, I, K, mode):
-    """Small batches with 128 experts, other caps and top-K mode: the warp
-    router (T <= 16) or the fused router, the decode GEMMs, every token vs the
+    """Small batches with 128 experts, other caps and top-K mode: the split
+    router GEMM with warp routing (its largest shared-memory case at T = 64,
+    N = 128; 2 to 32 slices of d), the decode GEMMs, every token vs the
     oracle."""
     import torch
     inp = synth.layer_inputs(T=T, d=d, N=N, I=I, seed=900 + T + N)
