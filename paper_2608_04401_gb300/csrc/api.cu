@@ -16,6 +16,10 @@ int32_t* dispatch_counts(void* ws);
 cudaError_t launch_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
                             int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
                             int32_t* offsets_copy, bool counts_ready, cudaStream_t stream);
+cudaError_t launch_dispatch_gather(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
+                                   int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
+                                   int32_t* offsets_copy, const uint16_t* x, int d, uint16_t* xs,
+                                   int num_sms, cudaStream_t stream);
 cudaError_t launch_gather(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int N,
                           int64_t P, int d, uint16_t* xs, int num_sms, cudaStream_t stream);
 cudaError_t launch_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_pos,
@@ -375,19 +379,21 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
                                  moe::dispatch_counts(w.disp), w.err, nsm, s);
   }
   if (e != cudaSuccess) return MOE_ERR_CUDA;
-  e = moe::launch_dispatch(kk, ids, T, N, K, w.offsets, w.perm, w.pair_pos, w.disp, offsets_out,
-                           true, s);
-  if (e != cudaSuccess) return MOE_ERR_CUDA;
   if (T <= kDecodeMaxTokens) {
-    // decode-sized: gather the few token rows (into o, which the down GEMM
-    // overwrites afterwards) and stream the weights as the M operand
-    e = moe::launch_gather(x, w.perm, w.offsets, N, P, d, w.o, nsm, s);
+    // decode-sized: the single-chunk dispatch also gathers the few token rows
+    // (into o, which the down GEMM overwrites afterwards); the GEMMs stream
+    // the weights as the M operand
+    e = moe::launch_dispatch_gather(kk, ids, T, N, K, w.offsets, w.perm, w.pair_pos, w.disp,
+                                    offsets_out, x, d, w.o, nsm, s);
     if (e != cudaSuccess) return MOE_ERR_CUDA;
     e = moe::launch_gateup_decode_gemm(w.o, w_gate_up, w.offsets, P, d, N, I, w.h, w.err, nsm, s);
     if (e != cudaSuccess) return MOE_ERR_CUDA;
     e = moe::launch_down_decode_gemm(w.h, w_down, w.offsets, P, d, N, I, w.o, w.err, nsm, s);
     if (e != cudaSuccess) return MOE_ERR_CUDA;
   } else {
+    e = moe::launch_dispatch(kk, ids, T, N, K, w.offsets, w.perm, w.pair_pos, w.disp, offsets_out,
+                             true, s);
+    if (e != cudaSuccess) return MOE_ERR_CUDA;
     const int32_t* tile_off = moe::dispatch_tile_off(w.disp, T, N);
     // gate/up GEMM gathers its token rows itself (no dispatched copy of x)
     e = moe::launch_gateup_gather_gemm(x, T, w.perm, w_gate_up, w.offsets, tile_off, P, d, N, I,

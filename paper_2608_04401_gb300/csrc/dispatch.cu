@@ -170,12 +170,19 @@ MOE_DEV int block_exclusive_scan_small(int v, int* warp_tmp, int& total) {
 
 // SINGLE: the batch is one chunk (T <= 128); its own counts are the expert
 // totals and its scan the expert offsets, so no count or scan pass runs.
-template <int N, bool SINGLE>
+// GATHER (with SINGLE): every block of the grid computes the chunk's dispatch
+// in shared memory, block 0 writes it out, and all blocks copy the dispatched
+// token rows xs[r] = x[perm[r]] (one warp per row, rows strided over the grid),
+// so the gather needs no launch of its own.
+template <int N, bool SINGLE, bool GATHER = false>
 __global__ void __launch_bounds__(kChunk) scatter_kernel(
     const int32_t* __restrict__ k, const int32_t* __restrict__ ids, int64_t T, int K, int nblk,
     const int32_t* __restrict__ base, const int32_t* __restrict__ totals,
     int32_t* __restrict__ perm, int32_t* __restrict__ pair_pos, int32_t* __restrict__ offsets,
-    int32_t* __restrict__ tile_off, int32_t* __restrict__ offsets_copy) {
+    int32_t* __restrict__ tile_off, int32_t* __restrict__ offsets_copy,
+    const uint4* __restrict__ x = nullptr, int d8 = 0, uint4* __restrict__ xs = nullptr) {
+  static_assert(SINGLE || !GATHER, "the fused gather needs the single-chunk dispatch");
+  const bool writer = !GATHER || blockIdx.x == 0;
   __shared__ int exp_off[N];
   __shared__ uint32_t bal[kWarps][N];
   __shared__ int wbase[kWarps][N];   // global position of each warp's first pair per expert
@@ -211,7 +218,8 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
     if (blockIdx.x == 0) write_offsets(tot, off, total_pairs);
   }
 
-  const int64_t t = static_cast<int64_t>(blockIdx.x) * kChunk + tid;
+  // (with GATHER every block works on the one chunk)
+  const int64_t t = (GATHER ? 0 : static_cast<int64_t>(blockIdx.x) * kChunk) + tid;
   const bool valid = t < T;
   int kt, my[8];
   uint64_t m0, m1;
@@ -227,7 +235,9 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
   }
   int chunk_pairs;
   const int chunk_off = block_exclusive_scan_small<N>(c_e, warp_tmp, chunk_pairs);
-  if constexpr (SINGLE) write_offsets(c_e, chunk_off, chunk_pairs);
+  if constexpr (SINGLE) {
+    if (writer) write_offsets(c_e, chunk_off, chunk_pairs);  // block-uniform condition
+  }
   if (tid < N) {
     int acc = SINGLE ? chunk_off : exp_off[tid] + base[static_cast<int64_t>(tid) * nblk + blockIdx.x];
     int lacc = chunk_off;
@@ -253,8 +263,8 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
           const int lpos = lbase[warp][e] + below;
           s_tok[lpos] = static_cast<int32_t>(t);
           s_gpos[lpos] = pos;
-          pair_pos[t * K + s] = pos;
-        } else {
+          if (writer) pair_pos[t * K + s] = pos;
+        } else if (writer) {
           pair_pos[t * K + s] = -1;
         }
       }
@@ -263,10 +273,20 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
   __syncthreads();
   // write perm from the expert-sorted list: consecutive threads write
   // consecutive positions inside each expert's run
-  for (int i = tid; i < chunk_pairs; i += kChunk) {
-    const int pos = s_gpos[i];
-    // positions stay below T*K when the counts match the ids
-    if (pos >= 0 && static_cast<int64_t>(pos) < T * K) perm[pos] = s_tok[i];
+  if (writer) {
+    for (int i = tid; i < chunk_pairs; i += kChunk) {
+      const int pos = s_gpos[i];
+      // positions stay below T*K when the counts match the ids
+      if (pos >= 0 && static_cast<int64_t>(pos) < T * K) perm[pos] = s_tok[i];
+    }
+  }
+  if constexpr (GATHER) {
+    // single chunk: the global position of list entry r is r itself
+    for (int r = blockIdx.x * kWarps + warp; r < chunk_pairs; r += gridDim.x * kWarps) {
+      const uint4* src = x + static_cast<int64_t>(s_tok[r]) * d8;
+      uint4* dst = xs + static_cast<int64_t>(r) * d8;
+      for (int c = lane; c < d8; c += 32) dst[c] = __ldg(src + c);
+    }
   }
 }
 
@@ -521,6 +541,23 @@ cudaError_t launch_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int
   return run_dispatch(k, ids, T, N, K, offsets, perm, pair_pos, dispatch_counts(ws),
                       dispatch_totals(ws, T, N), dispatch_tile_off(ws, T, N), offsets_copy,
                       counts_ready, stream);
+}
+
+// Single-chunk dispatch (T <= 128) fused with the row gather xs[r] = x[perm[r]].
+cudaError_t launch_dispatch_gather(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
+                                   int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
+                                   int32_t* offsets_copy, const uint16_t* x, int d, uint16_t* xs,
+                                   int num_sms, cudaStream_t stream) {
+  if (num_chunks(T) != 1) return cudaErrorInvalidValue;
+  // one warp per dispatched row: T * K rows at most
+  int64_t blocks = (T * K + disp::kWarps - 1) / disp::kWarps;
+  if (blocks > num_sms) blocks = num_sms;
+  auto kern = N == 64 ? disp::scatter_kernel<64, true, true> : disp::scatter_kernel<128, true, true>;
+  kern<<<static_cast<unsigned>(blocks), disp::kChunk, 0, stream>>>(
+      k, ids, T, K, 1, dispatch_counts(ws), dispatch_totals(ws, T, N), perm, pair_pos, offsets,
+      dispatch_tile_off(ws, T, N), offsets_copy, reinterpret_cast<const uint4*>(x), d / 8,
+      reinterpret_cast<uint4*>(xs));
+  return cudaGetLastError();
 }
 
 cudaError_t launch_gather(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int N,
