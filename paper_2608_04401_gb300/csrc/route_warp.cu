@@ -235,8 +235,8 @@ __global__ void __launch_bounds__(32 * kWarps) route_warp_kernel(
 
 // The small-batch router in one launch: block (s, j) writes the partial sums
 // of slice s for token group j; the block of group j that finishes last (a
-// ticket counter per group, after a memory fence: no block waits for
-// another) adds them up in slice order with all its threads (two pairs'
+// ticket counter per group, taken by an acquire-release atomic after a block
+// barrier: no block waits for another) adds them up in slice order with all its threads (two pairs'
 // loads in flight per thread), keeps the group's logits in shared memory,
 // routes its tokens with one warp each and resets the counter.
 template <int N>
@@ -250,12 +250,17 @@ __global__ void __launch_bounds__(kSmallThreads) router_small_route_kernel(
   const int t0 = blockIdx.y * kGroupT;
   const int nj = min(kGroupT, T - t0);
   router_small_body<N>(x, w, T, d, t0, nj, partial);
-  __threadfence();
+  // the block's partial sums happen before thread 0's release (the barrier);
+  // the acquire half makes every earlier block's sums visible to the last one
   __syncthreads();
-  if (threadIdx.x == 0) last = atomicAdd(ticket + blockIdx.y, 1u) == gridDim.x - 1;
+  if (threadIdx.x == 0) {
+    unsigned int prev;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;"
+                 : "=r"(prev) : "l"(ticket + blockIdx.y) : "memory");
+    last = prev == gridDim.x - 1;
+  }
   __syncthreads();
   if (!last) return;
-  __threadfence();
   const int nslice = static_cast<int>(gridDim.x);
   const int64_t stride = static_cast<int64_t>(T) * N;
   const float* src = partial + static_cast<int64_t>(t0) * N;
