@@ -25,6 +25,35 @@ __host__ __device__ __forceinline__ T min_of(T a, T b) {
   return a < b ? a : b;
 }
 
+// Programmatic dependent launch. The layer's kernels are launched with the
+// programmatic-serialization attribute, so the next kernel in the stream may
+// be scheduled before this one ends: each kernel first does set-up that
+// touches no global memory, then waits (grid_dep_wait: until the preceding
+// grids have completed and their writes are visible) before its first global
+// read or write, and then lets its own dependents launch (grid_dep_launch).
+// Without the attribute (or without a preceding grid) the wait returns at once.
+MOE_DEV void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+MOE_DEV void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// Launches kern<<<grid, block, smem, stream>>>(args...) with programmatic
+// stream serialization allowed (the kernel must call grid_dep_wait before it
+// touches global memory).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t stream, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 MOE_DEV uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

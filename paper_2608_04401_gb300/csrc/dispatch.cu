@@ -79,6 +79,8 @@ __global__ void __launch_bounds__(kChunk) count_kernel(const int32_t* __restrict
                                                        const int32_t* __restrict__ ids, int64_t T,
                                                        int K, int nblk, int32_t* __restrict__ cnt) {
   __shared__ int wcnt[kWarps][N];
+  grid_dep_wait();
+  grid_dep_launch();
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   const int64_t t = static_cast<int64_t>(blockIdx.x) * kChunk + threadIdx.x;
   int kt, my[8];
@@ -104,6 +106,8 @@ __global__ void __launch_bounds__(kScanThreads) scan_kernel(int32_t* __restrict_
                                                             int32_t* __restrict__ totals) {
   constexpr int kW = kScanThreads / 32;
   __shared__ int warp_sum[kW];
+  grid_dep_wait();
+  grid_dep_launch();
   int32_t* col = cnt + static_cast<int64_t>(blockIdx.x) * nblk;
   const int lane = threadIdx.x % 32, warp = threadIdx.x / 32;
   const int seg = (((nblk + kW - 1) / kW) + 31) & ~31;
@@ -182,6 +186,8 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
     int32_t* __restrict__ tile_off, int32_t* __restrict__ offsets_copy,
     const uint4* __restrict__ x = nullptr, int d8 = 0, uint4* __restrict__ xs = nullptr) {
   static_assert(SINGLE || !GATHER, "the fused gather needs the single-chunk dispatch");
+  grid_dep_wait();
+  grid_dep_launch();
   const bool writer = !GATHER || blockIdx.x == 0;
   __shared__ int exp_off[N];
   __shared__ uint32_t bal[kWarps][N];
@@ -347,6 +353,8 @@ __global__ void __launch_bounds__(32 * kCombineWarps) combine_kernel(
   using C = CombineCfg<RES>;
   constexpr int CH = C::CH;
   extern __shared__ uint4 cmb_smem[];
+  grid_dep_wait();
+  grid_dep_launch();
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x / 32;
   uint4* ring = cmb_smem + static_cast<size_t>(warp) * 2 * C::kStage;
@@ -504,35 +512,29 @@ static cudaError_t run_dispatch(const int32_t* k, const int32_t* ids, int64_t T,
                                 int32_t* totals, int32_t* tile_off, int32_t* offsets_copy,
                                 bool counts_ready, cudaStream_t stream) {
   const int nblk = num_chunks(T);
+  const uint4* no_x = nullptr;
+  uint4* no_xs = nullptr;
   if (nblk == 1) {
-    if (N == 64)
-      disp::scatter_kernel<64, true><<<1, disp::kChunk, 0, stream>>>(
-          k, ids, T, K, nblk, cnt, totals, perm, pair_pos, offsets, tile_off, offsets_copy);
-    else
-      disp::scatter_kernel<128, true><<<1, disp::kChunk, 0, stream>>>(
-          k, ids, T, K, nblk, cnt, totals, perm, pair_pos, offsets, tile_off, offsets_copy);
-    return cudaGetLastError();
+    auto kern = N == 64 ? disp::scatter_kernel<64, true> : disp::scatter_kernel<128, true>;
+    return launch_pdl(kern, dim3(1), dim3(disp::kChunk), 0, stream, k, ids, T, K, nblk, cnt, totals,
+                      perm, pair_pos, offsets, tile_off, offsets_copy, no_x, 0, no_xs);
   }
+  cudaError_t e;
   if (nblk > 0 && !counts_ready) {
-    if (N == 64) disp::count_kernel<64><<<nblk, disp::kChunk, 0, stream>>>(k, ids, T, K, nblk, cnt);
-    else disp::count_kernel<128><<<nblk, disp::kChunk, 0, stream>>>(k, ids, T, K, nblk, cnt);
-  }
-  if (nblk > 0) {
-    disp::scan_kernel<<<N, disp::kScanThreads, 0, stream>>>(cnt, nblk, totals);
-  } else {
-    cudaError_t e = cudaMemsetAsync(totals, 0, N * sizeof(int32_t), stream);
+    auto kern = N == 64 ? disp::count_kernel<64> : disp::count_kernel<128>;
+    e = launch_pdl(kern, dim3(nblk), dim3(disp::kChunk), 0, stream, k, ids, T, K, nblk, cnt);
     if (e != cudaSuccess) return e;
   }
+  if (nblk > 0) {
+    e = launch_pdl(disp::scan_kernel, dim3(N), dim3(disp::kScanThreads), 0, stream, cnt, nblk, totals);
+  } else {
+    e = cudaMemsetAsync(totals, 0, N * sizeof(int32_t), stream);
+  }
+  if (e != cudaSuccess) return e;
   const int grid = nblk > 0 ? nblk : 1;
-  if (N == 64)
-    disp::scatter_kernel<64, false><<<grid, disp::kChunk, 0, stream>>>(k, ids, T, K, nblk, cnt, totals, perm,
-                                                                pair_pos, offsets, tile_off,
-                                                                offsets_copy);
-  else
-    disp::scatter_kernel<128, false><<<grid, disp::kChunk, 0, stream>>>(k, ids, T, K, nblk, cnt, totals,
-                                                                 perm, pair_pos, offsets, tile_off,
-                                                                 offsets_copy);
-  return cudaGetLastError();
+  auto kern = N == 64 ? disp::scatter_kernel<64, false> : disp::scatter_kernel<128, false>;
+  return launch_pdl(kern, dim3(grid), dim3(disp::kChunk), 0, stream, k, ids, T, K, nblk, cnt, totals,
+                    perm, pair_pos, offsets, tile_off, offsets_copy, no_x, 0, no_xs);
 }
 
 cudaError_t launch_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
@@ -553,11 +555,11 @@ cudaError_t launch_dispatch_gather(const int32_t* k, const int32_t* ids, int64_t
   int64_t blocks = (T * K + disp::kWarps - 1) / disp::kWarps;
   if (blocks > num_sms) blocks = num_sms;
   auto kern = N == 64 ? disp::scatter_kernel<64, true, true> : disp::scatter_kernel<128, true, true>;
-  kern<<<static_cast<unsigned>(blocks), disp::kChunk, 0, stream>>>(
-      k, ids, T, K, 1, dispatch_counts(ws), dispatch_totals(ws, T, N), perm, pair_pos, offsets,
-      dispatch_tile_off(ws, T, N), offsets_copy, reinterpret_cast<const uint4*>(x), d / 8,
-      reinterpret_cast<uint4*>(xs));
-  return cudaGetLastError();
+  return launch_pdl(kern, dim3(static_cast<unsigned>(blocks)), dim3(disp::kChunk), 0, stream, k, ids,
+                    T, K, 1, static_cast<const int32_t*>(dispatch_counts(ws)),
+                    static_cast<const int32_t*>(dispatch_totals(ws, T, N)), perm, pair_pos, offsets,
+                    dispatch_tile_off(ws, T, N), offsets_copy, reinterpret_cast<const uint4*>(x),
+                    d / 8, reinterpret_cast<uint4*>(xs));
 }
 
 cudaError_t launch_gather(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int N,
@@ -603,10 +605,10 @@ cudaError_t launch_combine(const uint16_t* o, const int32_t* k, const int32_t* p
   int64_t blocks = (units + disp::kCombineWarps - 1) / disp::kCombineWarps;
   const int64_t cap = static_cast<int64_t>(num_sms) * per_sm;
   if (blocks > cap) blocks = cap;
-  kern<<<static_cast<unsigned>(blocks), 32 * disp::kCombineWarps, smem, stream>>>(
-      reinterpret_cast<const uint4*>(o), k, pair_pos, gates,
-      reinterpret_cast<const uint4*>(residual), T, d / 8, K, reinterpret_cast<uint4*>(y));
-  return cudaGetLastError();
+  return launch_pdl(kern, dim3(static_cast<unsigned>(blocks)), dim3(32 * disp::kCombineWarps), smem,
+                    stream, reinterpret_cast<const uint4*>(o), k, pair_pos, gates,
+                    reinterpret_cast<const uint4*>(residual), T, d / 8, K,
+                    reinterpret_cast<uint4*>(y));
 }
 
 }  // namespace moe

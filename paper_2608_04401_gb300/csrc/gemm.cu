@@ -263,6 +263,14 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
     *abort_flag = 0;
     fence_mbar_init();
   }
+  if (warp == 0 && lane == 0) {
+    prefetch_tensormap(&tmA);
+    prefetch_tensormap(&tmB);
+  }
+  // everything above touches no global memory; from here on the preceding
+  // kernels' results are read (and TMEM is taken only once they have ended)
+  grid_dep_wait();
+  grid_dep_launch();
   if (!is_router<MODE>()) {  // grouped schedule tables (router modes have none)
     for (int i = threadIdx.x; i <= args.groups; i += kThreads) {
       s_off[i] = args.offsets[i];
@@ -270,10 +278,6 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
       // (their tile_off is null)
       s_toff[i] = is_decode<MODE>() ? 0 : args.tile_off[i];
     }
-  }
-  if (warp == 0 && lane == 0) {
-    prefetch_tensormap(&tmA);
-    prefetch_tensormap(&tmB);
   }
   if (warp == R::kMmaWarp) {
     __syncwarp();
@@ -722,8 +726,8 @@ static cudaError_t launch_mode(const CUtensorMap& a, const CUtensorMap& b, const
     if (e != cudaSuccess) return e;
     attr_dev = dev;
   }
-  gemm_kernel<MODE, BN><<<grid, Roles<MODE>::kThreads, C::kSmemBytes, stream>>>(a, b, c, args);
-  return cudaGetLastError();
+  return launch_pdl(gemm_kernel<MODE, BN>, dim3(grid), dim3(Roles<MODE>::kThreads), C::kSmemBytes,
+                    stream, a, b, c, args);
 }
 
 }  // namespace gemm

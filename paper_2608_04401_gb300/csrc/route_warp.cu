@@ -247,6 +247,8 @@ __global__ void __launch_bounds__(kSmallThreads) router_small_route_kernel(
     int32_t* __restrict__ ids_out, float* __restrict__ gates_out) {
   __shared__ float lg[kGroupT * N];
   __shared__ bool last;
+  grid_dep_wait();
+  grid_dep_launch();
   const int t0 = blockIdx.y * kGroupT;
   const int nj = min(kGroupT, T - t0);
   router_small_body<N>(x, w, T, d, t0, nj, partial);
@@ -333,9 +335,8 @@ cudaError_t launch_router_small_route(const uint16_t* x, const uint16_t* w_route
   auto xx = reinterpret_cast<const uint32_t*>(x);
   auto ww = reinterpret_cast<const uint32_t*>(w_router);
   auto kern = N == 64 ? rwarp::router_small_route_kernel<64> : rwarp::router_small_route_kernel<128>;
-  kern<<<grid, rwarp::kSmallThreads, 0, stream>>>(xx, ww, T, d, partial, ticket, K, eps, topk_mode,
-                                                  renorm, logits_out, k_out, ids_out, gates_out);
-  return cudaGetLastError();
+  return launch_pdl(kern, grid, dim3(rwarp::kSmallThreads), 0, stream, xx, ww, T, d, partial, ticket, K,
+                    eps, topk_mode, renorm, logits_out, k_out, ids_out, gates_out);
 }
 
 }  // namespace moe
