@@ -17,7 +17,8 @@
 // block per slice and group) so that many SMs share the work instead of one
 // SM streaming all of x and W_r:
 // partial[s][t][e] = sum_{k in slice s} x[t][k] w[e][k], fp32 fma in k order;
-// the block that finishes last routes every token (slices added in order).
+// in each group the block that finishes last adds the slices in order and
+// routes the group's tokens.
 #include "route_impl.cuh"
 
 namespace moe {
