@@ -98,11 +98,13 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 size_t up256(size_t b) { return (b + 255) & ~static_cast<size_t>(255); }
 
+// SM count of the current device, or 0 if it cannot be queried (the entry
+// points then return MOE_ERR_CUDA).
 int sm_count() {
   int dev = 0, n = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
   if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-    return 148;
+    return 0;
   return n;
 }
 
@@ -362,6 +364,7 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   float* gates = gates_out ? gates_out : w.gates;
   const int64_t P = T * K;
   const int nsm = sm_count();
+  if (nsm <= 0) return MOE_ERR_CUDA;
 
   cudaError_t e;
   if (T <= kSmallRouterMaxTokens) {
@@ -432,7 +435,9 @@ moe_status moe_router_logits(const uint16_t* x, const uint16_t* w_router, int64_
   if (T == 0) return MOE_OK;
   if (!x || !w_router || !logits || !aligned16(x) || !aligned16(w_router) || !aligned16(logits))
     return MOE_ERR_INVALID_ARG;
-  return cuda_status(moe::launch_router_gemm(x, w_router, T, d, N, logits, err_word, sm_count(),
+  const int nsm = sm_count();
+  if (nsm <= 0) return MOE_ERR_CUDA;
+  return cuda_status(moe::launch_router_gemm(x, w_router, T, d, N, logits, err_word, nsm,
                                              static_cast<cudaStream_t>(stream)));
 }
 
@@ -447,8 +452,10 @@ moe_status moe_expert_gate_up(const uint16_t* xs, const uint16_t* w_gate_up, con
   if (!xs || !w_gate_up || !offsets || !tile_off || !h || !aligned16(xs) || !aligned16(w_gate_up) ||
       !aligned16(h))
     return MOE_ERR_INVALID_ARG;
+  const int nsm = sm_count();
+  if (nsm <= 0) return MOE_ERR_CUDA;
   return cuda_status(moe::launch_gateup_gemm(xs, w_gate_up, offsets, tile_off, P, d, N, I, h,
-                                             err_word, sm_count(), static_cast<cudaStream_t>(stream)));
+                                             err_word, nsm, static_cast<cudaStream_t>(stream)));
 }
 
 moe_status moe_expert_down(const uint16_t* h, const uint16_t* w_down, const int32_t* offsets,
@@ -462,8 +469,10 @@ moe_status moe_expert_down(const uint16_t* h, const uint16_t* w_down, const int3
   if (!h || !w_down || !offsets || !tile_off || !o || !aligned16(h) || !aligned16(w_down) ||
       !aligned16(o))
     return MOE_ERR_INVALID_ARG;
+  const int nsm = sm_count();
+  if (nsm <= 0) return MOE_ERR_CUDA;
   return cuda_status(moe::launch_down_gemm(h, w_down, offsets, tile_off, P, d, N, I, o, err_word,
-                                           sm_count(), static_cast<cudaStream_t>(stream)));
+                                           nsm, static_cast<cudaStream_t>(stream)));
 }
 
 moe_status moe_expert_gate_up_decode(const uint16_t* xs, const uint16_t* w_gate_up,
@@ -478,8 +487,10 @@ moe_status moe_expert_gate_up_decode(const uint16_t* xs, const uint16_t* w_gate_
   if (!xs || !w_gate_up || !offsets || !h || !aligned16(xs) || !aligned16(w_gate_up) ||
       !aligned16(h))
     return MOE_ERR_INVALID_ARG;
+  const int nsm = sm_count();
+  if (nsm <= 0) return MOE_ERR_CUDA;
   return cuda_status(moe::launch_gateup_decode_gemm(xs, w_gate_up, offsets, P, d, N, I, h, err_word,
-                                                    sm_count(), static_cast<cudaStream_t>(stream)));
+                                                    nsm, static_cast<cudaStream_t>(stream)));
 }
 
 moe_status moe_expert_down_decode(const uint16_t* h, const uint16_t* w_down, const int32_t* offsets,
@@ -493,8 +504,10 @@ moe_status moe_expert_down_decode(const uint16_t* h, const uint16_t* w_down, con
   if (P == 0 || T == 0) return MOE_OK;
   if (!h || !w_down || !offsets || !o || !aligned16(h) || !aligned16(w_down) || !aligned16(o))
     return MOE_ERR_INVALID_ARG;
+  const int nsm = sm_count();
+  if (nsm <= 0) return MOE_ERR_CUDA;
   return cuda_status(moe::launch_down_decode_gemm(h, w_down, offsets, P, d, N, I, o, err_word,
-                                                  sm_count(), static_cast<cudaStream_t>(stream)));
+                                                  nsm, static_cast<cudaStream_t>(stream)));
 }
 
 moe_status moe_gather_rows(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int64_t T,
@@ -504,7 +517,9 @@ moe_status moe_gather_rows(const uint16_t* x, const int32_t* perm, const int32_t
   if (!supported_n(N)) return MOE_ERR_UNSUPPORTED;
   if (P == 0) return MOE_OK;
   if (!x || !perm || !offsets || !xs || !aligned16(x) || !aligned16(xs)) return MOE_ERR_INVALID_ARG;
-  return cuda_status(moe::launch_gather(x, perm, offsets, N, P, d, xs, sm_count(),
+  const int nsm = sm_count();
+  if (nsm <= 0) return MOE_ERR_CUDA;
+  return cuda_status(moe::launch_gather(x, perm, offsets, N, P, d, xs, nsm,
                                         static_cast<cudaStream_t>(stream)));
 }
 
@@ -521,10 +536,12 @@ moe_status moe_router_route(const uint16_t* x, const uint16_t* w_router, int64_t
       !aligned16(ids_out) || !aligned16(gates_out) || (logits_out && !aligned16(logits_out)) ||
       (reinterpret_cast<uintptr_t>(k_out) & 3u))
     return MOE_ERR_INVALID_ARG;
+  const int nsm = sm_count();
+  if (nsm <= 0) return MOE_ERR_CUDA;
   return cuda_status(moe::launch_router_route(x, w_router, T, d, N, rp->K, rp->eps,
                                               rp->mode == MOE_ROUTE_TOPK, rp->renorm, logits_out,
                                               k_out, ids_out, gates_out, chunk_counts, err_word,
-                                              sm_count(), static_cast<cudaStream_t>(stream)));
+                                              nsm, static_cast<cudaStream_t>(stream)));
 }
 
 moe_status moe_expert_gate_up_gathered(const uint16_t* x, int64_t T, const int32_t* perm,
@@ -539,8 +556,10 @@ moe_status moe_expert_gate_up_gathered(const uint16_t* x, int64_t T, const int32
   if (!x || !perm || !w_gate_up || !offsets || !tile_off || !h || !aligned16(x) ||
       !aligned16(w_gate_up) || !aligned16(h))
     return MOE_ERR_INVALID_ARG;
+  const int nsm = sm_count();
+  if (nsm <= 0) return MOE_ERR_CUDA;
   return cuda_status(moe::launch_gateup_gather_gemm(x, T, perm, w_gate_up, offsets, tile_off, P, d, N,
-                                                    I, h, err_word, sm_count(),
+                                                    I, h, err_word, nsm,
                                                     static_cast<cudaStream_t>(stream)));
 }
 
@@ -552,7 +571,9 @@ moe_status moe_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_
   if (!o || !k || !pair_pos || !gates || !y || !aligned16(o) || !aligned16(y) ||
       (residual && !aligned16(residual)))
     return MOE_ERR_INVALID_ARG;
-  return cuda_status(moe::launch_combine(o, k, pair_pos, gates, residual, T, d, K, y, sm_count(),
+  const int nsm = sm_count();
+  if (nsm <= 0) return MOE_ERR_CUDA;
+  return cuda_status(moe::launch_combine(o, k, pair_pos, gates, residual, T, d, K, y, nsm,
                                          static_cast<cudaStream_t>(stream)));
 }
 

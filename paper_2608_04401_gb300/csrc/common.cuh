@@ -7,6 +7,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "../../include/elbow_moe.h"
 
 #define MOE_DEV __device__ __forceinline__
@@ -52,6 +54,21 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
+// One-time per-device set-up (a kernel attribute), safe under concurrent host
+// threads: `done` holds one bit per device ordinal below 64; ordinals past 63
+// simply repeat the set-up. Returns the set-up's error, or cudaSuccess.
+template <typename SetUp>
+inline cudaError_t once_per_device(std::atomic<uint64_t>& done, SetUp set_up) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = dev < 64 ? uint64_t(1) << dev : 0;
+  if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+  e = set_up();
+  if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_release);
+  return e;
 }
 
 MOE_DEV uint32_t smem_u32(const void* p) {

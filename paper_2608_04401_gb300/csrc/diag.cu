@@ -158,15 +158,12 @@ cudaError_t launch(const float* logits, int64_t T, int K, float eps, int32_t* el
     RouteConsts<N> rc;
     route::fill_route_consts(rc, N);
     constexpr size_t smem = route::smem_bytes<N>();
-    static int attr_dev = -1;
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (attr_dev != dev) {
-      err = cudaFuncSetAttribute(diag_kernel<N>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 static_cast<int>(smem));
-      if (err != cudaSuccess) return err;
-      attr_dev = dev;
-    }
+    static std::atomic<uint64_t> attr_done{0};
+    err = once_per_device(attr_done, [&] {
+      return cudaFuncSetAttribute(diag_kernel<N>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  static_cast<int>(smem));
+    });
+    if (err != cudaSuccess) return err;
     const int64_t blocks = (T + kTok - 1) / kTok;
     diag_kernel<N><<<static_cast<unsigned>(blocks), kTok, smem, stream>>>(
         logits, T, K, eps, rc, elbow_out, theta_out, dg);

@@ -585,18 +585,17 @@ cudaError_t launch_combine(const uint16_t* o, const int32_t* k, const int32_t* p
   const int smem = residual ? disp::CombineCfg<true>::kBlockBytes : disp::CombineCfg<false>::kBlockBytes;
   auto kern = residual ? (split ? disp::combine_kernel<true, true> : disp::combine_kernel<true, false>)
                        : (split ? disp::combine_kernel<false, true> : disp::combine_kernel<false, false>);
-  static int attr_dev = -1;
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (attr_dev != dev) {
+  static std::atomic<uint64_t> attr_done{0};
+  const cudaError_t ae = once_per_device(attr_done, [] {
     for (auto f : {disp::combine_kernel<true, true>, disp::combine_kernel<true, false>,
                    disp::combine_kernel<false, true>, disp::combine_kernel<false, false>}) {
-      cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           disp::CombineCfg<false>::kBlockBytes);
+      const cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 disp::CombineCfg<false>::kBlockBytes);
       if (e != cudaSuccess) return e;
     }
-    attr_dev = dev;
-  }
+    return cudaSuccess;
+  });
+  if (ae != cudaSuccess) return ae;
   int per_sm = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 32 * disp::kCombineWarps, smem) !=
           cudaSuccess ||

@@ -717,15 +717,12 @@ template <int MODE, int BN>
 static cudaError_t launch_mode(const CUtensorMap& a, const CUtensorMap& b, const CUtensorMap& c,
                                const Args& args, int grid, cudaStream_t stream) {
   using C = Cfg<MODE, BN>;
-  static int attr_dev = -1;
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (attr_dev != dev) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_kernel<MODE, BN>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
-    if (e != cudaSuccess) return e;
-    attr_dev = dev;
-  }
+  static std::atomic<uint64_t> attr_done{0};
+  const cudaError_t e = once_per_device(attr_done, [] {
+    return cudaFuncSetAttribute(gemm_kernel<MODE, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                C::kSmemBytes);
+  });
+  if (e != cudaSuccess) return e;
   return launch_pdl(gemm_kernel<MODE, BN>, dim3(grid), dim3(Roles<MODE>::kThreads), C::kSmemBytes,
                     stream, a, b, c, args);
 }

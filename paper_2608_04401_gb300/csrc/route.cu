@@ -128,17 +128,16 @@ cudaError_t launch(const float* logits, int64_t T, int K, float eps, int topk_mo
   fill_route_consts(rc, N);
   constexpr size_t smem = smem_bytes<N>();
   auto kern = rand_mode ? elbow_route_kernel<N, true> : elbow_route_kernel<N, false>;
-  static int attr_dev = -1;
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (attr_dev != dev) {
+  static std::atomic<uint64_t> attr_done{0};
+  const cudaError_t ae = once_per_device(attr_done, [] {
     for (auto f : {elbow_route_kernel<N, true>, elbow_route_kernel<N, false>}) {
-      cudaError_t e =
+      const cudaError_t e =
           cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
       if (e != cudaSuccess) return e;
     }
-    attr_dev = dev;
-  }
+    return cudaSuccess;
+  });
+  if (ae != cudaSuccess) return ae;
   const int64_t blocks = (T + kTok - 1) / kTok;
   kern<<<static_cast<unsigned>(blocks), kTok, smem, stream>>>(
       logits, T, K, eps, topk_mode, renorm, rc, k_out, ids_out, gates_out, blk_cnt,
