@@ -112,6 +112,10 @@ def test_layer_decode_sizes(moe, T):
                                   to_dev_bf16(inp["w_down"]), K=8, ws=ws, return_intermediates=True)
     moe.read_device_error(ws)
     lg = it["logits"].cpu().numpy()
+    # T <= 64: the split router GEMM on CUDA cores; T = 65: the tensor-core router
+    ref_lg = oracle.router_logits(inp["x"], inp["w_router"]).astype(np.float64)
+    abs_sum = np.abs(f64(inp["x"])) @ np.abs(f64(inp["w_router"])).T
+    assert np.all(np.abs(lg.astype(np.float64) - ref_lg) <= 2048 * 2.0 ** -24 * abs_sum + 1e-30)
     r = oracle.route(lg, K=8)
     assert np.array_equal(r["k"], it["k"].cpu().numpy())
     assert np.array_equal(r["ids"], it["ids"].cpu().numpy())
@@ -138,6 +142,12 @@ def test_layer_small_batches_shapes(moe, T, N, d, I, K, mode):
                                   to_dev_bf16(inp["w_gate_up"]), to_dev_bf16(inp["w_down"]), K=K,
                                   mode=mode, ws=ws, return_intermediates=True)
     moe.read_device_error(ws)
+    # the split router GEMM's logits: fp32 sums of d products (64-column
+    # slices added in order) within the recursive-sum bound d 2^-24 sum|x w|
+    lg = it["logits"].cpu().numpy().astype(np.float64)
+    ref_lg = oracle.router_logits(inp["x"], inp["w_router"]).astype(np.float64)
+    abs_sum = np.abs(f64(inp["x"])) @ np.abs(f64(inp["w_router"])).T
+    assert np.all(np.abs(lg - ref_lg) <= d * 2.0 ** -24 * abs_sum + 1e-30)
     r = oracle.route(it["logits"].cpu().numpy(), K=K, mode=mode)
     assert np.array_equal(r["k"], it["k"].cpu().numpy())
     assert np.array_equal(r["ids"], it["ids"].cpu().numpy())
