@@ -235,13 +235,15 @@ moe_status moe_expert_down(const uint16_t* h, const uint16_t* w_down, const int3
                            const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* o,
                            int32_t* err_word, void* stream);
 
-/* Decode-shaped expert contractions for batches of T <= 64 tokens, where no
- * expert has more than 64 rows: the same results as moe_expert_gate_up and
- * moe_expert_down, computed with the weights as the M operand (128 weight
- * rows per tile, the expert's <= 64 rows as N), so a tile streams weights
- * instead of a mostly empty 128-row token block. moe_layer_forward takes this
- * path by itself when T <= 64. T is the token count the rows came from
- * (T > 64: MOE_ERR_UNSUPPORTED); xs [P, d] holds the dispatched rows
+/* Decode-shaped expert contractions for batches of T <= 64 tokens, where an
+ * expert has at most T rows (a token selects an expert at most once): the
+ * same results as moe_expert_gate_up and moe_expert_down, computed with the
+ * weights as the M operand (128 weight rows per tile, the expert's rows as N,
+ * in a 16-, 32- or 64-column tile for T <= 16, <= 32, <= 64), so a tile
+ * streams weights instead of a mostly empty 128-row token block.
+ * moe_layer_forward takes this path by itself when T <= 64. T is the token
+ * count the rows came from (T > 64: MOE_ERR_UNSUPPORTED; rows of an expert
+ * past T are not computed); xs [P, d] holds the dispatched rows
  * (moe_gather_rows), offsets [N + 1] the expert row offsets. I a multiple of
  * 64; d a multiple of 64 (gate/up) or 128 (down). */
 moe_status moe_expert_gate_up_decode(const uint16_t* xs, const uint16_t* w_gate_up,

@@ -42,11 +42,12 @@ cudaError_t launch_gateup_gather_gemm(const uint16_t* x, int64_t T, const int32_
                                       const int32_t* tile_off, int64_t P, int d, int N, int I,
                                       uint16_t* h, int32_t* err, int num_sms, cudaStream_t stream);
 cudaError_t launch_gateup_decode_gemm(const uint16_t* xs, const uint16_t* wgu,
-                                      const int32_t* offsets, int64_t P, int d, int N, int I,
-                                      uint16_t* h, int32_t* err, int num_sms, cudaStream_t stream);
+                                      const int32_t* offsets, int64_t P, int64_t max_rows, int d,
+                                      int N, int I, uint16_t* h, int32_t* err, int num_sms,
+                                      cudaStream_t stream);
 cudaError_t launch_down_decode_gemm(const uint16_t* h, const uint16_t* wd, const int32_t* offsets,
-                                    int64_t P, int d, int N, int I, uint16_t* o, int32_t* err,
-                                    int num_sms, cudaStream_t stream);
+                                    int64_t P, int64_t max_rows, int d, int N, int I, uint16_t* o,
+                                    int32_t* err, int num_sms, cudaStream_t stream);
 cudaError_t launch_route_warp(const float* logits, int64_t T, int N, int K, float eps,
                               int topk_mode, int renorm, int32_t* k_out, int32_t* ids_out,
                               float* gates_out, cudaStream_t stream);
@@ -389,9 +390,10 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
     e = moe::launch_dispatch_gather(kk, ids, T, N, K, w.offsets, w.perm, w.pair_pos, w.disp,
                                     offsets_out, x, d, w.o, nsm, s);
     if (e != cudaSuccess) return MOE_ERR_CUDA;
-    e = moe::launch_gateup_decode_gemm(w.o, w_gate_up, w.offsets, P, d, N, I, w.h, w.err, nsm, s);
+    e = moe::launch_gateup_decode_gemm(w.o, w_gate_up, w.offsets, P, T, d, N, I, w.h, w.err, nsm,
+                                       s);
     if (e != cudaSuccess) return MOE_ERR_CUDA;
-    e = moe::launch_down_decode_gemm(w.h, w_down, w.offsets, P, d, N, I, w.o, w.err, nsm, s);
+    e = moe::launch_down_decode_gemm(w.h, w_down, w.offsets, P, T, d, N, I, w.o, w.err, nsm, s);
     if (e != cudaSuccess) return MOE_ERR_CUDA;
   } else {
     e = moe::launch_dispatch(kk, ids, T, N, K, w.offsets, w.perm, w.pair_pos, w.disp, offsets_out,
@@ -489,8 +491,9 @@ moe_status moe_expert_gate_up_decode(const uint16_t* xs, const uint16_t* w_gate_
     return MOE_ERR_INVALID_ARG;
   const int nsm = sm_count();
   if (nsm <= 0) return MOE_ERR_CUDA;
-  return cuda_status(moe::launch_gateup_decode_gemm(xs, w_gate_up, offsets, P, d, N, I, h, err_word,
-                                                    nsm, static_cast<cudaStream_t>(stream)));
+  return cuda_status(moe::launch_gateup_decode_gemm(xs, w_gate_up, offsets, P, T, d, N, I, h,
+                                                    err_word, nsm,
+                                                    static_cast<cudaStream_t>(stream)));
 }
 
 moe_status moe_expert_down_decode(const uint16_t* h, const uint16_t* w_down, const int32_t* offsets,
@@ -506,7 +509,7 @@ moe_status moe_expert_down_decode(const uint16_t* h, const uint16_t* w_down, con
     return MOE_ERR_INVALID_ARG;
   const int nsm = sm_count();
   if (nsm <= 0) return MOE_ERR_CUDA;
-  return cuda_status(moe::launch_down_decode_gemm(h, w_down, offsets, P, d, N, I, o, err_word,
+  return cuda_status(moe::launch_down_decode_gemm(h, w_down, offsets, P, T, d, N, I, o, err_word,
                                                   nsm, static_cast<cudaStream_t>(stream)));
 }
 

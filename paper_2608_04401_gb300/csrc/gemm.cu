@@ -95,7 +95,11 @@ struct Cfg {
   static constexpr int kEpiBytes =
       MODE == kDown ? 4 * 2 * 32 * 64 : (MODE == kDecGateUp ? 64 * 65 * 4 : 0);
   static constexpr int kStages = (208 * 1024 - kRouteBytes - kEpiBytes) / kStageBytes;
-  static constexpr int kTmemCols = (2 * BN <= 64) ? 64 : (2 * BN <= 128 ? 128 : (2 * BN <= 256 ? 256 : 512));
+  // TMEM columns per accumulator: at least 32, so that a 32-column load of one
+  // accumulator never reaches into the other
+  static constexpr int kAccStride = BN < 32 ? 32 : BN;
+  static constexpr int kTmemCols = (2 * kAccStride <= 64) ? 64
+                                 : (2 * kAccStride <= 128 ? 128 : (2 * kAccStride <= 256 ? 256 : 512));
   static constexpr int kBarOff = kStages * kStageBytes;
   // barriers: full[S], empty[S], tfull[2], tempty[2], drain
   static constexpr int kNumBars = 2 * kStages + 5;
@@ -419,7 +423,7 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
         const uint32_t acc_phase = (local >> 1) & 1;
         if (!mbar_wait_bounded(tempty_bar(acc), acc_phase ^ 1u, abort_flag)) break;
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + acc * BN;
+        const uint32_t d_tmem = tmem_base + acc * C::kAccStride;
         bool ok = true;
         for (int kb = 0; kb < args.k_blocks; ++kb) {
           if (!mbar_wait_bounded(full_bar(stage), phase, abort_flag)) { ok = false; break; }
@@ -477,7 +481,7 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
         if (!__all_sync(0xffffffffu, ok)) break;
       }
       tc_fence_after();
-      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN;
+      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * C::kAccStride;
       const bool valid = r < t.rows;
       const int64_t grow = static_cast<int64_t>(t.row0) + r;
       if (MODE == kRouter) {
@@ -541,9 +545,11 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
         continue;
       } else if (is_decode<MODE>()) {
         // TMEM lane r = weight row of the tile, column c = the expert's c-th row
+        // (BN = 16, 32 or 64 columns; only columns below the expert's rows are stored)
+        static_assert(!is_decode<MODE>() || BN == 16 || BN == 32 || BN == 64, "decode tile width");
         uint32_t v0[32], v1[32];
         tmem_ld_32x32b_x32(taddr, v0);
-        tmem_ld_32x32b_x32(taddr + 32, v1);
+        if constexpr (BN > 32) tmem_ld_32x32b_x32(taddr + 32, v1);
         tmem_ld_wait();
         tc_fence_before();
         __syncwarp();
@@ -558,7 +564,7 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
 #pragma unroll
             for (int c = 0; c < 32; ++c) {
               xch[(r - 64) * 65 + c] = __uint_as_float(v0[c]);
-              xch[(r - 64) * 65 + 32 + c] = __uint_as_float(v1[c]);
+              if constexpr (BN > 32) xch[(r - 64) * 65 + 32 + c] = __uint_as_float(v1[c]);
             }
           }
           epilogue_sync();
@@ -568,9 +574,11 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
             for (int c = 0; c < 32; ++c) {
               if (c < ncols)
                 o[c * args.ldo] = __float2bfloat16_rn(silu(__uint_as_float(v0[c])) * xch[r * 65 + c]);
-              if (32 + c < ncols)
-                o[(32 + c) * args.ldo] =
-                    __float2bfloat16_rn(silu(__uint_as_float(v1[c])) * xch[r * 65 + 32 + c]);
+              if constexpr (BN > 32) {
+                if (32 + c < ncols)
+                  o[(32 + c) * args.ldo] =
+                      __float2bfloat16_rn(silu(__uint_as_float(v1[c])) * xch[r * 65 + 32 + c]);
+              }
             }
           }
           epilogue_sync();  // the exchange buffer is reused by the next tile
@@ -579,7 +587,9 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
 #pragma unroll
           for (int c = 0; c < 32; ++c) {
             if (c < ncols) o[c * args.ldo] = __float2bfloat16_rn(__uint_as_float(v0[c]));
-            if (32 + c < ncols) o[(32 + c) * args.ldo] = __float2bfloat16_rn(__uint_as_float(v1[c]));
+            if constexpr (BN > 32) {
+              if (32 + c < ncols) o[(32 + c) * args.ldo] = __float2bfloat16_rn(__uint_as_float(v1[c]));
+            }
           }
         }
         continue;
@@ -863,14 +873,23 @@ cudaError_t launch_down_gemm(const uint16_t* h, const uint16_t* wd, const int32_
 }
 
 // Decode-sized batches (every expert has at most 64 rows):
-// h[P, I] = silu(xs W_g^T) * (xs W_u^T) per expert, weights as the M operand
+// Width of the decode GEMMs' token operand: an expert of a T-token batch has at
+// most T rows, so 16, 32 or 64 columns cover it.
+static int decode_width(int64_t max_rows) { return max_rows <= 16 ? 16 : (max_rows <= 32 ? 32 : 64); }
+
+// h[P, I] = silu(xs W_g^T) * (xs W_u^T) per expert, weights as the M operand;
+// max_rows (<= 64) bounds the rows of any expert (the batch's token count).
 cudaError_t launch_gateup_decode_gemm(const uint16_t* xs, const uint16_t* wgu,
-                                      const int32_t* offsets, int64_t P, int d, int N, int I,
-                                      uint16_t* h, int32_t* err, int num_sms, cudaStream_t stream) {
+                                      const int32_t* offsets, int64_t P, int64_t max_rows, int d,
+                                      int N, int I, uint16_t* h, int32_t* err, int num_sms,
+                                      cudaStream_t stream) {
   using namespace gemm;
   if (P == 0) return cudaSuccess;
+  if (max_rows > 64) return cudaErrorInvalidValue;
+  const int bn = decode_width(max_rows);
   CUtensorMap ma, mb;
-  if (!make_map(&ma, wgu, d, static_cast<uint64_t>(N) * 2 * I, 64) || !make_map(&mb, xs, d, P, 64))
+  if (!make_map(&ma, wgu, d, static_cast<uint64_t>(N) * 2 * I, 64) ||
+      !make_map(&mb, xs, d, P, static_cast<uint32_t>(bn)))
     return cudaErrorInvalidValue;
   Args a{};
   a.offsets = offsets;
@@ -883,17 +902,23 @@ cudaError_t launch_gateup_decode_gemm(const uint16_t* xs, const uint16_t* wgu,
   a.ldo = I;
   a.err = err;
   const int tiles = N * a.n_tiles;
-  return launch_mode<kDecGateUp, 64>(ma, mb, ma, a, tiles < num_sms ? tiles : num_sms, stream);
+  const int grid = tiles < num_sms ? tiles : num_sms;
+  if (bn == 16) return launch_mode<kDecGateUp, 16>(ma, mb, ma, a, grid, stream);
+  if (bn == 32) return launch_mode<kDecGateUp, 32>(ma, mb, ma, a, grid, stream);
+  return launch_mode<kDecGateUp, 64>(ma, mb, ma, a, grid, stream);
 }
 
-// o[P, d] = h W_d[e]^T per expert, weights as the M operand
+// o[P, d] = h W_d[e]^T per expert, weights as the M operand; max_rows as above
 cudaError_t launch_down_decode_gemm(const uint16_t* h, const uint16_t* wd, const int32_t* offsets,
-                                    int64_t P, int d, int N, int I, uint16_t* o, int32_t* err,
-                                    int num_sms, cudaStream_t stream) {
+                                    int64_t P, int64_t max_rows, int d, int N, int I, uint16_t* o,
+                                    int32_t* err, int num_sms, cudaStream_t stream) {
   using namespace gemm;
   if (P == 0) return cudaSuccess;
+  if (max_rows > 64) return cudaErrorInvalidValue;
+  const int bn = decode_width(max_rows);
   CUtensorMap ma, mb;
-  if (!make_map(&ma, wd, I, static_cast<uint64_t>(N) * d, BM) || !make_map(&mb, h, I, P, 64))
+  if (!make_map(&ma, wd, I, static_cast<uint64_t>(N) * d, BM) ||
+      !make_map(&mb, h, I, P, static_cast<uint32_t>(bn)))
     return cudaErrorInvalidValue;
   Args a{};
   a.offsets = offsets;
@@ -905,7 +930,10 @@ cudaError_t launch_down_decode_gemm(const uint16_t* h, const uint16_t* wd, const
   a.ldo = d;
   a.err = err;
   const int tiles = N * a.n_tiles;
-  return launch_mode<kDecDown, 64>(ma, mb, ma, a, tiles < num_sms ? tiles : num_sms, stream);
+  const int grid = tiles < num_sms ? tiles : num_sms;
+  if (bn == 16) return launch_mode<kDecDown, 16>(ma, mb, ma, a, grid, stream);
+  if (bn == 32) return launch_mode<kDecDown, 32>(ma, mb, ma, a, grid, stream);
+  return launch_mode<kDecDown, 64>(ma, mb, ma, a, grid, stream);
 }
 
 }  // namespace moe

@@ -35,22 +35,32 @@ def _swiglu64(xs, wgu, I):
     return g / (1.0 + np.exp(-g)) * u
 
 
-@pytest.mark.parametrize("N,d,I,case", [
-    (64, 512, 256, "random"),
-    (64, 2048, 1024, "random"),
-    (128, 1024, 512, "random"),
-    (64, 512, 256, "edges"),
+@pytest.mark.parametrize("N,d,I,case,T", [
+    (64, 512, 256, "random", 64),
+    (64, 2048, 1024, "random", 64),
+    (128, 1024, 512, "random", 64),
+    (64, 512, 256, "edges", 64),
+    (64, 512, 256, "random", 1),
+    (64, 1024, 512, "random", 16),
+    (128, 512, 256, "random", 32),
+    (64, 512, 256, "edges", 16),
+    (64, 512, 256, "edges", 32),
 ])
-def test_decode_gemm_steps(moe, N, d, I, case):
+def test_decode_gemm_steps(moe, N, d, I, case, T):
+    """T <= 16, <= 32 and <= 64 take 16-, 32- and 64-column token tiles."""
     import torch
-    rng = np.random.default_rng(N + d + I)
-    K, T = 8, 64
+    rng = np.random.default_rng(N + d + I + T)
+    K = 8
     if case == "random":
         r = oracle.route(synth.boosted_logits(rng, T, N), K=K)
         k, ids = r["k"], r["ids"]
     else:
         # expert e has sizes[e] rows: tokens t < sizes[e] select it
+        # (capped at T, plus one expert of T - 1 rows: the full and the
+        # one-short tile of each width)
         sizes = {0: 64, 2: 1, 5: 31, 6: 32, 7: 33, 9: 63, N - 1: 64}
+        sizes = {e: min(n, T) for e, n in sizes.items()}
+        sizes[3] = T - 1
         ids = np.zeros((T, K), np.int32)
         k = np.zeros(T, np.int32)
         for t in range(T):
@@ -75,7 +85,7 @@ def test_decode_gemm_steps(moe, N, d, I, case):
     o_ref = np.zeros((n, d))
     for e in range(N):
         a, b = offs[e], offs[e + 1]
-        assert b - a <= 64
+        assert b - a <= T
         if b > a:
             h_ref[a:b] = _swiglu64(xsf[a:b], f64(wgu[e]), I)
             o_ref[a:b] = h_ref[a:b] @ f64(wd[e]).T
