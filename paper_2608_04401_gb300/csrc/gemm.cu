@@ -152,9 +152,10 @@ MOE_DEV Tile decode(int tile, const Args& a, const int* s_off, const int* s_toff
     return t;
   }
   if (is_decode<MODE>()) {
-    // tile = expert * n_tiles + weight-row block; the expert's rows are its
-    // B columns (an expert without rows has nothing to compute)
-    t.g = tile / a.n_tiles;
+    // tile = j * n_tiles + weight-row block, j indexing the experts that have
+    // rows (s_toff holds their ids in ascending order); the expert's rows are
+    // its B columns
+    t.g = s_toff[tile / a.n_tiles];
     t.nb = tile % a.n_tiles;
     t.row0 = s_off[t.g];
     t.rows = s_off[t.g + 1] - t.row0;
@@ -283,6 +284,23 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
       s_toff[i] = is_decode<MODE>() ? 0 : args.tile_off[i];
     }
   }
+  if constexpr (is_decode<MODE>()) {
+    // the experts with rows, in ascending order, into s_toff[0 ..), their
+    // count into s_toff[kMaxGroups]: tiles are numbered over these experts
+    // only, so the round-robin over CTAs stays balanced however many are empty
+    __syncthreads();
+    if (warp == 0) {
+      int base = 0;
+      for (int e0 = 0; e0 < args.groups; e0 += 32) {
+        const int e = e0 + lane;
+        const bool used = e < args.groups && s_off[e + 1] > s_off[e];
+        const unsigned m = __ballot_sync(0xffffffffu, used);
+        if (used) s_toff[base + __popc(m & ((1u << lane) - 1u))] = e;
+        base += __popc(m);
+      }
+      if (lane == 0) s_toff[C::kMaxGroups] = base;
+    }
+  }
   if (warp == R::kMmaWarp) {
     __syncwarp();
     tmem_alloc<C::kTmemCols>(smem_u32(tmem_slot));
@@ -294,7 +312,7 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
   const uint32_t tmem_base = *tmem_slot;
 
   const int total = is_router<MODE>()   ? static_cast<int>((args.m_rows + BM - 1) / BM)
-                    : is_decode<MODE>() ? args.groups * args.n_tiles
+                    : is_decode<MODE>() ? s_toff[C::kMaxGroups] * args.n_tiles
                                         : s_toff[args.groups] * args.n_tiles;
 
   if (MODE == kGateUpGather && warp < R::kProdWarps) {
