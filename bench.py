@@ -259,7 +259,7 @@ def run_ours(args, rank, world, local, pg):
     kern["gate_up"].update(tflops=gu_tf, frac=gu_tf / pk["bf16_sus"])
     kern["down"].update(tflops=dn_tf, frac=dn_tf / pk["bf16_sus"])
 
-    route = route_stress(moe, args, stream, dev, pk)
+    route = route_stress(moe, args, stream, dev, pk, cpu=rank == 0 and not args.no_cpu_baseline)
     others = other_configs(moe, args, stream, dev, pk, pg)
 
     # end to end through the public API with host buffers: every step copies
@@ -561,14 +561,16 @@ def other_configs(moe, args, stream, dev, pk, pg):
     return res
 
 
-def route_stress(moe, args, stream, dev, pk):
-    """elbow_route and moe_dispatch on the 1,048,576 x 64 fp32-logit stress."""
+def route_stress(moe, args, stream, dev, pk, cpu=False):
+    """elbow_route and moe_dispatch on the 1,048,576 x 64 fp32-logit stress;
+    with cpu, also the oracle routing a bounded sample of the same logits."""
     import torch
     from paper_2608_04401_gb300 import synth
     w = synth.WORKLOADS[ROUTE_WORKLOAD]
     T, N, K = w["T"], w["N"], w["K"]
     rng = np.random.Generator(np.random.PCG64(w["seed"]))
-    lg = torch.from_numpy(synth.boosted_logits(rng, T, N)).to(dev)
+    lg_host = synth.boosted_logits(rng, T, N)
+    lg = torch.from_numpy(lg_host).to(dev)
     k = torch.empty(T, dtype=torch.int32, device=dev)
     ids = torch.empty(T, K, dtype=torch.int32, device=dev)
     gates = torch.empty(T, K, dtype=torch.float32, device=dev)
@@ -624,7 +626,26 @@ def route_stress(moe, args, stream, dev, pk):
     bd = T * (4 + 4 * K) + 4 * sum_k + 4 * T * K
     gr = br / (ms_r * 1e-3) / 1e9
     gd = bd / (ms_d * 1e-3) / 1e9
+    cpu_route = None
+    if cpu:
+        # the oracle (C, fp32 routing, OpenMP) on the first 2^17 tokens, and
+        # whether the GPU's k and ids of that sample are its bits
+        import oracle
+        n = 1 << 17
+        route()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        r = oracle.route(lg_host[:n], K=K)
+        dt = time.perf_counter() - t0
+        same = bool(np.array_equal(r["k"], k[:n].cpu().numpy()) and
+                    np.array_equal(r["ids"], ids[:n].cpu().numpy()))
+        cpu_route = {"tokens_per_s": n / dt, "GBps": n * (4 * N + 4 + 8 * K) / dt / 1e9,
+                     "cores": int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1)),
+                     "cpu": cpu_model(), "kind": "oracle",
+                     "sample": f"the first {n} of the {T} tokens, {dt:.2f} s",
+                     "gpu_bitexact_on_sample": same}
     return {"workload": f"{ROUTE_WORKLOAD}: T={T} x N={N} fp32 logits, K={K}",
+            "cpu_oracle_route": cpu_route,
             "route": {"ms": ms_r, "GBps": gr, "frac": gr / pk["hbm"], "bytes": br,
                       "tokens_per_s": T / (ms_r * 1e-3)},
             "dispatch": {"ms": ms_d, "GBps": gd, "frac": gd / pk["hbm"], "bytes": bd},
@@ -644,6 +665,27 @@ def route_stress(moe, args, stream, dev, pk):
                 "elbow_index_hist": st["elbow_hist"][:16].tolist()}}
 
 
+def cpu_model():
+    """The host CPU's model string from /proc/cpuinfo (Arm hosts: implementer/part)."""
+    try:
+        with open("/proc/cpuinfo") as f:
+            info = f.read()
+    except OSError:
+        return "unknown"
+    for key in ("model name", "Model"):
+        for line in info.splitlines():
+            if line.startswith(key) and ":" in line:
+                return line.split(":", 1)[1].strip()
+    fields = {}
+    for line in info.splitlines():
+        if ":" in line:
+            k_, v_ = (x.strip() for x in line.split(":", 1))
+            fields.setdefault(k_, v_)
+    if "CPU implementer" in fields:
+        return f"Arm implementer {fields['CPU implementer']}, part {fields.get('CPU part', '?')}"
+    return "unknown"
+
+
 def cpu_baseline(inp, K, budget_s=12.0):
     """The CPU oracle, as it stands, on a bounded sample of the same workload."""
     import oracle
@@ -658,7 +700,7 @@ def cpu_baseline(inp, K, budget_s=12.0):
     oracle.layer_rows(inp["x"], inp["w_router"], inp["w_gate_up"], inp["w_down"], rows=rows, K=K)
     dt = time.perf_counter() - t0
     cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
-    return {"value": n / dt, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+    return {"value": n / dt, "unit": "tokens/s", "cores": cores, "kind": "oracle", "cpu": cpu_model(),
             "sample": f"{n} of the {T} tokens of the same layer (fp64 C oracle, OpenMP), {dt:.1f} s"}
 
 
