@@ -442,25 +442,29 @@ MOE_DEV int route_token(float* row, int64_t t, int tid, int K, float eps, int to
   float emin;
   const float r = softmax_row<N>(row, emin);
 
-  // ---- the kTop largest e, each key = truncated value | (N-1 - id)
-  uint32_t key[N];
+  // ---- the kTop largest e, each key = truncated value | (N-1 - id): one
+  // 32-key network (a loop, not unrolled, so its code is fetched once) sorts
+  // each 32-expert slice into key[32..64); the running top 32 is key[0..32)
+  uint32_t key[64];
+#pragma unroll 1
+  for (int h = 0; h < N / 32; ++h) {
 #pragma unroll
-  for (int c = 0; c < N; c += 4) {
-    const float4 q = *reinterpret_cast<const float4*>(row + c);
-    key[c] = (__float_as_uint(q.x) & ~kIdMask) | (kIdMask - c);
-    key[c + 1] = (__float_as_uint(q.y) & ~kIdMask) | (kIdMask - (c + 1));
-    key[c + 2] = (__float_as_uint(q.z) & ~kIdMask) | (kIdMask - (c + 2));
-    key[c + 3] = (__float_as_uint(q.w) & ~kIdMask) | (kIdMask - (c + 3));
+    for (int c = 0; c < 32; c += 4) {
+      const int j = 32 * h + c;
+      const float4 q = *reinterpret_cast<const float4*>(row + j);
+      key[32 + c] = (__float_as_uint(q.x) & ~kIdMask) | (kIdMask - j);
+      key[32 + c + 1] = (__float_as_uint(q.y) & ~kIdMask) | (kIdMask - (j + 1));
+      key[32 + c + 2] = (__float_as_uint(q.z) & ~kIdMask) | (kIdMask - (j + 2));
+      key[32 + c + 3] = (__float_as_uint(q.w) & ~kIdMask) | (kIdMask - (j + 3));
+    }
+    sort_desc_at<32, 32>(key);
+    if (h == 0) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i) key[i] = key[32 + i];
+    } else {
+      merge_keep_top32<0, 32>(key);
+    }
   }
-  sort_desc_at<32, 0>(key);
-  sort_desc_at<32, 32>(key);
-  if constexpr (N == 128) {
-    sort_desc_at<32, 64>(key);
-    sort_desc_at<32, 96>(key);
-    merge_keep_top32<64, 96>(key);
-  }
-  merge_keep_top32<0, 32>(key);
-  if constexpr (N == 128) merge_keep_top32<0, 64>(key);
 
   // ---- exact values of the selected ranks, and the proof that they are the
   // exact top ranks in exact order
