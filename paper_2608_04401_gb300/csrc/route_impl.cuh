@@ -294,7 +294,7 @@ MOE_DEV void write_outputs(int64_t t, int K, int k, const int (&ids)[8], const f
 // with s the balanced tree sum of the e_j.
 template <int N>
 MOE_DEV float softmax_row(float* row, float& emin) {
-  uint64_t ep[N / 2];
+  float m;
   {
     float l[N];
 #pragma unroll
@@ -306,15 +306,29 @@ MOE_DEV float softmax_row(float* row, float& emin) {
     float acc[4] = {l[0], l[1], l[2], l[3]};
 #pragma unroll
     for (int j = 4; j < N; j += 2) acc[(j / 2) % 4] = max3f(acc[(j / 2) % 4], l[j], l[j + 1]);
-    const float m = fmaxf(max3f(acc[0], acc[1], acc[2]), acc[3]);
-    const uint64_t mm = pk(m, m);
-#pragma unroll
-    for (int a = 0; a < N / 2; ++a) ep[a] = exp_spec2(sub2(pk(l[2 * a], l[2 * a + 1]), mm));
+    m = fmaxf(max3f(acc[0], acc[1], acc[2]), acc[3]);
   }
+  const uint64_t mm = pk(m, m);
+  // e_j = EXP(l_j - m), eight at a time in place in the row; the loop is not
+  // unrolled, so its code is fetched once instead of N / 8 times
+#pragma unroll 1
+  for (int c = 0; c < N; c += 8) {
+    const float4 q0 = *reinterpret_cast<const float4*>(row + c);
+    const float4 q1 = *reinterpret_cast<const float4*>(row + c + 4);
+    const uint64_t e0 = exp_spec2(sub2(pk(q0.x, q0.y), mm));
+    const uint64_t e1 = exp_spec2(sub2(pk(q0.z, q0.w), mm));
+    const uint64_t e2 = exp_spec2(sub2(pk(q1.x, q1.y), mm));
+    const uint64_t e3 = exp_spec2(sub2(pk(q1.z, q1.w), mm));
+    *reinterpret_cast<float4*>(row + c) = make_float4(lo_of(e0), hi_of(e0), lo_of(e1), hi_of(e1));
+    *reinterpret_cast<float4*>(row + c + 4) = make_float4(lo_of(e2), hi_of(e2), lo_of(e3), hi_of(e3));
+  }
+  uint64_t ep[N / 2];
 #pragma unroll
-  for (int c = 0; c < N; c += 4)
-    *reinterpret_cast<float4*>(row + c) =
-        make_float4(lo_of(ep[c / 2]), hi_of(ep[c / 2]), lo_of(ep[c / 2 + 1]), hi_of(ep[c / 2 + 1]));
+  for (int c = 0; c < N; c += 4) {
+    const float4 q = *reinterpret_cast<const float4*>(row + c);
+    ep[c / 2] = pk(q.x, q.y);
+    ep[c / 2 + 1] = pk(q.z, q.w);
+  }
   {
     // four interleaved 3-input min chains over the pairs ep[2 ..)
     float acc[4] = {lo_of(ep[0]), hi_of(ep[0]), lo_of(ep[1]), hi_of(ep[1])};
