@@ -128,6 +128,27 @@ MOE_DEV uint64_t exp_spec2(uint64_t z) {
   return mul2(q, scale);
 }
 
+// exp_spec2 for arguments z >= -87 (so that n >= -126): both clamps above are
+// then no-ops, and this is the same sequence of operations without them.
+MOE_DEV uint64_t exp_spec2_inrange(uint64_t z) {
+  const uint64_t t = mul2(z, pk(kLog2e, kLog2e));
+  const uint64_t tm = add2(t, pk(kMagic, kMagic));
+  const uint64_t n = sub2(tm, pk(kMagic, kMagic));
+  uint64_t r = fma2(n, pk(-kLn2Hi, -kLn2Hi), z);
+  r = fma2(n, pk(-kLn2Lo, -kLn2Lo), r);
+  uint64_t q = fma2(pk(kTay7, kTay7), r, pk(kTay6, kTay6));
+  q = fma2(q, r, pk(kTay5, kTay5));
+  q = fma2(q, r, pk(kTay4, kTay4));
+  q = fma2(q, r, pk(kTay3, kTay3));
+  q = fma2(q, r, pk(kTay2, kTay2));
+  q = fma2(q, r, pk(kTay1, kTay1));
+  q = fma2(q, r, pk(kTay0, kTay0));
+  const int32_t b0 = __float_as_int(lo_of(tm)), b1 = __float_as_int(hi_of(tm));
+  const uint64_t scale = pk(__int_as_float((b0 - kMagicBits + 127) << 23),
+                            __int_as_float((b1 - kMagicBits + 127) << 23));
+  return mul2(q, scale);
+}
+
 // -------------------------------------------------------- sorting networks
 // Batcher's odd-even merge sort network for M keys, as a flat comparator list
 // built at compile time (so that every register index is a constant).
@@ -294,7 +315,7 @@ MOE_DEV void write_outputs(int64_t t, int K, int k, const int (&ids)[8], const f
 // with s the balanced tree sum of the e_j.
 template <int N>
 MOE_DEV float softmax_row(float* row, float& emin) {
-  float m;
+  float m, lmin;
   {
     float l[N];
 #pragma unroll
@@ -302,26 +323,40 @@ MOE_DEV float softmax_row(float* row, float& emin) {
       const float4 q = *reinterpret_cast<const float4*>(row + c);
       l[c] = q.x; l[c + 1] = q.y; l[c + 2] = q.z; l[c + 3] = q.w;
     }
-    // four interleaved 3-input max chains over l[4 ..), two elements per step
+    // four interleaved 3-input max (and min) chains over l[4 ..), two elements per step
     float acc[4] = {l[0], l[1], l[2], l[3]};
+    float acn[4] = {l[0], l[1], l[2], l[3]};
 #pragma unroll
-    for (int j = 4; j < N; j += 2) acc[(j / 2) % 4] = max3f(acc[(j / 2) % 4], l[j], l[j + 1]);
+    for (int j = 4; j < N; j += 2) {
+      acc[(j / 2) % 4] = max3f(acc[(j / 2) % 4], l[j], l[j + 1]);
+      acn[(j / 2) % 4] = min3f(acn[(j / 2) % 4], l[j], l[j + 1]);
+    }
     m = fmaxf(max3f(acc[0], acc[1], acc[2]), acc[3]);
+    lmin = fminf(min3f(acn[0], acn[1], acn[2]), acn[3]);
   }
   const uint64_t mm = pk(m, m);
   // e_j = EXP(l_j - m), eight at a time in place in the row; the loop is not
-  // unrolled, so its code is fetched once instead of N / 8 times
+  // unrolled, so its code is fetched once instead of N / 8 times. When every
+  // l_j - m >= -87 (rounded as in the loop) the clamps of EXP cannot act, and
+  // the same operations run without them.
+  auto exp_pass = [&](auto ex) {
 #pragma unroll 1
-  for (int c = 0; c < N; c += 8) {
-    const float4 q0 = *reinterpret_cast<const float4*>(row + c);
-    const float4 q1 = *reinterpret_cast<const float4*>(row + c + 4);
-    const uint64_t e0 = exp_spec2(sub2(pk(q0.x, q0.y), mm));
-    const uint64_t e1 = exp_spec2(sub2(pk(q0.z, q0.w), mm));
-    const uint64_t e2 = exp_spec2(sub2(pk(q1.x, q1.y), mm));
-    const uint64_t e3 = exp_spec2(sub2(pk(q1.z, q1.w), mm));
-    *reinterpret_cast<float4*>(row + c) = make_float4(lo_of(e0), hi_of(e0), lo_of(e1), hi_of(e1));
-    *reinterpret_cast<float4*>(row + c + 4) = make_float4(lo_of(e2), hi_of(e2), lo_of(e3), hi_of(e3));
-  }
+    for (int c = 0; c < N; c += 8) {
+      const float4 q0 = *reinterpret_cast<const float4*>(row + c);
+      const float4 q1 = *reinterpret_cast<const float4*>(row + c + 4);
+      const uint64_t e0 = ex(sub2(pk(q0.x, q0.y), mm));
+      const uint64_t e1 = ex(sub2(pk(q0.z, q0.w), mm));
+      const uint64_t e2 = ex(sub2(pk(q1.x, q1.y), mm));
+      const uint64_t e3 = ex(sub2(pk(q1.z, q1.w), mm));
+      *reinterpret_cast<float4*>(row + c) = make_float4(lo_of(e0), hi_of(e0), lo_of(e1), hi_of(e1));
+      *reinterpret_cast<float4*>(row + c + 4) =
+          make_float4(lo_of(e2), hi_of(e2), lo_of(e3), hi_of(e3));
+    }
+  };
+  if (__fsub_rn(lmin, m) >= -87.0f)
+    exp_pass([](uint64_t z) { return exp_spec2_inrange(z); });
+  else
+    exp_pass([](uint64_t z) { return exp_spec2(z); });
   uint64_t ep[N / 2];
 #pragma unroll
   for (int c = 0; c < N; c += 4) {

@@ -66,9 +66,11 @@ def test_route_edge_cases(moe):
     r = np.zeros(N); r[::2] = 1e-7; rows.append(r)   # distinct logits, equal probabilities
     r = np.linspace(-60, 30, N); rows.append(r)      # wide range
     rng = np.random.default_rng(0)
-    # logit ranges around 86 (the unclamped exponential's domain ends there)
-    # and around the exponential's underflow limits (-87.3, -104)
-    for zlow in (-85.99, -86.0, -86.01, -87.0, -87.4, -87.8, -103.9, -104.0, -104.3, -104.6):
+    # logit ranges around 87 (rows whose range is within 87 run the exponential
+    # without its clamps) and around the exponential's underflow limits
+    # (-87.3, -104)
+    for zlow in (-85.99, -86.0, -86.01, -86.999, -87.0, -87.001, -87.4, -87.8, -103.9, -104.0,
+                 -104.3, -104.6):
         r = rng.uniform(-3.0, 0.0, N); r[0] = 0.0; r[7] = zlow; rows.append(r)
         r = rng.uniform(zlow, zlow + 1.5, N); r[3] = 0.0; r[4] = -0.5; rows.append(r)
     q = np.round(rng.standard_normal((200, N)) * 2) / 2   # many exact ties
