@@ -86,10 +86,9 @@ struct Cfg {
   static constexpr int kABytes = BM * BK * 2;
   static constexpr int kBBytes = BN * BK * 2;
   static constexpr int kStageBytes = kABytes + kBBytes;
-  // fused routing: logit rows [128][BN + 4] fp32, 8 x 128 key slots, histogram
+  // fused routing: logit rows [128][BN + 4] fp32, histogram
   static constexpr int kRouteTileBytes = 128 * (BN + 4) * 4;
-  static constexpr int kRouteBytes =
-      MODE == kRouterFused ? kRouteTileBytes + 8 * 128 * 8 + BN * 4 : 0;
+  static constexpr int kRouteBytes = MODE == kRouterFused ? kRouteTileBytes + BN * 4 : 0;
   // kDown: per epilogue warp two 32 x 32 bf16 staging tiles for TMA stores;
   // kDecGateUp: the up half of the accumulator, [64 rows][65] fp32
   static constexpr int kEpiBytes =
@@ -520,8 +519,7 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
       } else if (MODE == kRouterFused) {
         // logits -> this thread's row in shared memory (and to global if asked)
         float* rtile = reinterpret_cast<float*>(smem + C::kRouteOff);
-        uint64_t* keys64 = reinterpret_cast<uint64_t*>(smem + C::kRouteOff + C::kRouteTileBytes);
-        int* hist = reinterpret_cast<int*>(smem + C::kRouteOff + C::kRouteTileBytes + 8 * 128 * 8);
+        int* hist = reinterpret_cast<int*>(smem + C::kRouteOff + C::kRouteTileBytes);
         float* row = rtile + r * (BN + 4);
         float* gout = args.out ? static_cast<float*>(args.out) + grow * args.ldo : nullptr;
 #pragma unroll
@@ -547,10 +545,20 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
         }
         int ids_sel[8];
         int k_sel = 0;
+        float rs = 0.0f;
         if (valid)
-          k_sel = route::route_token<BN, RouteX>(row, grow, r, args.K, args.eps, args.topk_mode,
-                                                 args.renorm, args.rx, keys64, args.k_out,
-                                                 args.ids_out, args.gates_out, ids_sel);
+          k_sel = route::route_token<BN, RouteX>(row, grow, args.K, args.eps, args.topk_mode,
+                                                 args.renorm, args.rx, args.k_out, args.ids_out,
+                                                 args.gates_out, ids_sel, rs);
+        // tokens the fast path left undecided: routed by their whole warp
+        const unsigned undecided = __ballot_sync(0xffffffffu, valid && k_sel < 0);
+        if constexpr (BN >= 64) if (undecided) {
+          const float* wrow = rtile + q * 32 * (BN + 4);
+          route::route_undecided<BN>(
+              undecided, [&](int l) { return wrow + l * (BN + 4); }, rs, grow, args.K, args.eps,
+              args.topk_mode, args.renorm, args.k_out, args.ids_out, args.gates_out, k_sel,
+              ids_sel);
+        }
         if (args.blk_cnt) {
 #pragma unroll
           for (int s2 = 0; s2 < 8; ++s2)

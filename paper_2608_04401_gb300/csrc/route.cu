@@ -79,7 +79,6 @@ __global__ void __launch_bounds__(kTok) elbow_route_kernel(
   extern __shared__ float4 smem4[];
   __shared__ int hist[N];
   float* tile = reinterpret_cast<float*>(smem4);
-  uint64_t* keys64 = reinterpret_cast<uint64_t*>(tile + kTok * kPitch);  // [8][kTok]
 
   const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kTok;
   const int ntok = static_cast<int>(min_of<int64_t>(kTok, T - t0));
@@ -99,9 +98,19 @@ __global__ void __launch_bounds__(kTok) elbow_route_kernel(
   __syncthreads();
   int ids_sel[8];
   int k_sel = 0;
-  if (tid < ntok) {
-    k_sel = route_token<N, RouteConsts<N>>(tile + tid * kPitch, t0 + tid, tid, K, eps, topk_mode,
-                                           renorm, rc, keys64, k_out, ids_out, gates_out, ids_sel);
+  float r = 0.0f;
+  const bool valid = tid < ntok;
+  if (valid)
+    k_sel = route_token<N, RouteConsts<N>>(tile + tid * kPitch, t0 + tid, K, eps, topk_mode,
+                                           renorm, rc, k_out, ids_out, gates_out, ids_sel, r);
+  // tokens the fast path left undecided: routed by their whole warp
+  const unsigned undecided = __ballot_sync(0xffffffffu, valid && k_sel < 0);
+  if (undecided) {
+    const float* wrow = tile + (tid & ~31) * kPitch;
+    route_undecided<N>(undecided, [&](int l) { return wrow + l * kPitch; }, r, t0 + tid, K, eps,
+                       topk_mode, renorm, k_out, ids_out, gates_out, k_sel, ids_sel);
+  }
+  if (valid) {
     if constexpr (RAND) {
       randomize_token<N>(tile + tid * kPitch, t0 + tid, K, rand_mode, renorm, k_sel, ids_sel, rand,
                          k_out, ids_out, gates_out);
@@ -126,7 +135,7 @@ cudaError_t launch(const float* logits, int64_t T, int K, float eps, int topk_mo
                    const uint32_t* rand, int rand_mode, cudaStream_t stream) {
   RouteConsts<N> rc;
   fill_route_consts(rc, N);
-  constexpr size_t smem = smem_bytes<N>();
+  constexpr size_t smem = route_smem_bytes<N>();
   auto kern = rand_mode ? elbow_route_kernel<N, true> : elbow_route_kernel<N, false>;
   static std::atomic<uint64_t> attr_done{0};
   const cudaError_t ae = once_per_device(attr_done, [] {

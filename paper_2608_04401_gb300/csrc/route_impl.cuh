@@ -19,15 +19,15 @@
 //   M_head = max_{i < K-1} D_i (first argmax), M_mid = max_{K-1 <= i < kTop-1} D_i
 //   M_head >= M_mid and M_head >= bound  ->  k = argmax + 1
 //   M_mid > M_head                        ->  k = K (the elbow lies at or past K-1)
-//   otherwise, or when a check fails      ->  exact full path (rare)
+//   otherwise, or when a check fails      ->  undecided (rare)
 // Sorting is by e, not p; p = fl(e * (1/s)) is monotone in e, so the curve is
 // the same, and ids inside groups of equal p are re-ordered by ascending id.
-// A p tie across the K boundary also takes the full path.
+// A p tie across the K boundary also leaves the token undecided.
 //
-// Full path (fallback, one thread, same arithmetic): all N probabilities are
-// sorted with a 543/1471-comparator Batcher network of fmaxf/fminf, the elbow
-// is evaluated on every rank, and the top-K ids are recovered by a threshold
-// scan of the unsorted row plus an 8-key network.
+// Undecided tokens (same arithmetic, every rank): the whole warp routes each
+// of them in turn from its softmax numerators, sorting all N (p, id) keys by
+// a bitonic network of shuffles (route_undecided / warp_route_from_e), instead
+// of one lane running a full sort while the rest of its warp waits.
 #pragma once
 
 #include <utility>
@@ -281,9 +281,16 @@ inline void fill_route_consts(RC& rc, int N) {
   rc.bound = 1.0f - rc.x[kTop - 1];
 }
 
+// Shared memory of a 128-token block: the [kTok][N + 4] row tile, plus eight
+// 8-byte key slots per token for the full-sort helpers (topk_ids).
 template <int N>
 constexpr size_t smem_bytes() {
   return sizeof(float) * kTok * (N + 4) + sizeof(uint64_t) * 8 * kTok;
+}
+// ... and of the routing kernel, which needs the row tile only.
+template <int N>
+constexpr size_t route_smem_bytes() {
+  return sizeof(float) * kTok * (N + 4);
 }
 
 MOE_DEV void write_outputs(int64_t t, int K, int k, const int (&ids)[8], const float (&g)[8],
@@ -307,9 +314,6 @@ MOE_DEV void write_outputs(int64_t t, int K, int k, const int (&ids)[8], const f
   }
 }
 
-// Exact full path for one token, from the row of e values in shared memory
-// and r = 1/s: every probability sorted, the elbow evaluated on every rank,
-// the top-K ids from a threshold scan. Writes the token's outputs.
 // Softmax numerators of one token: e_j = EXP(l_j - m) for the N logits in
 // row, written back into the row; the smallest e_j in emin; returns r = 1/s
 // with s the balanced tree sum of the e_j.
@@ -430,66 +434,145 @@ MOE_DEV void topk_ids(const float* row, float r, const float (&v)[N], int K, uin
   for (int s = 0; s < 8; ++s) ids[s] = ~static_cast<int>(key[s]);
 }
 
-template <int N, typename RC>
-__device__ __noinline__ int route_full(const float* row, float r, int K, float eps, int topk_mode,
-                                        int renorm, const RC& rc, uint64_t* keys,
-                                        int tid, int64_t t, int32_t* k_out, int32_t* ids_out,
-                                        float* gates_out) {
-  float v[N];
-  sorted_probs<N>(row, r, v);
-
-  int k = K;
-  if (!topk_mode) {
-    const float p_min = v[N - 1];
-    const float inv = __frcp_rn(__fadd_rn(__fsub_rn(v[0], p_min), eps));
-    float best = -__int_as_float(0x7f800000), tail = -__int_as_float(0x7f800000);
-    int e = 0;
+// Routes token t with the calling (whole, converged) warp from the token's
+// softmax numerators e (lane l holds experts l + 32c in e[c]) and r = 1/s,
+// in the routing specification's arithmetic: p_j = e_j * r; a bitonic sort of
+// the N keys (p bits << 32 | ~id) across the warp, which orders by p
+// descending and ascending id on ties; p'_i and D_i on every rank; the first
+// argmax by a (max D, min index) warp reduction; k = min(e + 1, K). Writes the
+// token's outputs; returns k, and lane s < K gets the id of rank s in sel_id.
+template <int N>
+MOE_DEV int warp_route_from_e(const float (&e)[N / 32], float r, int64_t t, int K, float eps,
+                              int topk_mode, int renorm, int32_t* __restrict__ k_out,
+                              int32_t* __restrict__ ids_out, float* __restrict__ gates_out,
+                              int& sel_id) {
+  constexpr int C = N / 32;
+  const unsigned full = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  uint64_t key[C];
 #pragma unroll
-    for (int i = 0; i < N; ++i) {
-      const float pn = __fmul_rn(__fsub_rn(v[i], p_min), inv);
-      const float D = __fsub_rn(__fsub_rn(1.0f, pn), rc.x[i]);
-      if (i < 7 && i < K - 1) {
-        if (D > best) { best = D; e = i; }
-      } else {
-        tail = fmaxf(tail, D);
+  for (int c = 0; c < C; ++c) {
+    const float p = __fmul_rn(e[c], r);
+    key[c] = (static_cast<uint64_t>(__float_as_uint(p)) << 32) |
+             static_cast<uint32_t>(~(32 * c + lane));
+  }
+  // bitonic sort, descending; element j = 32 c + lane
+#pragma unroll
+  for (int k2 = 2; k2 <= N; k2 <<= 1) {
+#pragma unroll
+    for (int jj = k2 >> 1; jj > 0; jj >>= 1) {
+      uint64_t nk[C];
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const int j = 32 * c + lane;
+        const uint64_t other =
+            jj >= 32 ? key[c ^ (jj / 32)] : __shfl_xor_sync(full, key[c], jj);
+        const bool lower = (j & jj) == 0;
+        const bool desc = (j & k2) == 0;
+        const uint64_t hi = key[c] > other ? key[c] : other;
+        const uint64_t lo = key[c] > other ? other : key[c];
+        nk[c] = (lower == desc) ? hi : lo;
       }
+#pragma unroll
+      for (int c = 0; c < C; ++c) key[c] = nk[c];
     }
-    k = (best >= tail) ? e + 1 : K;
   }
-
-  int ids[8];
-  topk_ids<N>(row, r, v, K, keys, tid, ids);
-  float g[8];
+  // the elbow over all ranks (rank of element j is j)
+  const float pmax = __uint_as_float(static_cast<uint32_t>(__shfl_sync(full, key[0], 0) >> 32));
+  const float pmin =
+      __uint_as_float(static_cast<uint32_t>(__shfl_sync(full, key[C - 1], 31) >> 32));
+  const float inv = __frcp_rn(__fadd_rn(__fsub_rn(pmax, pmin), eps));
+  float best = 0.0f;
+  int bi = 0;
+#pragma unroll
+  for (int c = 0; c < C; ++c) {
+    const int i = 32 * c + lane;
+    const float p = __uint_as_float(static_cast<uint32_t>(key[c] >> 32));
+    const float pn = __fmul_rn(__fsub_rn(p, pmin), inv);
+    const float xi = __fdiv_rn(static_cast<float>(i), static_cast<float>(N - 1));
+    const float D = __fsub_rn(__fsub_rn(1.0f, pn), xi);
+    if (c == 0 || D > best) {
+      best = D;
+      bi = i;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+    const float ob = __shfl_xor_sync(full, best, o);
+    const int oi = __shfl_xor_sync(full, bi, o);
+    if (ob > best || (ob == best && oi < bi)) {
+      best = ob;
+      bi = oi;
+    }
+  }
+  const int k = topk_mode ? K : min(bi + 1, K);
+  // ranks 0 .. K-1 are slot 0 of lanes 0 .. K-1
+  const float p = __uint_as_float(static_cast<uint32_t>(key[0] >> 32));
+  const int id = static_cast<int>(~static_cast<uint32_t>(key[0]));
   float S = 0.0f;
+  if (renorm) {
 #pragma unroll
-  for (int s = 0; s < 8; ++s)
-    if (s < k) S = __fadd_rn(S, v[s]);
-#pragma unroll
-  for (int s = 0; s < 8; ++s) {
-    const float p = renorm ? __fdiv_rn(v[s], S) : v[s];
-    g[s] = (s < k) ? p : 0.0f;
+    for (int s2 = 0; s2 < 8; ++s2) {
+      const float ps = __shfl_sync(full, p, s2);
+      if (s2 < k) S = __fadd_rn(S, ps);
+    }
   }
-  write_outputs(t, K, k, ids, g, k_out, ids_out, gates_out);
-  // leave the ids for the caller in this thread's own 8-byte key slots
-  // (keys[s * kTok + tid]; a 4-byte view of that array would overlap the
-  // slots of other threads, which may still be staging their keys)
-#pragma unroll
-  for (int s = 0; s < 8; ++s) keys[s * kTok + tid] = static_cast<uint32_t>(ids[s]);
+  if (lane < K) {
+    ids_out[t * K + lane] = id;
+    gates_out[t * K + lane] = lane < k ? (renorm ? __fdiv_rn(p, S) : p) : 0.0f;
+  }
+  if (lane == 0) k_out[t] = k;
+  sel_id = id;
   return k;
 }
 
-// Routes the token of this thread (its logits are in `row`); writes its
-// outputs and returns k, with the selected ids in ids_sel.
+// The tokens of this warp that route_token left undecided (lane l's bit in
+// `undecided`; its softmax numerators in row_of(l)[0 .. N), its 1/s in r,
+// its token index in t) are routed one after another by the whole warp;
+// their lanes receive k in k_sel and the selected ids in ids_sel. Every lane
+// of the warp must call this.
+template <int N, typename RowOf>
+MOE_DEV void route_undecided(unsigned undecided, RowOf row_of, float r, int64_t t, int K,
+                             float eps, int topk_mode, int renorm, int32_t* __restrict__ k_out,
+                             int32_t* __restrict__ ids_out, float* __restrict__ gates_out,
+                             int& k_sel, int (&ids_sel)[8]) {
+  const unsigned full = 0xffffffffu;
+  const int lane = threadIdx.x & 31;
+  while (undecided) {
+    const int src = __ffs(static_cast<int>(undecided)) - 1;
+    undecided &= undecided - 1u;
+    const float* srow = row_of(src);
+    float e[N / 32];
+#pragma unroll
+    for (int c = 0; c < N / 32; ++c) e[c] = srow[32 * c + lane];
+    const float rs = __shfl_sync(full, r, src);
+    const int64_t ts = __shfl_sync(full, t, src);
+    int sel = 0;
+    const int kf = warp_route_from_e<N>(e, rs, ts, K, eps, topk_mode, renorm, k_out, ids_out,
+                                        gates_out, sel);
+#pragma unroll
+    for (int s2 = 0; s2 < 8; ++s2) {
+      const int id_s = __shfl_sync(full, sel, s2);
+      if (lane == src) ids_sel[s2] = id_s;
+    }
+    if (lane == src) k_sel = kf;
+  }
+}
+
+// Routes the token of this thread (its logits are in `row`): writes its
+// outputs and returns k, with the selected ids in ids_sel; or, when the fast
+// path cannot settle the token, returns -1 and writes nothing (the row then
+// holds the softmax numerators and r_out = 1/s, for route_undecided).
 template <int N, typename RC>
-MOE_DEV int route_token(float* row, int64_t t, int tid, int K, float eps, int topk_mode, int renorm,
-                        const RC& rc, uint64_t* keys64, int32_t* __restrict__ k_out,
-                        int32_t* __restrict__ ids_out, float* __restrict__ gates_out,
-                        int (&ids_sel)[8]) {
+MOE_DEV int route_token(float* row, int64_t t, int K, float eps, int topk_mode, int renorm,
+                        const RC& rc, int32_t* __restrict__ k_out, int32_t* __restrict__ ids_out,
+                        float* __restrict__ gates_out, int (&ids_sel)[8], float& r_out) {
   constexpr uint32_t kIdMask = N - 1;
 
   // ---- e_j = EXP(l_j - m), stored back into the row; e_min; s; r = 1/s
   float emin;
   const float r = softmax_row<N>(row, emin);
+  r_out = r;
 
   // ---- the kTop largest e, each key = truncated value | (N-1 - id): one
   // 32-key network (a loop, not unrolled, so its code is fetched once) sorts
@@ -582,14 +665,7 @@ MOE_DEV int route_token(float* row, int64_t t, int tid, int K, float eps, int to
     if (s < K) pKm1 = fminf(pKm1, pv[s]);
   if (pKm1 == pK) ok = false;  // a tie across the K boundary
 
-  if (!ok) {
-    const int kf =
-        route_full<N, RC>(row, r, K, eps, topk_mode, renorm, rc, keys64, tid, t, k_out, ids_out,
-                          gates_out);
-#pragma unroll
-    for (int s = 0; s < 8; ++s) ids_sel[s] = static_cast<int>(keys64[s * kTok + tid]);
-    return kf;
-  }
+  if (!ok) return -1;
 
   int ids[8];
   float g[8];
