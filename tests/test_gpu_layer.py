@@ -66,8 +66,9 @@ def test_grouped_gemm_steps(moe, N, counts):
         k, ids = r["k"], r["ids"]
         gates = r["gates"]
     else:
-        # expert sizes 0, 1, 127, 128, 129, 256, 300 (ragged m-tiles)
-        sizes = {3: 1, 5: 127, 6: 128, 7: 129, 9: 256, 11: 300}
+        # expert sizes 0, 1, 65, 127, 128, 129, 192, 193, 300: ragged last
+        # m-tiles of 1, 44, 64, 65, 127 and 128 rows
+        sizes = {3: 1, 5: 127, 6: 128, 7: 129, 9: 192, 11: 300, 13: 65, 15: 193}
         T = 300
         ids = np.zeros((T, K), np.int32)
         k = np.zeros(T, np.int32)
