@@ -215,7 +215,18 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
       if (offsets_copy) offsets_copy[N] = total_pairs;
     }
   };
+  // every global input of the block is requested first, so that their
+  // latencies overlap: the tokens' selections, the expert totals and this
+  // chunk's per-expert base counts
+  // (with GATHER every block works on the one chunk)
+  const int64_t t = (GATHER ? 0 : static_cast<int64_t>(blockIdx.x) * kChunk) + tid;
+  const bool valid = t < T;
+  int kt, my[8];
+  uint64_t m0, m1;
+  load_selection(k, ids, t, valid, K, kt, my, m0, m1);
+  int chunk_base = 0;
   if constexpr (!SINGLE) {
+    if (tid < N) chunk_base = base[static_cast<int64_t>(tid) * nblk + blockIdx.x];
     // expert offsets from the totals (every chunk recomputes them)
     const int tot = tid < N ? totals[tid] : 0;
     int total_pairs;
@@ -223,13 +234,6 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
     if (tid < N) exp_off[tid] = off;
     if (blockIdx.x == 0) write_offsets(tot, off, total_pairs);
   }
-
-  // (with GATHER every block works on the one chunk)
-  const int64_t t = (GATHER ? 0 : static_cast<int64_t>(blockIdx.x) * kChunk) + tid;
-  const bool valid = t < T;
-  int kt, my[8];
-  uint64_t m0, m1;
-  load_selection(k, ids, t, valid, K, kt, my, m0, m1);
 #pragma unroll
   for (int q = 0; q < N / 32; ++q) bal[warp][32 * q + lane] = transpose32(mask_word(q, m0, m1), lane);
   __syncthreads();
@@ -245,7 +249,7 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
     if (writer) write_offsets(c_e, chunk_off, chunk_pairs);  // block-uniform condition
   }
   if (tid < N) {
-    int acc = SINGLE ? chunk_off : exp_off[tid] + base[static_cast<int64_t>(tid) * nblk + blockIdx.x];
+    int acc = SINGLE ? chunk_off : exp_off[tid] + chunk_base;
     int lacc = chunk_off;
 #pragma unroll
     for (int w = 0; w < kWarps; ++w) {
