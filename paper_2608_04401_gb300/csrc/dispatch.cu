@@ -2,7 +2,7 @@
 // plus the row gather and the gate-weighted combine.
 //
 // Dispatch is a deterministic counting sort over chunks of 128 tokens:
-//   count   : per chunk, per-expert pair counts (bit-transposed warp masks), stored
+//   count   : per chunk, per-expert pair counts (shared-memory increments), stored
 //             expert-major: cnt[e][chunk]. The elbow router can write these
 //             itself, in which case this pass is skipped.
 //   scan    : one block per expert: exclusive prefix over the chunks, in
@@ -78,24 +78,32 @@ template <int N>
 __global__ void __launch_bounds__(kChunk) count_kernel(const int32_t* __restrict__ k,
                                                        const int32_t* __restrict__ ids, int64_t T,
                                                        int K, int nblk, int32_t* __restrict__ cnt) {
-  __shared__ int wcnt[kWarps][N];
+  // one shared-memory increment per selected pair (ids outside [0, N) are
+  // not counted: they cannot come from the router)
+  __shared__ int hist[N];
   grid_dep_wait();
   grid_dep_launch();
-  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  for (int e = threadIdx.x; e < N; e += kChunk) hist[e] = 0;
   const int64_t t = static_cast<int64_t>(blockIdx.x) * kChunk + threadIdx.x;
-  int kt, my[8];
-  uint64_t m0, m1;
-  load_selection(k, ids, t, t < T, K, kt, my, m0, m1);
+  const bool valid = t < T;
+  const int kt = valid ? min(k[t], K) : 0;
+  int my[8];
+  if (valid && K == 8) {
+    const int4 a = reinterpret_cast<const int4*>(ids + t * 8)[0];
+    const int4 b = reinterpret_cast<const int4*>(ids + t * 8)[1];
+    my[0] = a.x; my[1] = a.y; my[2] = a.z; my[3] = a.w;
+    my[4] = b.x; my[5] = b.y; my[6] = b.z; my[7] = b.w;
+  } else {
 #pragma unroll
-  for (int q = 0; q < N / 32; ++q)
-    wcnt[warp][32 * q + lane] = __popc(transpose32(mask_word(q, m0, m1), lane));
-  __syncthreads();
-  for (int e = threadIdx.x; e < N; e += kChunk) {
-    int c = 0;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) c += wcnt[w][e];
-    cnt[static_cast<int64_t>(e) * nblk + blockIdx.x] = c;
+    for (int s = 0; s < 8; ++s) my[s] = (s < kt) ? ids[t * K + s] : 0;
   }
+  __syncthreads();
+#pragma unroll
+  for (int s = 0; s < 8; ++s)
+    if (s < kt && static_cast<unsigned>(my[s]) < static_cast<unsigned>(N)) atomicAdd(&hist[my[s]], 1);
+  __syncthreads();
+  for (int e = threadIdx.x; e < N; e += kChunk)
+    cnt[static_cast<int64_t>(e) * nblk + blockIdx.x] = hist[e];
 }
 
 // Block e: exclusive prefix sum of cnt[e][0 .. nblk) in place; total -> totals[e].
