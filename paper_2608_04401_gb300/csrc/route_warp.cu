@@ -10,7 +10,9 @@
 //   a bitonic sort of the N keys (p bits << 32 | ~id) across the warp (64-bit
 //   shuffles), which orders by p descending and ascending id on ties;
 //   p'_i, D_i on each rank, the first argmax by a (max D, min index) warp
-//   reduction, k = min(e + 1, K).
+//   reduction, k = min(e + 1, K). The steps from p on are warp_route_from_e
+//   (route_impl.cuh), which also routes the tokens that the thread-per-token
+//   kernels leave undecided.
 //
 // router_small_route_kernel: the router GEMM for T <= 64 tokens on CUDA cores,
 // split over d in slices of 64 columns and over tokens in groups of 16 (one
@@ -147,82 +149,9 @@ MOE_DEV void route_one_warp(const float* __restrict__ row, int64_t t, int K, flo
   }
   const float r = __frcp_rn(__shfl_sync(full, v0, 0));
 
-  // keys: p bits above, ~id below; element j = 32 c + lane
-  uint64_t key[C];
-#pragma unroll
-  for (int c = 0; c < C; ++c) {
-    const float p = __fmul_rn(e[c], r);
-    key[c] = (static_cast<uint64_t>(__float_as_uint(p)) << 32) |
-             static_cast<uint32_t>(~(32 * c + lane));
-  }
-  // bitonic sort, descending
-#pragma unroll
-  for (int k2 = 2; k2 <= N; k2 <<= 1) {
-#pragma unroll
-    for (int jj = k2 >> 1; jj > 0; jj >>= 1) {
-      uint64_t nk[C];
-#pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const int j = 32 * c + lane;
-        const uint64_t other =
-            jj >= 32 ? key[c ^ (jj / 32)] : __shfl_xor_sync(full, key[c], jj);
-        const bool lower = (j & jj) == 0;
-        const bool desc = (j & k2) == 0;
-        const uint64_t hi = key[c] > other ? key[c] : other;
-        const uint64_t lo = key[c] > other ? other : key[c];
-        nk[c] = (lower == desc) ? hi : lo;
-      }
-#pragma unroll
-      for (int c = 0; c < C; ++c) key[c] = nk[c];
-    }
-  }
-
-  // the elbow over all ranks (rank of element j is j)
-  const float pmax = __uint_as_float(static_cast<uint32_t>(__shfl_sync(full, key[0], 0) >> 32));
-  const float pmin =
-      __uint_as_float(static_cast<uint32_t>(__shfl_sync(full, key[C - 1], 31) >> 32));
-  const float inv = __frcp_rn(__fadd_rn(__fsub_rn(pmax, pmin), eps));
-  float best = 0.0f;
-  int bi = 0;
-#pragma unroll
-  for (int c = 0; c < C; ++c) {
-    const int i = 32 * c + lane;
-    const float p = __uint_as_float(static_cast<uint32_t>(key[c] >> 32));
-    const float pn = __fmul_rn(__fsub_rn(p, pmin), inv);
-    const float xi = __fdiv_rn(static_cast<float>(i), static_cast<float>(N - 1));
-    const float D = __fsub_rn(__fsub_rn(1.0f, pn), xi);
-    if (c == 0 || D > best) {
-      best = D;
-      bi = i;
-    }
-  }
-#pragma unroll
-  for (int o = 16; o >= 1; o >>= 1) {
-    const float ob = __shfl_xor_sync(full, best, o);
-    const int oi = __shfl_xor_sync(full, bi, o);
-    if (ob > best || (ob == best && oi < bi)) {
-      best = ob;
-      bi = oi;
-    }
-  }
-  const int k = topk_mode ? K : min(bi + 1, K);
-
-  // ranks 0 .. K-1 are slot 0 of lanes 0 .. K-1
-  const float p = __uint_as_float(static_cast<uint32_t>(key[0] >> 32));
-  const int id = static_cast<int>(~static_cast<uint32_t>(key[0]));
-  float S = 0.0f;
-  if (renorm) {
-#pragma unroll
-    for (int s = 0; s < 8; ++s) {
-      const float ps = __shfl_sync(full, p, s);
-      if (s < k) S = __fadd_rn(S, ps);
-    }
-  }
-  if (lane < K) {
-    ids_out[t * K + lane] = id;
-    gates_out[t * K + lane] = lane < k ? (renorm ? __fdiv_rn(p, S) : p) : 0.0f;
-  }
-  if (lane == 0) k_out[t] = k;
+  int sel_id;
+  route::warp_route_from_e<N>(e, r, t, K, eps, topk_mode, renorm, k_out, ids_out, gates_out,
+                              sel_id);
 }
 
 template <int N>
