@@ -176,6 +176,19 @@ def elbow_route_warp(logits, K: int = 8, eps: float = 1e-8, mode: int = MODE_ELB
     return k, ids, gates
 
 
+def _check_chunk_counts(cc, T, N):
+    """The per-chunk counts a router writes: int32 [N, ceil(T/128)], contiguous."""
+    torch = _torch()
+    _cuda(cc, torch.int32, "chunk_counts")
+    if tuple(cc.shape) != (N, _num_chunks(T)):
+        raise ValueError(f"chunk_counts must be a contiguous [{N}, {_num_chunks(T)}] int32 tensor")
+
+
+def _num_chunks(T):
+    """128-token chunks of the dispatch counts."""
+    return (T + 127) // 128
+
+
 def elbow_route_with_counts(logits, chunk_counts, K: int = 8, eps: float = 1e-8,
                             mode: int = MODE_ELBOW, renorm: int = 0, stream=None):
     """elbow_route that also writes the per-chunk expert counts (an int32 tensor of
@@ -187,6 +200,7 @@ def elbow_route_with_counts(logits, chunk_counts, K: int = 8, eps: float = 1e-8,
     k = torch.empty(T, dtype=torch.int32, device=logits.device)
     ids = torch.empty(T, K, dtype=torch.int32, device=logits.device)
     gates = torch.empty(T, K, dtype=torch.float32, device=logits.device)
+    _check_chunk_counts(chunk_counts, T, N)
     _check(lib.elbow_route_with_counts(_p(logits), T, N, _params(K, eps, mode, renorm), _p(k),
                                        _p(ids), _p(gates), _p(chunk_counts), _stream(stream)),
            "elbow_route_with_counts")
@@ -277,11 +291,12 @@ def moe_dispatch(k, ids, N: int, ws=None, stream=None):
 
 
 def dispatch_chunk_counts(ws, T: int, N: int, K: int):
-    """View of the [N, ceil(T/128)] per-chunk expert counts inside a dispatch workspace."""
+    """View of the [N, ceil(T/128)] per-chunk expert counts inside a dispatch workspace
+    (chunk c = tokens 128 c .. 128 c + 127)."""
     torch = _torch()
     ptr = library().moe_dispatch_chunk_counts(_p(ws), T, N, K)
     off = ptr - ws.data_ptr()
-    nblk = (T + 127) // 128
+    nblk = _num_chunks(T)
     return ws[off: off + 4 * N * nblk].view(torch.int32).view(N, nblk)
 
 
@@ -402,7 +417,9 @@ def router_route(x, w_router, K: int = 8, eps: float = 1e-8, mode: int = MODE_EL
     lg = torch.empty(T, N, dtype=torch.float32, device=dev) if with_logits else None
     cc = chunk_counts
     if cc is None and with_counts:
-        cc = torch.zeros(N, (T + 127) // 128, dtype=torch.int32, device=dev)
+        cc = torch.zeros(N, _num_chunks(T), dtype=torch.int32, device=dev)
+    if cc is not None:
+        _check_chunk_counts(cc, T, N)
     _check(library().moe_router_route(_p(x), _p(w_router), T, d, N, _params(K, eps, mode, renorm),
                                       _p(lg), _p(k), _p(ids), _p(gates), _p(cc), _p(err),
                                       _stream(stream)), "moe_router_route")

@@ -82,6 +82,12 @@ def test_dispatch_counted_matches_dispatch(moe, T, N):
     ws = torch.empty(moe.dispatch_workspace_size(T, N, 8), dtype=torch.uint8, device="cuda")
     cc = moe.dispatch_chunk_counts(ws, T, N, 8)
     k, ids, gates, _, _ = moe.router_route(x, wr, with_logits=False, chunk_counts=cc)
+    # counts [N][ceil(T/128)]: the pairs of expert e among tokens 128 c .. 128 c + 127
+    kh, idh = k.cpu().numpy(), ids.cpu().numpy()
+    sel = np.arange(8)[None, :] < kh[:, None]
+    want = np.zeros((N, (T + 127) // 128), np.int64)
+    np.add.at(want, (idh[sel], np.repeat(np.arange(T) // 128, kh)), 1)
+    assert np.array_equal(cc.cpu().numpy(), want)
     off_a, perm_a, pp_a = moe.moe_dispatch_counted(k, ids, N, ws)
     off_b, perm_b, pp_b, _ = moe.moe_dispatch(k, ids, N)
     torch.cuda.synchronize()

@@ -140,6 +140,41 @@ def _dispatch_both(moe, k, ids, N):
     return ref
 
 
+@pytest.mark.parametrize("N,T,kind", [(64, 700, "routed"), (128, 2049, "routed"),
+                                        (64, 2049, "same"), (128, 1700, "same")])
+def test_dispatch_ignores_stale_workspace(moe, N, T, kind):
+    """Every part of the dispatch workspace is written before it is read: a
+    workspace full of 0xff bytes gives the same dispatch, with and without the
+    router's counts. kind "same": every token selects experts 0..7 (128 pairs
+    of each of them per chunk, 0 of every other expert)."""
+    import torch
+    rng = np.random.default_rng(T + 7 * N)
+    lg = synth.boosted_logits(rng, T, N)
+    if kind == "same":
+        k = np.full(T, 8, np.int32)
+        ids = np.tile(np.arange(8, dtype=np.int32), (T, 1))
+    else:
+        r = oracle.route(lg, K=8)
+        k, ids = r["k"], r["ids"]
+    ref = oracle.dispatch(k, ids, N)
+    P = int(ref["offsets"][-1])
+    ws = torch.full((moe.dispatch_workspace_size(T, N, 8),), 255, dtype=torch.uint8, device="cuda")
+    off, perm, pp, _ = moe.moe_dispatch(to_dev(k), to_dev(ids), N, ws=ws)
+    torch.cuda.synchronize()
+    assert np.array_equal(off.cpu().numpy(), ref["offsets"])
+    assert np.array_equal(perm.cpu().numpy()[:P], ref["perm"])
+    assert np.array_equal(pp.cpu().numpy(), ref["pair_pos"])
+    if kind == "routed":
+        ws.fill_(255)
+        cc = moe.dispatch_chunk_counts(ws, T, N, 8)
+        k2, ids2, _ = moe.elbow_route_with_counts(to_dev(lg), cc)
+        off2, perm2, pp2 = moe.moe_dispatch_counted(k2, ids2, N, ws)
+        torch.cuda.synchronize()
+        assert np.array_equal(off2.cpu().numpy(), ref["offsets"])
+        assert np.array_equal(perm2.cpu().numpy()[:P], ref["perm"])
+        assert np.array_equal(pp2.cpu().numpy(), ref["pair_pos"])
+
+
 @pytest.mark.parametrize("N", [64, 128])
 @pytest.mark.parametrize("T", [1, 33, 2047, 2048, 2049, 20000])
 def test_dispatch_bitexact(moe, N, T):
@@ -184,9 +219,15 @@ def test_route_with_counts_then_counted_dispatch(moe, N, T):
     ws = torch.empty(moe.dispatch_workspace_size(T, N, 8), dtype=torch.uint8, device="cuda")
     cc = moe.dispatch_chunk_counts(ws, T, N, 8)
     k, ids, gates = moe.elbow_route_with_counts(to_dev(lg), cc)
-    off, perm, pp = moe.moe_dispatch_counted(k, ids, N, ws)
     torch.cuda.synchronize()
     ref = oracle.route(lg, K=8)
+    # counts [N][ceil(T/128)]: the pairs of expert e among tokens 128 c .. 128 c + 127
+    sel = np.arange(8)[None, :] < ref["k"][:, None]
+    want = np.zeros((N, (T + 127) // 128), np.int64)
+    np.add.at(want, (ref["ids"][sel], np.repeat(np.arange(T) // 128, ref["k"])), 1)
+    assert np.array_equal(cc.cpu().numpy(), want)
+    off, perm, pp = moe.moe_dispatch_counted(k, ids, N, ws)
+    torch.cuda.synchronize()
     _assert_route_equal((k.cpu().numpy(), ids.cpu().numpy(), gates.cpu().numpy()), ref)
     d = oracle.dispatch(ref["k"], ref["ids"], N)
     assert np.array_equal(off.cpu().numpy(), d["offsets"])
