@@ -713,11 +713,15 @@ def cpu_baseline(inp, K, budget_s=12.0):
     """The CPU oracle, as it stands, on a bounded sample of the same workload."""
     import oracle
     T = inp["x"].shape[0]
-    rows = np.arange(8, dtype=np.int64)
+    # calibrate the per-token cost on 128 tokens after an 8-token warm-up (the
+    # first call also pays for starting the threads)
+    oracle.layer_rows(inp["x"], inp["w_router"], inp["w_gate_up"], inp["w_down"],
+                      rows=np.arange(8, dtype=np.int64), K=K)
+    rows = np.arange(128, dtype=np.int64)
     t0 = time.perf_counter()
     oracle.layer_rows(inp["x"], inp["w_router"], inp["w_gate_up"], inp["w_down"], rows=rows, K=K)
     dt = time.perf_counter() - t0
-    n = int(min(T, max(8, 8 * budget_s / max(dt, 1e-3))))
+    n = int(min(T, max(128, 128 * budget_s / max(dt, 1e-3))))
     rows = np.linspace(0, T - 1, n).astype(np.int64)
     t0 = time.perf_counter()
     oracle.layer_rows(inp["x"], inp["w_router"], inp["w_gate_up"], inp["w_down"], rows=rows, K=K)
@@ -745,12 +749,13 @@ def run_reference(args, rank, world):
         oracle.layer_rows(inp["x"], inp["w_router"], inp["w_gate_up"], inp["w_down"], rows=rows,
                           K=K)
 
-    for _ in range(max(1, min(args.warmup, 3))):
+    # W untimed warm-up steps, then exactly K timed steps (about 20 ms each)
+    for _ in range(args.warmup):
         step()
+    n = max(1, args.steps)
     t0 = time.perf_counter()
-    for _ in range(args.steps if args.steps <= 50 else 50):
+    for _ in range(n):
         step()
-    n = args.steps if args.steps <= 50 else 50
     dt = (time.perf_counter() - t0) / n
     val = sample / dt
     cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
