@@ -3,9 +3,10 @@
  *
  * The method is "Elbow-based MoE Routing" (arxiv 2608.04401): per token, the
  * router's softmax probabilities are sorted in descending order, a
- * Kneedle-style elbow e is found on the curve normalised to [0,1] (Alg. 1),
- * and only k = min(e, K) experts are used instead of a fixed top-K
- * (Sec. 2.1). This library runs that MoE layer forward on one GPU.
+ * Kneedle-style elbow index e (0-based) is found on the curve normalised to
+ * [0,1] (Alg. 1, which returns e + 1), and only k = min(e + 1, K) experts are
+ * used instead of a fixed top-K (Sec. 2.1). This library runs that MoE layer
+ * forward on one GPU.
  *
  * Conventions for every entry point:
  *   - All tensor pointers are DEVICE pointers owned by the caller; the library
@@ -18,7 +19,9 @@
  *   - Every call returns a moe_status and never aborts the process. Argument
  *     errors are detected on the host before anything is enqueued.
  *   - Supported shapes: N (experts) in {64, 128}; 1 <= K <= 8 and K <= N;
- *     T >= 0 tokens (T = 0 is a no-op); for the layer, d_model a multiple of
+ *     0 <= T < 2^28 tokens (T = 0 is a no-op; larger T returns
+ *     MOE_ERR_INVALID_ARG, so that the T * K pair counts fit in int32); for
+ *     the layer, d_model a multiple of
  *     256 and the SwiGLU intermediate I a multiple of 128, d, I <= 16384.
  *   - Pointers must be 16-byte aligned.
  *
@@ -125,6 +128,8 @@ moe_status elbow_route_with_counts(const float* logits, int64_t T, int N,
  * Ids outside [0, N) are not checked on the device: they are undefined
  * behaviour (elbow_route never produces them).
  */
+/* Bytes of moe_dispatch's workspace; 0 for unsupported sizes (T outside
+ * [0, 2^28), N not 64 or 128). */
 size_t moe_dispatch_workspace_size(int64_t T, int N, int K);
 moe_status moe_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
                         int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
@@ -177,6 +182,8 @@ moe_status moe_dispatch_noalloc(const int32_t* k, const int32_t* ids, int64_t T,
  *              256-byte aligned; it also holds the device error word read by
  *              moe_read_device_error.
  * TOPK mode runs the same kernels with k = K.
+ * moe_layer_workspace_size returns 0 for unsupported sizes (T outside
+ * [0, 2^28), N not 64 or 128, K outside [1, 8], d or I outside [1, 16384]).
  */
 size_t moe_layer_workspace_size(int64_t T, int d, int N, int I, int K);
 moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const uint16_t* w_gate_up,

@@ -78,7 +78,8 @@ __global__ void bounded_wait_check_kernel(int32_t* err, uint64_t limit_ns) {
     atomicExch(err, moe::kDevErrTimeout);
 }
 
-constexpr int64_t kMaxTokens = int64_t(1) << 28;  // keeps T * K * 8 row counts in int32
+// T < 2^28 keeps the pair counts and positions (up to T * K <= 2^31 - 8) in int32
+constexpr int64_t kMaxTokens = (int64_t(1) << 28) - 1;
 constexpr int kMaxDim = 16384;
 // Batches of at most this many tokens take the decode-shaped expert GEMMs
 // (weights as the M operand; every expert then has at most 64 rows).
@@ -96,6 +97,9 @@ constexpr int64_t kSmallRouterMaxTokens = 64;
 constexpr int kSmallRouterSlice = 64;
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+// 4-byte alignment of int32 / fp32 arrays (a null pointer passes: optional
+// arguments are checked for null separately)
+bool aligned4(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; }
 
 size_t up256(size_t b) { return (b + 255) & ~static_cast<size_t>(255); }
 
@@ -279,7 +283,7 @@ moe_status elbow_route_with_counts(const float* logits, int64_t T, int N,
 
 size_t moe_dispatch_workspace_size(int64_t T, int N, int K) {
   (void)K;
-  if (T < 0 || !supported_n(N)) return 0;
+  if (T < 0 || T > kMaxTokens || !supported_n(N)) return 0;
   return moe::dispatch_ws_bytes(T, N);
 }
 
@@ -306,6 +310,8 @@ moe_status moe_dispatch_counted(const int32_t* k, const int32_t* ids, int64_t T,
   if (ws_bytes < moe::dispatch_ws_bytes(T, N)) return MOE_ERR_WORKSPACE;
   if ((reinterpret_cast<uintptr_t>(ws) & 255u)) return MOE_ERR_INVALID_ARG;
   if (T > 0 && !aligned16(ids)) return MOE_ERR_INVALID_ARG;
+  if (!aligned4(k) || !aligned4(offsets) || !aligned4(perm) || !aligned4(pair_pos))
+    return MOE_ERR_INVALID_ARG;
   return cuda_status(moe::launch_dispatch(k, ids, T, N, K, offsets, perm, pair_pos, ws, nullptr,
                                           true, static_cast<cudaStream_t>(stream)));
 }
@@ -320,12 +326,16 @@ moe_status moe_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, 
   if (ws_bytes < moe::dispatch_ws_bytes(T, N)) return MOE_ERR_WORKSPACE;
   if ((reinterpret_cast<uintptr_t>(ws) & 255u)) return MOE_ERR_INVALID_ARG;
   if (T > 0 && !aligned16(ids)) return MOE_ERR_INVALID_ARG;
+  if (!aligned4(k) || !aligned4(offsets) || !aligned4(perm) || !aligned4(pair_pos))
+    return MOE_ERR_INVALID_ARG;
   return cuda_status(moe::launch_dispatch(k, ids, T, N, K, offsets, perm, pair_pos, ws, nullptr,
                                           false, static_cast<cudaStream_t>(stream)));
 }
 
 size_t moe_layer_workspace_size(int64_t T, int d, int N, int I, int K) {
-  if (T < 0 || d <= 0 || I <= 0 || K < 1 || !supported_n(N)) return 0;
+  if (T < 0 || T > kMaxTokens || d <= 0 || d > kMaxDim || I <= 0 || I > kMaxDim || K < 1 ||
+      K > 8 || !supported_n(N))
+    return 0;
   return layer_ws(nullptr, T, d, N, I, K).bytes;
 }
 
@@ -346,19 +356,19 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   LayerWs w = layer_ws(ws, T, d, N, I, K);
   if (ws_bytes < w.bytes) return MOE_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (T > 0) {  // every argument is checked before anything is enqueued
+    const void* need[] = {x, w_router, w_gate_up, w_down, y};
+    for (const void* p : need)
+      if (!p || !aligned16(p)) return MOE_ERR_INVALID_ARG;
+    if (residual && !aligned16(residual)) return MOE_ERR_INVALID_ARG;
+    if ((logits_out && !aligned16(logits_out)) || (ids_out && !aligned16(ids_out)) ||
+        (gates_out && !aligned16(gates_out)) || !aligned4(k_out) || !aligned4(offsets_out))
+      return MOE_ERR_INVALID_ARG;
+  }
   // clear the device error word (and the small-batch router's four group
-  // tickets beside it) first, so that a no-op call reads clean
+  // tickets beside it), so that a no-op call reads clean
   if (cudaMemsetAsync(w.err, 0, 8 * sizeof(int32_t), s) != cudaSuccess) return MOE_ERR_CUDA;
   if (T == 0) return MOE_OK;
-  const void* need[] = {x, w_router, w_gate_up, w_down, y};
-  for (const void* p : need)
-    if (!p || !aligned16(p)) return MOE_ERR_INVALID_ARG;
-  if (residual && !aligned16(residual)) return MOE_ERR_INVALID_ARG;
-  if ((logits_out && !aligned16(logits_out)) || (ids_out && !aligned16(ids_out)) ||
-      (gates_out && !aligned16(gates_out)) ||
-      (k_out && (reinterpret_cast<uintptr_t>(k_out) & 3u)) ||
-      (offsets_out && (reinterpret_cast<uintptr_t>(offsets_out) & 3u)))
-    return MOE_ERR_INVALID_ARG;
 
   int32_t* kk = k_out ? k_out : w.k;
   int32_t* ids = ids_out ? ids_out : w.ids;
@@ -435,7 +445,8 @@ moe_status moe_router_logits(const uint16_t* x, const uint16_t* w_router, int64_
   if (T < 0 || T > kMaxTokens) return MOE_ERR_INVALID_ARG;
   if (!supported_n(N) || d <= 0 || d > kMaxDim || d % 64 != 0) return MOE_ERR_UNSUPPORTED;
   if (T == 0) return MOE_OK;
-  if (!x || !w_router || !logits || !aligned16(x) || !aligned16(w_router) || !aligned16(logits))
+  if (!x || !w_router || !logits || !aligned16(x) || !aligned16(w_router) || !aligned16(logits) ||
+      !aligned4(err_word))
     return MOE_ERR_INVALID_ARG;
   const int nsm = sm_count();
   if (nsm <= 0) return MOE_ERR_CUDA;
@@ -452,7 +463,7 @@ moe_status moe_expert_gate_up(const uint16_t* xs, const uint16_t* w_gate_up, con
     return MOE_ERR_UNSUPPORTED;
   if (P == 0) return MOE_OK;
   if (!xs || !w_gate_up || !offsets || !tile_off || !h || !aligned16(xs) || !aligned16(w_gate_up) ||
-      !aligned16(h))
+      !aligned16(h) || !aligned4(offsets) || !aligned4(tile_off) || !aligned4(err_word))
     return MOE_ERR_INVALID_ARG;
   const int nsm = sm_count();
   if (nsm <= 0) return MOE_ERR_CUDA;
@@ -469,7 +480,7 @@ moe_status moe_expert_down(const uint16_t* h, const uint16_t* w_down, const int3
     return MOE_ERR_UNSUPPORTED;
   if (P == 0) return MOE_OK;
   if (!h || !w_down || !offsets || !tile_off || !o || !aligned16(h) || !aligned16(w_down) ||
-      !aligned16(o))
+      !aligned16(o) || !aligned4(offsets) || !aligned4(tile_off) || !aligned4(err_word))
     return MOE_ERR_INVALID_ARG;
   const int nsm = sm_count();
   if (nsm <= 0) return MOE_ERR_CUDA;
@@ -487,7 +498,7 @@ moe_status moe_expert_gate_up_decode(const uint16_t* xs, const uint16_t* w_gate_
     return MOE_ERR_UNSUPPORTED;
   if (P == 0 || T == 0) return MOE_OK;
   if (!xs || !w_gate_up || !offsets || !h || !aligned16(xs) || !aligned16(w_gate_up) ||
-      !aligned16(h))
+      !aligned16(h) || !aligned4(offsets) || !aligned4(err_word))
     return MOE_ERR_INVALID_ARG;
   const int nsm = sm_count();
   if (nsm <= 0) return MOE_ERR_CUDA;
@@ -505,7 +516,8 @@ moe_status moe_expert_down_decode(const uint16_t* h, const uint16_t* w_down, con
       I % 64 != 0)
     return MOE_ERR_UNSUPPORTED;
   if (P == 0 || T == 0) return MOE_OK;
-  if (!h || !w_down || !offsets || !o || !aligned16(h) || !aligned16(w_down) || !aligned16(o))
+  if (!h || !w_down || !offsets || !o || !aligned16(h) || !aligned16(w_down) || !aligned16(o) ||
+      !aligned4(offsets) || !aligned4(err_word))
     return MOE_ERR_INVALID_ARG;
   const int nsm = sm_count();
   if (nsm <= 0) return MOE_ERR_CUDA;
@@ -515,11 +527,14 @@ moe_status moe_expert_down_decode(const uint16_t* h, const uint16_t* w_down, con
 
 moe_status moe_gather_rows(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int64_t T,
                            int64_t P, int d, int N, uint16_t* xs, void* stream) {
-  (void)T;
-  if (P < 0 || d <= 0 || d % 8 != 0) return MOE_ERR_INVALID_ARG;
+  if (T < 0 || T > kMaxTokens || P < 0 || P > kMaxTokens * 8 || d <= 0 || d > kMaxDim ||
+      d % 8 != 0)
+    return MOE_ERR_INVALID_ARG;
   if (!supported_n(N)) return MOE_ERR_UNSUPPORTED;
   if (P == 0) return MOE_OK;
-  if (!x || !perm || !offsets || !xs || !aligned16(x) || !aligned16(xs)) return MOE_ERR_INVALID_ARG;
+  if (!x || !perm || !offsets || !xs || !aligned16(x) || !aligned16(xs) || !aligned4(perm) ||
+      !aligned4(offsets))
+    return MOE_ERR_INVALID_ARG;
   const int nsm = sm_count();
   if (nsm <= 0) return MOE_ERR_CUDA;
   return cuda_status(moe::launch_gather(x, perm, offsets, N, P, d, xs, nsm,
@@ -537,7 +552,7 @@ moe_status moe_router_route(const uint16_t* x, const uint16_t* w_router, int64_t
   if (T == 0) return MOE_OK;
   if (!x || !w_router || !k_out || !ids_out || !gates_out || !aligned16(x) || !aligned16(w_router) ||
       !aligned16(ids_out) || !aligned16(gates_out) || (logits_out && !aligned16(logits_out)) ||
-      (reinterpret_cast<uintptr_t>(k_out) & 3u))
+      !aligned4(k_out) || !aligned4(chunk_counts) || !aligned4(err_word))
     return MOE_ERR_INVALID_ARG;
   const int nsm = sm_count();
   if (nsm <= 0) return MOE_ERR_CUDA;
@@ -557,7 +572,8 @@ moe_status moe_expert_gate_up_gathered(const uint16_t* x, int64_t T, const int32
     return MOE_ERR_UNSUPPORTED;
   if (P == 0 || T == 0) return MOE_OK;
   if (!x || !perm || !w_gate_up || !offsets || !tile_off || !h || !aligned16(x) ||
-      !aligned16(w_gate_up) || !aligned16(h))
+      !aligned16(w_gate_up) || !aligned16(h) || !aligned4(perm) || !aligned4(offsets) ||
+      !aligned4(tile_off) || !aligned4(err_word))
     return MOE_ERR_INVALID_ARG;
   const int nsm = sm_count();
   if (nsm <= 0) return MOE_ERR_CUDA;
@@ -569,10 +585,11 @@ moe_status moe_expert_gate_up_gathered(const uint16_t* x, int64_t T, const int32
 moe_status moe_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_pos,
                        const float* gates, const uint16_t* residual, int64_t T, int d, int K,
                        uint16_t* y, void* stream) {
-  if (T < 0 || d <= 0 || d % 8 != 0 || K < 1 || K > 8) return MOE_ERR_INVALID_ARG;
+  if (T < 0 || T > kMaxTokens || d <= 0 || d > kMaxDim || d % 8 != 0 || K < 1 || K > 8)
+    return MOE_ERR_INVALID_ARG;
   if (T == 0) return MOE_OK;
   if (!o || !k || !pair_pos || !gates || !y || !aligned16(o) || !aligned16(y) ||
-      (residual && !aligned16(residual)))
+      (residual && !aligned16(residual)) || !aligned4(k) || !aligned4(pair_pos) || !aligned4(gates))
     return MOE_ERR_INVALID_ARG;
   const int nsm = sm_count();
   if (nsm <= 0) return MOE_ERR_CUDA;

@@ -682,6 +682,9 @@ extern "C" moe_status moe_dispatch_noalloc(const int32_t* k, const int32_t* ids,
   if (!offsets) return MOE_ERR_INVALID_ARG;
   if (T > 0 && (!k || !ids || !perm || !pair_pos)) return MOE_ERR_INVALID_ARG;
   if (T > 0 && (reinterpret_cast<uintptr_t>(ids) & 15u)) return MOE_ERR_INVALID_ARG;
+  for (const void* p : {static_cast<const void*>(k), static_cast<const void*>(offsets),
+                        static_cast<const void*>(perm), static_cast<const void*>(pair_pos)})
+    if (reinterpret_cast<uintptr_t>(p) & 3u) return MOE_ERR_INVALID_ARG;
   int32_t* scratch = nullptr;
   if (noalloc_scratch(&scratch) != cudaSuccess) return MOE_ERR_CUDA;
   // Layout: per-chunk counts [N][chunks] | totals [N] | tile offsets [N+1]. The

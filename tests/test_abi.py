@@ -60,6 +60,8 @@ def test_route_validation(lib):
     assert lib.elbow_route(None, 10, 64, _rp(), fake, fake, fake, None) == 1
     assert lib.elbow_route(ctypes.c_void_p(258), 10, 64, _rp(), fake, fake, fake, None) == 1
     assert lib.elbow_route(fake, -1, 64, _rp(), fake, fake, fake, None) == 1
+    # T * K pair counts must fit in int32: T < 2^28
+    assert lib.elbow_route(fake, 1 << 28, 64, _rp(), fake, fake, fake, None) == 1
     assert lib.elbow_route(fake, 10, 64, None, fake, fake, fake, None) == 1
     # T = 0 is a no-op that launches nothing
     assert lib.elbow_route(None, 0, 64, _rp(), None, None, None, None) == 0
@@ -72,6 +74,9 @@ def test_dispatch_validation(lib):
     assert lib.moe_dispatch(fake, fake, 1000, 64, 8, fake, fake, fake, fake, need - 1, None) == 3
     assert lib.moe_dispatch(fake, fake, 1000, 96, 8, fake, fake, fake, fake, need, None) == 2
     assert lib.moe_dispatch(fake, fake, 1000, 64, 8, None, fake, fake, fake, need, None) == 1
+    big = lib.moe_dispatch_workspace_size((1 << 28) - 1, 64, 8)
+    assert big > 0 and lib.moe_dispatch_workspace_size(1 << 28, 64, 8) == 0
+    assert lib.moe_dispatch(fake, fake, 1 << 28, 64, 8, fake, fake, fake, fake, big, None) == 1
 
 
 def test_layer_validation(lib):
@@ -88,6 +93,8 @@ def test_layer_validation(lib):
     assert lib.moe_layer_forward(*args(wsb=ws - 1)) == 3
     assert lib.moe_layer_forward(*args(rp=_rp(renorm=2))) == 1
     assert lib.moe_layer_workspace_size(64, 2048, 63, 1024, 8) == 0
+    assert lib.moe_layer_workspace_size(1 << 28, 2048, 64, 1024, 8) == 0
+    assert lib.moe_layer_workspace_size(64, 2048, 64, 1024, 9) == 0
 
 
 def test_diagnostics_validation(lib):
@@ -114,3 +121,24 @@ def test_bounded_wait_check_validation(lib):
     assert lib.moe_check_bounded_wait(ctypes.c_void_p(256), 0.0, None) == 1
     assert lib.moe_check_bounded_wait(ctypes.c_void_p(256), 11.0, None) == 1
 
+
+
+def test_misaligned_int32_arrays_are_rejected(lib):
+    """4-byte arrays (counts, offsets, positions, gates, error words) that are
+    not 4-byte aligned return MOE_ERR_INVALID_ARG before anything is enqueued."""
+    fake = ctypes.c_void_p(256)
+    odd = ctypes.c_void_p(258)
+    need = lib.moe_dispatch_workspace_size(1000, 64, 8)
+    assert lib.moe_dispatch(odd, fake, 1000, 64, 8, fake, fake, fake, fake, need, None) == 1
+    assert lib.moe_dispatch(fake, fake, 1000, 64, 8, fake, odd, fake, fake, need, None) == 1
+    assert lib.moe_dispatch(fake, fake, 1000, 64, 8, fake, fake, odd, fake, need, None) == 1
+    assert lib.moe_dispatch(fake, fake, 1000, 64, 8, odd, fake, fake, fake, need, None) == 1
+    assert lib.moe_combine(fake, fake, fake, odd, None, 10, 2048, 8, fake, None) == 1
+    assert lib.moe_combine(fake, fake, odd, fake, None, 10, 2048, 8, fake, None) == 1
+    assert lib.moe_combine(fake, fake, fake, fake, None, 1 << 28, 2048, 8, fake, None) == 1
+    assert lib.moe_expert_down(fake, fake, odd, fake, 100, 2048, 64, 1024, fake, None, None) == 1
+    assert lib.moe_expert_down(fake, fake, fake, fake, 100, 2048, 64, 1024, fake, odd, None) == 1
+    assert lib.moe_gather_rows(fake, odd, fake, 10, 80, 2048, 64, fake, None) == 1
+    ws = lib.moe_layer_workspace_size(64, 2048, 64, 1024, 8)
+    assert lib.moe_layer_forward(fake, fake, fake, fake, 64, 2048, 64, 1024, _rp(), None, fake,
+                                 None, odd, None, None, None, fake, ws, None) == 1
