@@ -125,8 +125,10 @@ moe_status elbow_route_with_counts(const float* logits, int64_t T, int N,
  *                            (stable); entries from offsets[N] on are untouched
  *   pair_pos [T, K]   int32  position in perm of pair (t, s), -1 for s >= k_t
  *   ws       device workspace of at least moe_dispatch_workspace_size bytes
- * Ids outside [0, N) are not checked on the device: they are undefined
- * behaviour (elbow_route never produces them).
+ * A pair whose id lies outside [0, N) is dropped: it is not counted, not in
+ * perm, and its pair_pos is -1 (elbow_route never produces such ids). Ids
+ * repeated within a token give unspecified positions, but no access outside
+ * the arrays above.
  */
 /* Bytes of moe_dispatch's workspace; 0 for unsupported sizes (T outside
  * [0, 2^28), N not 64 or 128). */

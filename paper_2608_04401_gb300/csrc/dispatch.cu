@@ -23,7 +23,9 @@ constexpr int kChunk = 128;  // tokens per chunk = threads per block
 constexpr int kWarps = kChunk / 32;
 constexpr int kScanThreads = 1024;
 
-// Expert-membership bit masks of one token's selection (experts 0..63, 64..127).
+// Expert-membership bit masks of one token's selection (experts 0..63,
+// 64..127); ids outside [0, N) set no bit (their pairs are dropped).
+template <int N>
 MOE_DEV void load_selection(const int32_t* __restrict__ k, const int32_t* __restrict__ ids,
                             int64_t t, bool valid, int K, int& kt, int (&my)[8], uint64_t& m0,
                             uint64_t& m1) {
@@ -41,7 +43,7 @@ MOE_DEV void load_selection(const int32_t* __restrict__ k, const int32_t* __rest
   m1 = 0;
 #pragma unroll
   for (int s = 0; s < 8; ++s) {
-    if (s < kt) {
+    if (s < kt && static_cast<unsigned>(my[s]) < static_cast<unsigned>(N)) {
       if (my[s] < 64) m0 |= 1ull << my[s];
       else m1 |= 1ull << (my[s] - 64);
     }
@@ -231,7 +233,7 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
   const bool valid = t < T;
   int kt, my[8];
   uint64_t m0, m1;
-  load_selection(k, ids, t, valid, K, kt, my, m0, m1);
+  load_selection<N>(k, ids, t, valid, K, kt, my, m0, m1);
   int chunk_base = 0;
   if constexpr (!SINGLE) {
     if (tid < N) chunk_base = base[static_cast<int64_t>(tid) * nblk + blockIdx.x];
@@ -274,7 +276,7 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
 #pragma unroll
     for (int s = 0; s < 8; ++s) {
       if (s < K) {
-        if (s < kt) {
+        if (s < kt && static_cast<unsigned>(my[s]) < static_cast<unsigned>(N)) {
           const int e = my[s];
           const int below = __popc(bal[warp][e] & lt_mask);
           const int pos = wbase[warp][e] + below;

@@ -175,6 +175,31 @@ def test_dispatch_ignores_stale_workspace(moe, N, T, kind):
         assert np.array_equal(pp2.cpu().numpy(), ref["pair_pos"])
 
 
+@pytest.mark.parametrize("N,T", [(64, 100), (128, 100), (64, 3000), (128, 3000)])
+def test_dispatch_drops_out_of_range_ids(moe, N, T):
+    """Pairs whose id lies outside [0, N) are dropped (not counted, not in perm,
+    pair_pos -1); the other pairs keep the stable expert-major order."""
+    import torch
+    rng = np.random.default_rng(T + N + 11)
+    r = oracle.route(synth.boosted_logits(rng, T, N), K=8)
+    k, ids = r["k"], r["ids"].copy()
+    sel = np.arange(8)[None, :] < k[:, None]
+    bad = sel & (rng.random(ids.shape) < 0.05)
+    ids[bad] = rng.choice(np.array([-1, -7, N, N + 3, 1 << 20], np.int32), bad.sum())
+    off, perm, pp, _ = moe.moe_dispatch(to_dev(k), to_dev(ids), N)
+    torch.cuda.synchronize()
+    good = sel & ~bad
+    t_idx, s_idx = np.nonzero(good)
+    e_idx = ids[t_idx, s_idx]
+    order = np.lexsort((t_idx, e_idx))  # by expert, then token
+    want_off = np.concatenate([[0], np.cumsum(np.bincount(e_idx, minlength=N))])
+    want_pp = np.full(ids.shape, -1, np.int64)
+    want_pp[t_idx[order], s_idx[order]] = np.arange(len(order))
+    assert np.array_equal(off.cpu().numpy(), want_off)
+    assert np.array_equal(perm.cpu().numpy()[:len(order)], t_idx[order])
+    assert np.array_equal(pp.cpu().numpy(), want_pp)
+
+
 @pytest.mark.parametrize("N", [64, 128])
 @pytest.mark.parametrize("T", [1, 33, 2047, 2048, 2049, 20000])
 def test_dispatch_bitexact(moe, N, T):
