@@ -279,7 +279,9 @@ moe_status moe_dispatch_counted(const int32_t* k, const int32_t* ids, int64_t T,
                                 size_t ws_bytes, void* stream);
 
 /* Gather rows: xs[r] = x[perm[r]] for r < offsets[N] (x [T, d] bf16,
- * xs [P, d] bf16, P >= offsets[N]). */
+ * xs [P, d] bf16, P >= offsets[N]). Rows stop at P and tokens outside [0, T)
+ * are clamped into it, so inconsistent arguments cannot reach outside x or
+ * xs. */
 moe_status moe_gather_rows(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int64_t T,
                            int64_t P, int d, int N, uint16_t* xs, void* stream);
 

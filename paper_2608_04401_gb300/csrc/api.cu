@@ -20,8 +20,8 @@ cudaError_t launch_dispatch_gather(const int32_t* k, const int32_t* ids, int64_t
                                    int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
                                    int32_t* offsets_copy, const uint16_t* x, int d, uint16_t* xs,
                                    int num_sms, cudaStream_t stream);
-cudaError_t launch_gather(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int N,
-                          int64_t P, int d, uint16_t* xs, int num_sms, cudaStream_t stream);
+cudaError_t launch_gather(const uint16_t* x, int64_t T, const int32_t* perm, const int32_t* offsets,
+                          int N, int64_t P, int d, uint16_t* xs, int num_sms, cudaStream_t stream);
 cudaError_t launch_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_pos,
                            const float* gates, const uint16_t* residual, int64_t T, int d, int K,
                            uint16_t* y, int num_sms, cudaStream_t stream);
@@ -537,7 +537,7 @@ moe_status moe_gather_rows(const uint16_t* x, const int32_t* perm, const int32_t
     return MOE_ERR_INVALID_ARG;
   const int nsm = sm_count();
   if (nsm <= 0) return MOE_ERR_CUDA;
-  return cuda_status(moe::launch_gather(x, perm, offsets, N, P, d, xs, nsm,
+  return cuda_status(moe::launch_gather(x, T, perm, offsets, N, P, d, xs, nsm,
                                         static_cast<cudaStream_t>(stream)));
 }
 

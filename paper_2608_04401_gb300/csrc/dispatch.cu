@@ -311,15 +311,19 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
 }
 
 // xs[r] = x[perm[r]] for r < offsets[N]; one warp per row, 16-byte copies.
+// Rows stop at the capacity P and tokens are clamped to [0, T), so that
+// inconsistent arguments cannot reach outside x or xs.
 __global__ void __launch_bounds__(256) gather_kernel(const uint4* __restrict__ x,
                                                      const int32_t* __restrict__ perm,
                                                      const int32_t* __restrict__ offsets, int N,
-                                                     int d8, uint4* __restrict__ xs) {
-  const int total = offsets[N];
+                                                     int64_t T, int64_t P, int d8,
+                                                     uint4* __restrict__ xs) {
+  const int64_t total = min_of<int64_t>(offsets[N], P);
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
   for (int64_t r = static_cast<int64_t>(blockIdx.x) * 8 + warp; r < total;
        r += static_cast<int64_t>(gridDim.x) * 8) {
-    const int64_t t = perm[r];
+    const int64_t pt = perm[r];
+    const int64_t t = pt < 0 ? 0 : (pt >= T ? T - 1 : pt);
     const uint4* src = x + t * d8;
     uint4* dst = xs + r * d8;
     for (int c = lane; c < d8; c += 32) dst[c] = __ldg(src + c);
@@ -576,14 +580,14 @@ cudaError_t launch_dispatch_gather(const int32_t* k, const int32_t* ids, int64_t
                     d / 8, reinterpret_cast<uint4*>(xs));
 }
 
-cudaError_t launch_gather(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int N,
-                          int64_t P, int d, uint16_t* xs, int num_sms, cudaStream_t stream) {
-  if (P == 0) return cudaSuccess;
+cudaError_t launch_gather(const uint16_t* x, int64_t T, const int32_t* perm, const int32_t* offsets,
+                          int N, int64_t P, int d, uint16_t* xs, int num_sms, cudaStream_t stream) {
+  if (P == 0 || T == 0) return cudaSuccess;
   int64_t blocks = (P + 7) / 8;
   const int64_t cap = static_cast<int64_t>(num_sms) * 16;
   if (blocks > cap) blocks = cap;
   disp::gather_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
-      reinterpret_cast<const uint4*>(x), perm, offsets, N, d / 8, reinterpret_cast<uint4*>(xs));
+      reinterpret_cast<const uint4*>(x), perm, offsets, N, T, P, d / 8, reinterpret_cast<uint4*>(xs));
   return cudaGetLastError();
 }
 

@@ -115,7 +115,9 @@ struct Args {
   const int32_t* offsets;   // [G + 1] row offsets per group (grouped modes)
   const int32_t* tile_off;  // [G + 1] prefix sums of ceil(rows_g / 128)
   int groups;               // G
-  int64_t m_rows;           // router: T
+  int64_t m_rows;           // router: T (kGateUpGather: the rows of x)
+  int64_t p_rows;           // grouped and decode modes: the row capacity P of the
+                            // dispatched operand and the output
   int n_tiles;              // n-blocks per group
   int k_blocks;             // K / 64
   int b_rows;               // rows of B per group (2I for gate/up, d for down)
@@ -158,6 +160,10 @@ MOE_DEV Tile decode(int tile, const Args& a, const int* s_off, const int* s_toff
     t.nb = tile % a.n_tiles;
     t.row0 = s_off[t.g];
     t.rows = s_off[t.g + 1] - t.row0;
+    // rows stay inside [0, P) whatever the offsets say
+    t.rows = (t.row0 < 0 || t.row0 >= a.p_rows)
+                 ? 0
+                 : static_cast<int>(min_of<int64_t>(t.rows, a.p_rows - t.row0));
     return t;
   }
   int lo = 0, hi = a.groups;  // s_toff[lo] * n_tiles <= tile < s_toff[hi] * n_tiles
@@ -172,6 +178,10 @@ MOE_DEV Tile decode(int tile, const Args& a, const int* s_off, const int* s_toff
   t.nb = local / mt;
   t.row0 = s_off[lo] + mb * BM;
   t.rows = min(BM, s_off[lo + 1] - t.row0);
+  // rows stay inside [0, P) whatever the offsets say
+  t.rows = (t.row0 < 0 || t.row0 >= a.p_rows)
+               ? 0
+               : static_cast<int>(min_of<int64_t>(t.rows, a.p_rows - t.row0));
   return t;
 }
 
@@ -335,7 +345,9 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         const int r = 32 * warp + 4 * i + (lane >> 3);
-        int tok = args.perm[t.row0 + (r < t.rows ? r : 0)];
+        // rows past the expert's end (never stored) repeat its first token; a
+        // tile left without rows reads token 0
+        int tok = t.rows > 0 ? args.perm[t.row0 + (r < t.rows ? r : 0)] : 0;
         tok = min(max(tok, 0), static_cast<int>(args.m_rows - 1));
         roff[i] = static_cast<int64_t>(tok) * args.lda + chunk * 8;
       }
@@ -836,6 +848,7 @@ cudaError_t launch_gateup_gather_gemm(const uint16_t* x, int64_t T, const int32_
   a.offsets = offsets;
   a.tile_off = tile_off;
   a.groups = N;
+  a.p_rows = P;
   a.n_tiles = I / 128;
   a.k_blocks = d / BK;
   a.b_rows = 2 * I;
@@ -864,6 +877,7 @@ cudaError_t launch_gateup_gemm(const uint16_t* xs, const uint16_t* wgu, const in
   a.offsets = offsets;
   a.tile_off = tile_off;
   a.groups = N;
+  a.p_rows = P;
   a.n_tiles = I / 128;
   a.k_blocks = d / BK;
   a.b_rows = 2 * I;
@@ -887,6 +901,7 @@ cudaError_t launch_down_gemm(const uint16_t* h, const uint16_t* wd, const int32_
   a.offsets = offsets;
   a.tile_off = tile_off;
   a.groups = N;
+  a.p_rows = P;
   a.n_tiles = d / 256;
   a.k_blocks = I / BK;
   a.b_rows = d;
@@ -920,6 +935,7 @@ cudaError_t launch_gateup_decode_gemm(const uint16_t* xs, const uint16_t* wgu,
   Args a{};
   a.offsets = offsets;
   a.groups = N;
+  a.p_rows = P;
   a.n_tiles = I / 64;
   a.k_blocks = d / BK;
   a.b_rows = 2 * I;
@@ -949,6 +965,7 @@ cudaError_t launch_down_decode_gemm(const uint16_t* h, const uint16_t* wd, const
   Args a{};
   a.offsets = offsets;
   a.groups = N;
+  a.p_rows = P;
   a.n_tiles = d / BM;
   a.k_blocks = I / BK;
   a.b_rows = d;
