@@ -213,3 +213,17 @@ def test_layer_wide_sampled(moe):
     flip, _ = _routing_flip_fraction(inp, got)
     assert flip <= 2e-3, flip
     _compare_layer(inp, got, _sampled(w["T"], 24, 2), max_flip=0.05)
+
+
+@pytest.mark.parametrize("N,K,mode", [(64, 1, 1), (64, 3, 0), (128, 4, 0), (128, 5, 1)])
+def test_layer_prefill_other_caps(moe, N, K, mode):
+    """The prefill path (T > 64: multi-chunk dispatch, gathered gate/up GEMM,
+    down GEMM, combine) with caps K < 8, every token against the oracle."""
+    T, d, I = 1000, 512, 256
+    inp = synth.layer_inputs(T=T, d=d, N=N, I=I, seed=2100 + N + K)
+    got = _run_layer(moe, inp, K=K, mode=mode)
+    r = oracle.route(got["logits"], K=K, mode=mode)
+    assert np.array_equal(r["k"], got["k"]) and np.array_equal(r["ids"], got["ids"])
+    d_ref = oracle.dispatch(got["k"], got["ids"], N)
+    assert np.array_equal(d_ref["offsets"], got["offsets"])
+    _compare_layer(inp, got, np.arange(T), K=K, mode=mode, max_flip=0.02)

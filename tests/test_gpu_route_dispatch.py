@@ -201,6 +201,17 @@ def test_dispatch_drops_out_of_range_ids(moe, N, T):
 
 
 @pytest.mark.parametrize("N", [64, 128])
+@pytest.mark.parametrize("K", [1, 3, 5, 7])
+@pytest.mark.parametrize("T", [100, 3001])
+def test_dispatch_other_caps(moe, N, K, T):
+    """K < 8: rows of ids that are not 32 bytes (element loads instead of the
+    16-byte ones), in the one-block and the multi-chunk dispatch."""
+    rng = np.random.default_rng(T + N + 31 * K)
+    r = oracle.route(synth.boosted_logits(rng, T, N), K=K)
+    _dispatch_both(moe, r["k"], r["ids"], N)
+
+
+@pytest.mark.parametrize("N", [64, 128])
 @pytest.mark.parametrize("T", [1, 33, 2047, 2048, 2049, 20000])
 def test_dispatch_bitexact(moe, N, T):
     rng = np.random.default_rng(T + N)
