@@ -305,7 +305,8 @@ def run_ours(args, rank, world, local, pg):
             "parallelism": f"replicas x{world} (independent batches, no collective)",
         },
         "topk": {"value": job_tokens_per_s(T, world, ms_topk), "unit": "tokens/s", "ms_per_step": ms_topk,
-                 "elbow_speedup": ms_topk / ms_elbow},
+                 "elbow_speedup": ms_topk / ms_elbow,
+                 "gpu_launches": KERNELS_PER_STEP * args.steps},
         "routing": {"mean_k": sum_k / T, "k_hist": np.bincount(kk, minlength=K + 1)[1:].tolist(),
                     "expert_load_min": int(load.min()), "expert_load_max": int(load.max())},
         "roofline": {"kernel": "grouped gate/up GEMM + SwiGLU, gathered rows (tcgen05)",
@@ -324,7 +325,8 @@ def run_ours(args, rank, world, local, pg):
                 "pipelined": "copy-in and copy-out streams, two device x/y buffers: step i's "
                              "copy-out and step i+1's copy-in overlap step i's layer",
                 "serial_ms_per_step": ms_e2e_serial},
-        "gpu_launches": KERNELS_PER_STEP * args.steps * 2,
+        # kernels launched in the timed region of `value` (the elbow steps)
+        "gpu_launches": KERNELS_PER_STEP * args.steps,
         "clocks": clocks,
     }
     if rank == 0 and not args.no_cpu_baseline:
