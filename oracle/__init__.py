@@ -55,7 +55,9 @@ def _load():
     with _lock:
         if _lib is not None:
             return _lib
-        lib = ctypes.CDLL(build())
+        # ORACLE_LIBRARY: a library built from a modified copy of elbow_oracle.c
+        # (test support: the mutation tests check that the pins reject it)
+        lib = ctypes.CDLL(os.environ.get("ORACLE_LIBRARY") or build())
         P = ctypes.c_void_p
         i64, i32, f32 = ctypes.c_int64, ctypes.c_int, ctypes.c_float
         lib.oracle_exp.argtypes = [f32]

@@ -206,6 +206,23 @@ def test_renorm_gates():
     assert np.all(one["gates"][:, 0] == 1.0)
 
 
+@pytest.mark.parametrize("shift", [512.0, -512.0])
+def test_softmax_shift_invariance(shift):
+    """Softmax is invariant under adding one constant to all logits. On logits of a
+    2^-10 grid within +-32 the shifted logits, and their differences to the
+    shifted maximum, are exact in fp32, so the routing must be bit-identical;
+    a softmax that skipped the max subtraction would overflow (+512) or underflow
+    (-512) here."""
+    rng = np.random.default_rng(77)
+    for N in (64, 128):
+        lg = (np.round(rng.normal(0.0, 4.0, (300, N)) * 1024.0) / 1024.0).clip(-32, 32)
+        lg = lg.astype(np.float32)
+        a = oracle.route(lg, K=8)
+        b = oracle.route((lg + np.float32(shift)).astype(np.float32), K=8)
+        assert np.array_equal(a["k"], b["k"]) and np.array_equal(a["ids"], b["ids"])
+        assert np.array_equal(a["gates"].view(np.uint32), b["gates"].view(np.uint32))
+
+
 def test_flat_and_degenerate():
     N = 64
     # all logits equal: R = 0, k = 1 (documented degenerate case)
