@@ -46,6 +46,14 @@ MUTANTS = [
     ("dispatch_not_stable",
      "  for (int64_t t = 0; t < T; ++t) {\n    for (int s = 0; s < K; ++s) {",
      "  for (int64_t t = T - 1; t >= 0; --t) {\n    for (int s = 0; s < K; ++s) {"),
+    ("unselected_pair_pos_zero",
+     "        pair_pos[t * K + s] = -1;", "        pair_pos[t * K + s] = 0;"),
+    ("offsets_off_by_one",
+     "for (int e = 0; e < N; ++e) offsets[e + 1] = offsets[e] + (int32_t)cnt[e];",
+     "for (int e = 0; e < N; ++e) offsets[e + 1] = offsets[e] + (int32_t)cnt[e] + (e == 0);"),
+    ("residual_dropped",
+     "for (int c = 0; c < d; ++c) yr[c] += bf16_to_double(residual[t * d + c]);",
+     "for (int c = 0; c < d; ++c) yr[c] += 0.0 * bf16_to_double(residual[t * d + c]);"),
     ("router_weight_transposed",
      "acc += bf16_to_double(xr[c]) * bf16_to_double(w_router[(int64_t)j * d + c]);",
      "acc += bf16_to_double(xr[c]) * bf16_to_double(w_router[(int64_t)c * N + j]);"),
