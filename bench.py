@@ -663,7 +663,7 @@ def route_stress(moe, args, stream, dev, pk, cpu=False):
         same = bool(np.array_equal(r["k"], k[:n].cpu().numpy()) and
                     np.array_equal(r["ids"], ids[:n].cpu().numpy()))
         cpu_route = {"tokens_per_s": n / dt, "GBps": n * (4 * N + 4 + 8 * K) / dt / 1e9,
-                     "cores": int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1)),
+                     "cores": oracle.threads(),
                      "cpu": cpu_model(), "kind": "oracle",
                      "sample": f"the first {n} of the {T} tokens, {dt:.2f} s",
                      "gpu_bitexact_on_sample": same}
@@ -711,8 +711,9 @@ def cpu_model():
     return "unknown"
 
 
-def cpu_baseline(inp, K, budget_s=12.0):
-    """The CPU oracle, as it stands, on a bounded sample of the same workload."""
+def cpu_baseline(inp, K, budget_s=12.0, single_budget_s=4.0):
+    """The CPU oracle, as it stands, on a bounded sample of the same workload:
+    with all of its OpenMP threads (the reported value) and with one."""
     import oracle
     T = inp["x"].shape[0]
     # calibrate the per-token cost on 128 tokens after an 8-token warm-up (the
@@ -728,9 +729,23 @@ def cpu_baseline(inp, K, budget_s=12.0):
     t0 = time.perf_counter()
     oracle.layer_rows(inp["x"], inp["w_router"], inp["w_gate_up"], inp["w_down"], rows=rows, K=K)
     dt = time.perf_counter() - t0
-    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    cores = oracle.threads()
+    # one thread, on a sample sized from the per-token time above
+    threads = oracle.threads()
+    n1 = int(min(T, max(8, single_budget_s * n / (dt * threads))))
+    rows1 = np.linspace(0, T - 1, n1).astype(np.int64)
+    oracle.set_threads(1)
+    try:
+        t0 = time.perf_counter()
+        oracle.layer_rows(inp["x"], inp["w_router"], inp["w_gate_up"], inp["w_down"], rows=rows1,
+                          K=K)
+        dt1 = time.perf_counter() - t0
+    finally:
+        oracle.set_threads(threads)
     return {"value": n / dt, "unit": "tokens/s", "cores": cores, "kind": "oracle", "cpu": cpu_model(),
-            "sample": f"{n} of the {T} tokens of the same layer (fp64 C oracle, OpenMP), {dt:.1f} s"}
+            "sample": f"{n} of the {T} tokens of the same layer (fp64 C oracle, OpenMP), {dt:.1f} s",
+            "single_thread": {"value": n1 / dt1, "unit": "tokens/s", "cores": 1,
+                              "sample": f"{n1} of the {T} tokens, one thread, {dt1:.1f} s"}}
 
 
 def run_reference(args, rank, world):
@@ -760,7 +775,7 @@ def run_reference(args, rank, world):
         step()
     dt = (time.perf_counter() - t0) / n
     val = sample / dt
-    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    cores = oracle.threads()
     return {
         "impl": "reference", "metric": METRIC, "value": val, "unit": "tokens/s", "n_gpus": world,
         "steps": n, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,

@@ -15,6 +15,7 @@ Functions and the passages they follow:
   elbow_angle    the uncapped elbow index and the elbow angle of Sec. 2.3
   route_randomized  the tail / head randomisation experiment of Sec. 2.2
   exp / exp_max_ulp  the fp32 routing exponential and its error sweep
+  threads / set_threads  the OpenMP thread count (timing support)
 The readings taken where the paper is silent or garbled are listed in the
 header of elbow_oracle.c.
 """
@@ -60,6 +61,10 @@ def _load():
         lib = ctypes.CDLL(os.environ.get("ORACLE_LIBRARY") or build())
         P = ctypes.c_void_p
         i64, i32, f32 = ctypes.c_int64, ctypes.c_int, ctypes.c_float
+        lib.oracle_max_threads.argtypes = []
+        lib.oracle_max_threads.restype = i32
+        lib.oracle_set_threads.argtypes = [i32]
+        lib.oracle_set_threads.restype = None
         lib.oracle_exp.argtypes = [f32]
         lib.oracle_exp.restype = f32
         lib.oracle_exp_max_ulp.argtypes = [f32, f32, P]
@@ -89,6 +94,16 @@ def _ptr(a):
 
 def _c(a, dtype):
     return np.ascontiguousarray(a, dtype=dtype)
+
+
+def threads() -> int:
+    """OpenMP threads the oracle's parallel loops use."""
+    return int(_load().oracle_max_threads())
+
+
+def set_threads(n: int) -> None:
+    """Set the OpenMP threads of the oracle's parallel loops (timing support)."""
+    _load().oracle_set_threads(int(n))
 
 
 def exp(z):

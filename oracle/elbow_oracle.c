@@ -64,11 +64,19 @@
  * Build: gcc -O2 -std=c11 -ffp-contract=off (no fast-math), OpenMP over tokens.
  */
 #include <math.h>
+#include <omp.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
 
 #define ORACLE_MAX_N 1024
+
+/* OpenMP threads the oracle's parallel loops use, and setting them (timing
+ * support: the CPU baseline is reported with all cores and with one). */
+int oracle_max_threads(void) { return omp_get_max_threads(); }
+void oracle_set_threads(int n) {
+  if (n >= 1) omp_set_num_threads(n);
+}
 
 /* ---------------------------------------------------------------- EXP spec */
 static const float LOG2E = 0x1.715476p+0f;
