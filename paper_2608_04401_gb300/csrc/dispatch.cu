@@ -12,6 +12,8 @@
 //             warps of the chunk (per-expert warp masks in smem) + earlier lanes
 //             of the warp (popc of the mask). Chunk 0 also writes offsets [N+1] and the
 //             m-tile prefix sums ceil(count_e / 128) [N+1].
+// A pair whose expert id lies outside [0, N) is dropped by every pass (not
+// counted, not placed, pair_pos -1), so no id indexes outside the arrays.
 #include <mutex>
 
 #include "common.cuh"
