@@ -67,7 +67,8 @@ typedef struct {
   int renorm;
 } moe_route_params;
 
-/* Human-readable name of a status code (static storage). */
+/* Human-readable name of a status code (static storage; "unknown moe_status"
+ * for other values). No counterpart in the paper. */
 const char* moe_status_string(moe_status s);
 
 /*
@@ -93,7 +94,7 @@ const char* moe_status_string(moe_status s);
 moe_status elbow_route(const float* logits, int64_t T, int N, const moe_route_params* rp,
                        int32_t* k_out, int32_t* ids_out, float* gates_out, void* stream);
 
-/* elbow_route with one warp (instead of one thread) per token: lane l holds
+/* elbow_route (Alg. 1, Sec. 2.1) with one warp (instead of one thread) per token: lane l holds
  * experts l + 32c, the N (p, id) keys are sorted by a bitonic network of warp
  * shuffles and the argmax is a warp reduction. Same specification, same bits
  * as elbow_route; a much shorter critical path per token, at about three
@@ -104,7 +105,7 @@ moe_status elbow_route(const float* logits, int64_t T, int N, const moe_route_pa
 moe_status elbow_route_warp(const float* logits, int64_t T, int N, const moe_route_params* rp,
                             int32_t* k_out, int32_t* ids_out, float* gates_out, void* stream);
 
-/* elbow_route that also counts, for the dispatch, the selected pairs of each
+/* elbow_route (Alg. 1, Sec. 2.1) that also counts, for the dispatch (App. A.4), the selected pairs of each
  * expert in each chunk of 128 tokens: chunk_counts [N][ceil(T/128)] int32
  * (pass moe_dispatch_chunk_counts(ws) and follow with moe_dispatch_counted,
  * which then skips its own counting pass over k and ids). */
@@ -203,16 +204,23 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
  */
 moe_status moe_read_device_error(const void* ws, void* stream);
 
-/* ---- step-level entry points (the layer's stages, for testing and reuse) ---- */
+/* ---- step-level entry points (the layer's stages, for testing and reuse) ----
+ *
+ * Errors, for each of them: MOE_ERR_INVALID_ARG for a null or misaligned
+ * pointer (16 bytes for tensors, 4 bytes for int32 / fp32 arrays and the
+ * error word) or a size out of range; MOE_ERR_UNSUPPORTED for N, K, d or I
+ * outside the supported set; MOE_ERR_CUDA if a launch fails. A GEMM that gives
+ * up a bounded wait writes a nonzero code into err_word (when given). */
 
-/* Router logits l = W_r x: x [T, d] bf16, w_router [N, d] bf16 -> logits [T, N]
+/* Router logits l = W_r x (the router of Sec. 2): x [T, d] bf16, w_router [N, d] bf16 -> logits [T, N]
  * fp32 (tensor cores, fp32 accumulation). d a multiple of 64. err_word: a
  * device int32 that receives a nonzero code on a device timeout (may be NULL). */
 moe_status moe_router_logits(const uint16_t* x, const uint16_t* w_router, int64_t T, int d, int N,
                              float* logits, int32_t* err_word, void* stream);
 
 /* Router GEMM with the elbow routing fused into its epilogue (the layer's
- * first stage): the same logits as moe_router_logits, routed exactly as
+ * first stage; Sec. 2, Alg. 1 and Sec. 2.1): the same logits as
+ * moe_router_logits, routed exactly as
  * elbow_route routes them. logits_out [T, N] may be NULL (the logits then stay
  * on chip). chunk_counts [N][ceil(T/128)] int32 (may be NULL): the number of
  * selected pairs of each expert in each chunk of 128 tokens. */
@@ -222,13 +230,15 @@ moe_status moe_router_route(const uint16_t* x, const uint16_t* w_router, int64_t
                             int32_t* err_word, void* stream);
 
 /* moe_expert_gate_up with the rows gathered from x [T, d] by perm (row r of
- * expert e is token perm[r]), without a gathered copy of x. */
+ * expert e is token perm[r]), without a gathered copy of x (App. A.4: each
+ * expert applies its MLP to the tokens routed to it). */
 moe_status moe_expert_gate_up_gathered(const uint16_t* x, int64_t T, const int32_t* perm,
                                        const uint16_t* w_gate_up, const int32_t* offsets,
                                        const int32_t* tile_off, int64_t P, int d, int N, int I,
                                        uint16_t* h, int32_t* err_word, void* stream);
 
-/* Expert SwiGLU over dispatched rows: for each expert e and each row r in
+/* Expert SwiGLU over dispatched rows (the expert MLP of App. A.4, in the
+ * SwiGLU form of the OLMoE experts): for each expert e and each row r in
  * [offsets[e], offsets[e+1]): h[r] = silu(W_gate[e] xs[r]) * (W_up[e] xs[r]),
  * with xs [P, d] bf16 the tokens already gathered in dispatch order (P = the
  * row capacity, >= offsets[N]), h [P, I] bf16. `tile_off` [N + 1] int32 are
@@ -238,13 +248,15 @@ moe_status moe_expert_gate_up(const uint16_t* xs, const uint16_t* w_gate_up, con
                               const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* h,
                               int32_t* err_word, void* stream);
 
-/* Expert down projection: o[r] = W_down[e] h[r] for rows of expert e;
+/* Expert down projection (the second matrix of the expert MLP, App. A.4):
+ * o[r] = W_down[e] h[r] for rows of expert e;
  * h [P, I] bf16 -> o [P, d] bf16. */
 moe_status moe_expert_down(const uint16_t* h, const uint16_t* w_down, const int32_t* offsets,
                            const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* o,
                            int32_t* err_word, void* stream);
 
-/* Decode-shaped expert contractions for batches of T <= 64 tokens, where an
+/* Decode-shaped expert contractions (App. A.4, in the small-batch latency
+ * regime of Sec. 3) for batches of T <= 64 tokens, where an
  * expert has at most T rows (a token selects an expert at most once): the
  * same results as moe_expert_gate_up and moe_expert_down, computed with the
  * weights as the M operand (128 weight rows per tile, the expert's rows as N,
@@ -264,29 +276,36 @@ moe_status moe_expert_down_decode(const uint16_t* h, const uint16_t* w_down, con
 
 /* Device pointer, inside a moe_dispatch workspace, of the [N + 1] int32 tile
  * offsets (exclusive prefix sums of ceil(count_e / 128)) that the last
- * moe_dispatch on that workspace wrote. */
+ * moe_dispatch on that workspace wrote. No counterpart in the paper (the
+ * expert GEMMs' tile schedule). NULL for a NULL ws or unsupported N. */
 const int32_t* moe_dispatch_tile_offsets(const void* ws, int64_t T, int N, int K);
 
 /* Device pointer, inside a moe_dispatch workspace, of the [N][ceil(T/128)]
  * int32 per-chunk expert counts: pass it as moe_router_route's chunk_counts,
- * then call moe_dispatch_counted, which skips its own counting pass. */
+ * then call moe_dispatch_counted, which skips its own counting pass. The
+ * first pass of the dispatch (App. A.4); NULL for a NULL ws or unsupported N. */
 int32_t* moe_dispatch_chunk_counts(void* ws, int64_t T, int N, int K);
 
-/* moe_dispatch whose per-chunk expert counts are already in the workspace
- * (written there by moe_router_route); otherwise identical. */
+/* moe_dispatch (App. A.4) whose per-chunk expert counts are already in the
+ * workspace (written there by moe_router_route or elbow_route_with_counts);
+ * otherwise identical, errors included. */
 moe_status moe_dispatch_counted(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
                                 int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
                                 size_t ws_bytes, void* stream);
 
-/* Gather rows: xs[r] = x[perm[r]] for r < offsets[N] (x [T, d] bf16,
+/* Gather rows (sending each token to its experts, App. A.4):
+ * xs[r] = x[perm[r]] for r < offsets[N] (x [T, d] bf16,
  * xs [P, d] bf16, P >= offsets[N]). Rows stop at P and tokens outside [0, T)
  * are clamped into it, so inconsistent arguments cannot reach outside x or
  * xs. */
 moe_status moe_gather_rows(const uint16_t* x, const int32_t* perm, const int32_t* offsets, int64_t T,
                            int64_t P, int d, int N, uint16_t* xs, void* stream);
 
-/* Combine: y_t = sum_{s < k_t} gates[t,s] * o[pair_pos[t,s]] (+ residual_t),
- * fp32 in s order, rounded to bf16. o [P, d] bf16; residual may be NULL. */
+/* Combine (the gate-weighted sum of the selected experts' outputs that the MoE
+ * block returns, Sec. 1 and App. A.4):
+ * y_t = sum_{s < k_t} gates[t,s] * o[pair_pos[t,s]] (+ residual_t),
+ * fp32 in s order, rounded to bf16. o [P, d] bf16; residual may be NULL.
+ * Positions are clamped to the T * K rows of o. */
 moe_status moe_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_pos,
                        const float* gates, const uint16_t* residual, int64_t T, int d, int K,
                        uint16_t* y, void* stream);
