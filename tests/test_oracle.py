@@ -262,14 +262,17 @@ def test_theorem1_and_corollaries():
 def test_load_balance_hand_example():
     """Two tokens, N = 4, K = 2: token 0 keeps expert 0 of (0, 1), token 1 keeps
     both of (0, 2). By hand: q_top = (1/2, 1/4, 1/4, 0), q_elb = (2/3, 0, 1/3, 0),
-    delta = 1/4, l1 = 1/2 <= 2/3, CV^2 = 1/2 and 11/9, top-1 share change
-    (1/2 - 2/3) / (1/2) = -100/3 %, CV change (sqrt(1/2) - sqrt(11/9)) / sqrt(1/2)."""
+    delta = 1/4, l1 = 1/2 <= 2/3, top-1 share change |2/3 - 1/2| = 1/6, CV^2 = 1/2
+    and 11/9 with Corollary 2's bound 2 N delta / (1 - delta)^2 = 32/9, top-1 share
+    change (1/2 - 2/3) / (1/2) = -100/3 %, CV change (sqrt(1/2) - sqrt(11/9)) / sqrt(1/2)."""
     lb = oracle.load_balance(np.array([1, 2]), np.array([[0, 1], [0, 2]]), 4)
     np.testing.assert_allclose(lb["q_top"], [0.5, 0.25, 0.25, 0.0], atol=1e-15)
     np.testing.assert_allclose(lb["q_elb"], [2 / 3, 0.0, 1 / 3, 0.0], atol=1e-15)
     assert abs(lb["delta"] - 0.25) < 1e-15
     assert abs(lb["l1"] - 0.5) < 1e-15 and abs(lb["l1_bound"] - 2 / 3) < 1e-15
+    assert abs(lb["max_change"] - 1 / 6) < 1e-15
     assert abs(lb["cv2_change"] - (11 / 9 - 0.5)) < 1e-14
+    assert abs(lb["cv2_bound"] - 32 / 9) < 1e-14
     assert abs(lb["top1_share_change_pct"] + 100 / 3) < 1e-12
     want = (np.sqrt(0.5) - np.sqrt(11 / 9)) / np.sqrt(0.5) * 100
     assert abs(lb["cv_change_pct"] - want) < 1e-12

@@ -104,3 +104,40 @@ def test_control_build_passes_the_pins(tmp_path):
 def test_pins_reject_planted_mistake(tmp_path, name, old, new):
     rc, out = _run_pins(_build(str(tmp_path), name, old, new))
     assert rc == 1, f"no pin failed on {name}:\n{out}"
+
+
+# Mistakes planted in the oracle's Python part (the load metrics of App. A.3):
+# the function is rebuilt from its source with one change and swapped in for
+# the pins of test_oracle.py that exercise it.
+LOAD_MUTANTS = [
+    ("delta_sign", "delta = 1.0 - k_elb.mean() / K", "delta = k_elb.mean() / K"),
+    ("elbow_load_counts_slot_k", "if s < k_elb[t]:", "if s <= k_elb[t]:"),
+    ("l1_bound_missing_factor_2", "l1_bound=2 * delta / (1 - delta),",
+     "l1_bound=delta / (1 - delta),"),
+    ("cv2_bound_square_dropped", "cv2_bound=2 * N * delta / (1 - delta) ** 2,",
+     "cv2_bound=2 * N * delta / (1 - delta),"),
+    ("max_change_of_minima", "max_change=abs(q_elb.max() - q_top.max()),",
+     "max_change=abs(q_elb.min() - q_top.min()),"),
+    ("q_not_normalised", "q_elb = L_elb / L_elb.sum()", "q_elb = L_elb"),
+]
+
+
+@pytest.mark.parametrize("name,old,new", LOAD_MUTANTS, ids=[m[0] for m in LOAD_MUTANTS])
+def test_load_pins_reject_planted_mistake(monkeypatch, name, old, new):
+    import inspect
+
+    import oracle
+    import test_oracle as pins
+
+    src = inspect.getsource(oracle.load_balance)
+    assert src.count(old) == 1, f"{name}: the line to plant the mistake in is not unique"
+    ns = dict(vars(oracle))
+    exec(compile(src.replace(old, new), "<mutant>", "exec"), ns)
+    monkeypatch.setattr(oracle, "load_balance", ns["load_balance"])
+    failed = 0
+    for pin in (pins.test_theorem1_and_corollaries, pins.test_load_balance_hand_example):
+        try:
+            pin()
+        except AssertionError:
+            failed += 1
+    assert failed >= 1, f"no pin failed on {name}"
