@@ -154,10 +154,14 @@ moe_status moe_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, 
  * N in {64, 128}, K <= 8.
  * No cudaMalloc, cudaFree or other allocating call is made.
  * The first call on each device looks up the array's device address (with
- * that device current) and caches it; make that first call before any stream
- * capture. All calls share the one array and each call rewrites every part of
- * it that it reads, so no clearing is needed; calls whose kernels overlap on
- * the GPU (different streams, or different host threads) race on the array.
+ * that device current) and caches it for the life of the process; make that
+ * first call before any stream capture. cudaDeviceReset may move the array,
+ * so this entry point must not be called again after a reset of a device it
+ * has already been used on. All calls share the one array and each call
+ * rewrites every part of it that it reads, so no clearing is needed; calls
+ * whose kernels overlap on the GPU (different streams, or different host
+ * threads) race on the array. Launch failures return MOE_ERR_CUDA (errors
+ * left pending by earlier, unrelated calls are not read).
  */
 moe_status moe_dispatch_noalloc(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
                                 int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* stream);

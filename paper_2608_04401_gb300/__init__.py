@@ -321,14 +321,27 @@ def moe_dispatch_noalloc(k, ids, N: int, offsets=None, perm=None, pair_pos=None,
     lib = library()
     _cuda(k, torch.int32, "k")
     _cuda(ids, torch.int32, "ids")
+    if ids.dim() != 2:
+        raise ValueError("ids must be [T, K]")
     T, K = ids.shape
     dev = ids.device
+    if k.numel() != T or k.device != dev:
+        raise ValueError(f"k must hold T = {T} counts on {dev}")
     if offsets is None:
         offsets = torch.empty(N + 1, dtype=torch.int32, device=dev)
     if perm is None:
         perm = torch.empty(max(1, T * K), dtype=torch.int32, device=dev)
     if pair_pos is None:
         pair_pos = torch.empty(T, K, dtype=torch.int32, device=dev)
+    # the C entry point cannot see buffer sizes: every caller-supplied buffer is
+    # checked here, before the kernels could write past its end
+    for name, buf, need in (("offsets", offsets, N + 1), ("perm", perm, max(1, T * K)),
+                            ("pair_pos", pair_pos, T * K)):
+        _cuda(buf, torch.int32, name)
+        if buf.device != dev:
+            raise ValueError(f"{name} must be on {dev}")
+        if buf.numel() < need:
+            raise ValueError(f"{name} holds {buf.numel()} entries, needs {need}")
     _check(lib.moe_dispatch_noalloc(_p(k), _p(ids), T, N, K, _p(offsets), _p(perm), _p(pair_pos),
                                     _stream(stream)), "moe_dispatch_noalloc")
     return offsets, perm, pair_pos

@@ -701,8 +701,8 @@ extern "C" moe_status moe_dispatch_noalloc(const int32_t* k, const int32_t* ids,
   int32_t* cnt = scratch;
   int32_t* totals = scratch + kNoAllocChunks * kNoAllocMaxExperts;
   int32_t* tile_off = totals + kNoAllocMaxExperts;
-  if (moe::run_dispatch(k, ids, T, N, K, offsets, perm, pair_pos, cnt, totals, tile_off, nullptr,
-                        false, static_cast<cudaStream_t>(stream)) != cudaSuccess)
-    return MOE_ERR_CUDA;
-  return cudaGetLastError() == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
+  return moe::run_dispatch(k, ids, T, N, K, offsets, perm, pair_pos, cnt, totals, tile_off, nullptr,
+                           false, static_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? MOE_OK
+             : MOE_ERR_CUDA;
 }
