@@ -13,6 +13,7 @@ Functions and the passages they follow:
   load_balance   L_i, q_i, delta and the bounds of Theorem 1 / Corollaries 1-2
                  (App. A.3), the percentage changes of Sec. 2.4
   elbow_angle    the uncapped elbow index and the elbow angle of Sec. 2.3
+  elbow_curve    Alg. 1's sorted p, normalised p' and deviation D per rank
   route_randomized  the tail / head randomisation experiment of Sec. 2.2
   exp / exp_max_ulp  the fp32 routing exponential and its error sweep
   threads / set_threads  the OpenMP thread count (timing support)
@@ -73,6 +74,8 @@ def _load():
         lib.oracle_route.restype = i32
         lib.oracle_route_randomized.argtypes = [P, i64, i32, i32, f32, i32, i32, P, P, P, P]
         lib.oracle_route_randomized.restype = i32
+        lib.oracle_elbow_curve.argtypes = [P, i64, i32, f32, P, P, P]
+        lib.oracle_elbow_curve.restype = i32
         lib.oracle_elbow_angle.argtypes = [P, i64, i32, f32, P, P]
         lib.oracle_elbow_angle.restype = i32
         lib.oracle_angle_deg.argtypes = [i32, i32, f32]
@@ -119,6 +122,18 @@ def exp_max_ulp(lo: float, hi: float):
     wz = ctypes.c_float(0.0)
     err = lib.oracle_exp_max_ulp(lo, hi, ctypes.byref(wz))
     return err, wz.value
+
+
+def elbow_curve(logits, eps: float = 1e-8):
+    """Alg. 1's curve per token in sorted order: dict(p, pn, D), each [T, N]."""
+    lib = _load()
+    lg = _c(logits, np.float32)
+    T, N = lg.shape
+    out = {n: np.empty((T, N), np.float32) for n in ("p", "pn", "D")}
+    if lib.oracle_elbow_curve(_ptr(lg), T, N, eps, _ptr(out["p"]), _ptr(out["pn"]),
+                              _ptr(out["D"])) != 0:
+        raise ValueError("oracle_elbow_curve: unsupported arguments")
+    return out
 
 
 def route(logits, K: int = 8, eps: float = 1e-8, mode: int = MODE_ELBOW, renorm: int = 0,

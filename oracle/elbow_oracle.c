@@ -32,12 +32,14 @@
  *       probabilities, unrenormalised (renorm = 1 divides by their sum).
  *   R6  Precision of routing: the elbow decision is an integer taken from
  *       floating point, so it is specified here in fp32, step by step, with
- *       every operation rounded to nearest even and no contraction:
+ *       every operation of the printed formulas (the softmax of Sec. 2 and
+ *       Alg. 1's normalisation and deviation) rounded once to nearest even
+ *       and no contraction:
  *         m = max_j l_j;  z_j = l_j - m;  e_j = EXP(z_j) (spec below);
  *         s = balanced tree sum (v_i += v_{i+h}, h = N/2, ..., 1);
- *         r = 1 / s;  p_j = e_j * r;
- *         den = (p_max - p_min) + eps;  inv = 1 / den;
- *         p'_i = (p_(i) - p_min) * inv;  x'_i = i / (N - 1);
+ *         p_j = e_j / s;
+ *         den = (p_max - p_min) + eps;
+ *         p'_i = (p_(i) - p_min) / den;  x'_i = i / (N - 1);
  *         D_i = (1 - p'_i) - x'_i.
  *   R7  Expert MLP: SwiGLU, y_e = W_down (silu(W_gate x) * (W_up x)),
  *       silu(z) = z / (1 + exp(-z)), evaluated in fp64 on the bf16 inputs.
@@ -144,10 +146,12 @@ double oracle_exp_max_ulp(float lo, float hi, float* worst_z) {
 
 /* ------------------------------------------------------------- routing */
 
-/* Algorithm 1 plus capped selection for one token. Returns k. */
+/* Algorithm 1 plus capped selection for one token. Returns k. Optional
+ * outputs (NULL = not written): sorted_p [N], elbow_e, elbow_pn, p_out [N]
+ * (unsorted p), pn_all [N] and d_all [N] (p'_i and D_i in sorted order). */
 static int route_one(const float* l, int N, int K, float eps, int mode, int renorm,
                      int32_t* ids, float* gates, float* sorted_p, int32_t* elbow_e,
-                     float* elbow_pn, float* p_out) {
+                     float* elbow_pn, float* p_out, float* pn_all, float* d_all) {
   float e[ORACLE_MAX_N], p[ORACLE_MAX_N], v[ORACLE_MAX_N];
   int idx[ORACLE_MAX_N];
 
@@ -159,8 +163,8 @@ static int route_one(const float* l, int N, int K, float eps, int mode, int reno
   for (int j = 0; j < N; ++j) v[j] = e[j];
   for (int h = N / 2; h >= 1; h /= 2)
     for (int i = 0; i < h; ++i) v[i] = v[i] + v[i + h];
-  float r = 1.0f / v[0];
-  for (int j = 0; j < N; ++j) p[j] = e[j] * r;
+  float s = v[0];
+  for (int j = 0; j < N; ++j) p[j] = e[j] / s;
   if (p_out)
     for (int j = 0; j < N; ++j) p_out[j] = p[j];
 
@@ -180,13 +184,14 @@ static int route_one(const float* l, int N, int K, float eps, int mode, int reno
   /* Kneedle: p'_i, x'_i, D_i (R1, R6); e = argmax D_i (R3) */
   float p_max = p[idx[0]], p_min = p[idx[N - 1]];
   float den = (p_max - p_min) + eps;
-  float inv = 1.0f / den;
   int e_arg = 0;
   float d_best = 0.0f, pn_best = 0.0f;
   for (int i = 0; i < N; ++i) {
-    float pn = (p[idx[i]] - p_min) * inv;
+    float pn = (p[idx[i]] - p_min) / den;
     float xn = (float)i / (float)(N - 1);
     float D = (1.0f - pn) - xn;
+    if (pn_all) pn_all[i] = pn;
+    if (d_all) d_all[i] = D;
     if (i == 0 || D > d_best) {
       d_best = D;
       e_arg = i;
@@ -223,7 +228,23 @@ int oracle_route(const float* logits, int64_t T, int N, int K, float eps, int mo
   for (int64_t t = 0; t < T; ++t) {
     k_out[t] = route_one(logits + t * N, N, K, eps, mode, renorm, ids_out + t * K,
                          gates_out + t * K, sorted_p_out ? sorted_p_out + t * N : NULL,
-                         elbow_out ? elbow_out + t : NULL, NULL, NULL);
+                         elbow_out ? elbow_out + t : NULL, NULL, NULL, NULL, NULL);
+  }
+  return 0;
+}
+
+/* Per token, the normalised curve of Alg. 1 in sorted order: p_(i), p'_i and
+ * D_i for i = 0..N-1, each [T, N] (test support: the pins check each printed
+ * operation's rounding). Returns 0, or -1 on unsupported arguments. */
+int oracle_elbow_curve(const float* logits, int64_t T, int N, float eps, float* sorted_p,
+                       float* pn_out, float* d_out) {
+  if (N < 2 || N > ORACLE_MAX_N || (N & (N - 1)) != 0 || T < 0) return -1;
+#pragma omp parallel for schedule(static)
+  for (int64_t t = 0; t < T; ++t) {
+    int32_t id1;
+    float g1;
+    route_one(logits + t * N, N, 1, eps, 0, 0, &id1, &g1, sorted_p + t * N, NULL, NULL, NULL,
+              pn_out + t * N, d_out + t * N);
   }
   return 0;
 }
@@ -260,7 +281,7 @@ int oracle_elbow_angle(const float* logits, int64_t T, int N, float eps, int32_t
   for (int64_t t = 0; t < T; ++t) {
     int32_t id1, e;
     float g1, pn;
-    route_one(logits + t * N, N, 1, eps, 0, 0, &id1, &g1, NULL, &e, &pn, NULL);
+    route_one(logits + t * N, N, 1, eps, 0, 0, &id1, &g1, NULL, &e, &pn, NULL, NULL, NULL);
     elbow_out[t] = e;
     theta_out[t] = (float)oracle_angle_deg(e, N, pn);
   }
@@ -291,7 +312,8 @@ int oracle_route_randomized(const float* logits, int64_t T, int N, int K, float 
     int32_t ids[ORACLE_MAX_N];
     float gates[ORACLE_MAX_N], p[ORACLE_MAX_N];
     int taken[ORACLE_MAX_N];
-    int k = route_one(logits + t * N, N, K, eps, 0, 0, ids, gates, NULL, NULL, NULL, p);
+    int k = route_one(logits + t * N, N, K, eps, 0, 0, ids, gates, NULL, NULL, NULL, p, NULL,
+                      NULL);
     for (int j = 0; j < N; ++j) taken[j] = 0;
     int lo = (mode == 2) ? k : 0, hi = (mode == 2) ? K : k;
     int excl = (mode == 2) ? k : K; /* ranks 0..excl-1 are not candidates */
@@ -437,7 +459,7 @@ int oracle_layer_rows(const uint16_t* x, const uint16_t* w_router, const uint16_
       for (int c = 0; c < d; ++c) acc += xd[c] * bf16_to_double(w_router[(int64_t)j * d + c]);
       l[j] = (float)acc;
     }
-    int k = route_one(l, N, K, eps, mode, renorm, ids, gates, NULL, NULL, NULL, NULL);
+    int k = route_one(l, N, K, eps, mode, renorm, ids, gates, NULL, NULL, NULL, NULL, NULL, NULL);
     double* yr = y + r * d;
     for (int c = 0; c < d; ++c) yr[c] = 0.0;
     for (int s = 0; s < k; ++s) {

@@ -238,6 +238,51 @@ def test_flat_and_degenerate():
 
 
 # ----------------------------------------------- load balance (App. A.3)
+def _tree_sum_f32(v):
+    """The balanced tree sum of R6 in fp32: v_i += v_{i+h}, h = N/2 .. 1."""
+    v = np.array(v, dtype=np.float32)
+    h = v.shape[-1] // 2
+    while h >= 1:
+        v[..., :h] = v[..., :h] + v[..., h:2 * h]
+        h //= 2
+    return v[..., 0]
+
+
+@pytest.mark.parametrize("N", [64, 128])
+def test_printed_quotients_rounded_once(N):
+    """Every quotient of the printed formulas is the correctly rounded fp32
+    quotient: p_j = e_j / s (the softmax of Sec. 2) and p'_i = (p_(i) - p_min) /
+    den (Alg. 1's normalisation). An fp64 quotient of two fp32 numbers rounded
+    to fp32 is the correctly rounded fp32 quotient (53 >= 2 * 24 + 2 bits, so
+    the double rounding is innocuous: Figueroa, 1995), which a product with a
+    rounded reciprocal is not in general. D_i = (1 - p'_i) - x'_i, each
+    difference rounded once."""
+    rng = np.random.default_rng(700 + N)
+    T = 96
+    lg = np.concatenate([synth.boosted_logits(rng, T // 2, N),
+                         rng.standard_normal((T // 2, N)).astype(np.float32)])
+    cur = oracle.elbow_curve(lg, eps=1e-8)
+    f32, f64 = np.float32, np.float64
+    m = lg.max(axis=1, keepdims=True)
+    e = oracle.exp((lg - m).astype(np.float32))
+    s = _tree_sum_f32(e)
+    p = (e.astype(f64) / s[:, None].astype(f64)).astype(f32)
+    assert np.array_equal(np.sort(p, axis=1)[:, ::-1], cur["p"])
+    sp = cur["p"]
+    pmin = sp[:, -1:]
+    den = (f32(sp[:, :1] - pmin) + f32(1e-8)).astype(f32)
+    a = (sp - pmin).astype(f32)
+    pn = (a.astype(f64) / den.astype(f64)).astype(f32)
+    assert np.array_equal(pn, cur["pn"])
+    x = (np.arange(N, dtype=f32) / f32(N - 1)).astype(f32)
+    D = ((f32(1.0) - pn).astype(f32) - x).astype(f32)
+    assert np.array_equal(D, cur["D"])
+    # the reading matters: the reciprocal products differ from the quotients
+    # in some of these values, so the check above can tell the two apart
+    p_rcp = (e * (f32(1.0) / s)[:, None]).astype(f32)
+    assert np.count_nonzero(p_rcp != p) > 0
+
+
 def test_theorem1_and_corollaries():
     """Theorem 1 and Corollaries 1-2 hold exactly on the empirical loads of any
     batch, and q_elb - q_top = delta/(1-delta) (q_top - r) (the proof's identity)."""
@@ -317,8 +362,8 @@ def test_elbow_angle_vs_atan2(N):
     for t in range(500):
         sp = r["sorted_p"][t]
         e = int(a["elbow"][t])
-        inv = f(1) / (f(sp[0] - sp[-1]) + f(1e-8))
-        pn = f(f(sp[e] - sp[-1]) * inv)
+        den = f(f(sp[0] - sp[-1]) + f(1e-8))
+        pn = f(np.float64(f(sp[e] - sp[-1])) / np.float64(den))
         x = float(f(e) / f(N - 1))
         y = 1.0 - float(pn)
         a1 = np.arctan2(-y, -x)

@@ -21,7 +21,12 @@ MUTANTS = [
     ("deviation_sign_as_printed",  # Alg. 1 as printed: D = p' - x' (always k = 1)
      "float D = (1.0f - pn) - xn;", "float D = pn - xn;"),
     ("normalisation_drops_p_min",
-     "float pn = (p[idx[i]] - p_min) * inv;", "float pn = p[idx[i]] * inv;"),
+     "float pn = (p[idx[i]] - p_min) / den;", "float pn = p[idx[i]] / den;"),
+    ("normalisation_reciprocal_multiply",  # two roundings instead of Alg. 1's one quotient
+     "float pn = (p[idx[i]] - p_min) / den;", "float pn = (p[idx[i]] - p_min) * (1.0f / den);"),
+    ("softmax_reciprocal_multiply",
+     "for (int j = 0; j < N; ++j) p[j] = e[j] / s;",
+     "for (int j = 0; j < N; ++j) p[j] = e[j] * (1.0f / s);"),
     ("x_over_n_not_n_minus_1",
      "float xn = (float)i / (float)(N - 1);", "float xn = (float)i / (float)N;"),
     ("argmax_takes_last_tie",
