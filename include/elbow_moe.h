@@ -85,8 +85,9 @@ const char* moe_status_string(moe_status s);
  * fp32 specification (every operation rounded to nearest even, no
  * contraction): m = max_j l_j; e_j = EXP(l_j - m) with EXP the library's
  * Cody-Waite/Taylor exponential (zero below 2^-126); s = balanced tree sum
- * (v_i += v_{i+h}, h = N/2 .. 1); p_j = e_j * (1/s); sort p descending;
- * den = (p_max - p_min) + eps; p'_i = (p_(i) - p_min) * (1/den);
+ * (v_i += v_{i+h}, h = N/2 .. 1); p_j = e_j / s; sort p descending;
+ * den = (p_max - p_min) + eps; p'_i = (p_(i) - p_min) / den (both quotients
+ * correctly rounded, as the printed formulas divide);
  * x'_i = i/(N-1); D_i = (1 - p'_i) - x'_i (the deviation below the chord of
  * the descending curve; Alg. 1 prints the sign reversed, which would give
  * k = 1 always); e = smallest argmax_i D_i. Logits must be finite.
@@ -338,6 +339,17 @@ moe_status moe_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_
 moe_status elbow_route_randomized(const float* logits, int64_t T, int N, const moe_route_params* rp,
                                   const uint32_t* rand, int32_t* k_out, int32_t* ids_out,
                                   float* gates_out, void* stream);
+
+/* Self-check of the quotients the routing divides with (the softmax
+ * p_j = e_j / s of Sec. 2 and Alg. 1's normalisation p'_i = (p_(i) - p_min) /
+ * den, each a correctly rounded quotient): for i < n, out[3i] = the routing's
+ * quotient a_i / b_i (one reciprocal per divisor, then Markstein's fused
+ * multiply-add correction), out[3i + 1] = the same from the packed two-lane
+ * form, out[3i + 2] = CUDA's __fdiv_rn(a_i, b_i). All three must be equal for
+ * a_i >= 0 and b_i in [2^-32, 2^8]. a, b [n] and out [3n] fp32 device arrays,
+ * 4-byte aligned; 0 <= n <= 2^30 (else MOE_ERR_INVALID_ARG). */
+moe_status moe_check_quotients(const float* a, const float* b, int64_t n, float* out,
+                               void* stream);
 
 /* Exercises the bounded wait that every GEMM pipeline uses, on an mbarrier
  * that nothing arrives on: the kernel gives up after `seconds` (0 < seconds

@@ -18,7 +18,7 @@ import threading
 import numpy as np
 
 __all__ = [
-    "MODE_ELBOW", "MODE_TOPK", "MoeError", "library", "build", "route_diagnostics", "RouteDiag", "check_bounded_wait", "elbow_route_warp",
+    "MODE_ELBOW", "MODE_TOPK", "MoeError", "library", "build", "route_diagnostics", "RouteDiag", "check_bounded_wait", "check_quotients", "elbow_route_warp",
     "elbow_route_randomized", "MODE_RAND_TAIL", "MODE_RAND_HEAD",
     "elbow_route", "moe_dispatch", "moe_dispatch_noalloc", "dispatch_workspace_size", "layer_workspace_size",
     "moe_layer_forward", "read_device_error", "router_logits", "gather_rows",
@@ -87,6 +87,7 @@ def library():
             "moe_dispatch": ([P, P, i64, i32, i32, P, P, P, P, sz, P], i32),
             "moe_dispatch_tile_offsets": ([P, i64, i32, i32], P),
             "moe_dispatch_noalloc": ([P, P, i64, i32, i32, P, P, P, P], i32),
+            "moe_check_quotients": ([P, P, i64, P, P], i32),
             "moe_dispatch_chunk_counts": ([P, i64, i32, i32], P),
             "moe_dispatch_counted": ([P, P, i64, i32, i32, P, P, P, P, sz, P], i32),
             "moe_layer_workspace_size": ([i64, i32, i32, i32, i32], sz),
@@ -229,6 +230,20 @@ def elbow_route_randomized(logits, rand, K: int = 8, eps: float = 1e-8, mode: in
                                             _p(rand), _p(k), _p(ids), _p(gates), _stream(stream)),
            "elbow_route_randomized")
     return k, ids, gates
+
+
+def check_quotients(a, b, stream=None):
+    """The routing's correctly rounded quotients a / b on the device: returns
+    [n, 3] fp32 = (scalar form, packed two-lane form, CUDA's __fdiv_rn)."""
+    torch = _torch()
+    _cuda(a, torch.float32, "a")
+    _cuda(b, torch.float32, "b")
+    if a.numel() != b.numel():
+        raise ValueError("a and b must have the same size")
+    out = torch.empty(a.numel(), 3, dtype=torch.float32, device=a.device)
+    _check(library().moe_check_quotients(_p(a), _p(b), a.numel(), _p(out), _stream(stream)),
+           "moe_check_quotients")
+    return out
 
 
 def check_bounded_wait(err, seconds: float = 0.2, stream=None) -> int:

@@ -55,6 +55,8 @@ cudaError_t launch_router_small_route(const uint16_t* x, const uint16_t* w_route
                                       int N, float* partial, unsigned int* ticket, int K, float eps,
                                       int topk_mode, int renorm, float* logits_out, int32_t* k_out,
                                       int32_t* ids_out, float* gates_out, cudaStream_t stream);
+cudaError_t launch_quotient_check(const float* a, const float* b, int64_t n, float* out,
+                                  cudaStream_t stream);
 cudaError_t launch_route_diagnostics(const float* logits, int64_t T, int N, int K, float eps,
                                      int32_t* elbow_out, float* theta_out, moe_route_diag* dg,
                                      cudaStream_t stream);
@@ -420,6 +422,14 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   e = moe::launch_combine(w.o, kk, w.pair_pos, gates, residual, T, d, K, y, nsm, s);
   if (e != cudaSuccess) return MOE_ERR_CUDA;
   return MOE_OK;
+}
+
+moe_status moe_check_quotients(const float* a, const float* b, int64_t n, float* out,
+                               void* stream) {
+  if (n < 0 || n > (int64_t(1) << 30)) return MOE_ERR_INVALID_ARG;
+  if (n == 0) return MOE_OK;
+  if (!a || !b || !out || !aligned4(a) || !aligned4(b) || !aligned4(out)) return MOE_ERR_INVALID_ARG;
+  return cuda_status(moe::launch_quotient_check(a, b, n, out, static_cast<cudaStream_t>(stream)));
 }
 
 moe_status moe_check_bounded_wait(int32_t* err_word, double seconds, void* stream) {

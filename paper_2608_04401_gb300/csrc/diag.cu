@@ -61,16 +61,17 @@ __global__ void __launch_bounds__(kTok) diag_kernel(
   if (tid < ntok) {
     float* row = tile + tid * kPitch;
     float emin;
-    const float r = route::softmax_row<N>(row, emin);
+    const route::Softmax sm = route::softmax_row<N>(row, emin);
     float v[N];
-    route::sorted_probs<N>(row, r, v);
+    route::sorted_probs<N>(row, sm, v);
     const float p_min = v[N - 1];
-    const float inv = __frcp_rn(__fadd_rn(__fsub_rn(v[0], p_min), eps));
+    const float den = __fadd_rn(__fsub_rn(v[0], p_min), eps);
+    const float yd = __frcp_rn(den);
     float best = 0.0f, pn_e = 0.0f;
     int e = 0;
 #pragma unroll
     for (int i = 0; i < N; ++i) {
-      const float pn = __fmul_rn(__fsub_rn(v[i], p_min), inv);
+      const float pn = route::quot(__fsub_rn(v[i], p_min), den, yd);
       const float D = __fsub_rn(__fsub_rn(1.0f, pn), rc.x[i]);
       if (i == 0 || D > best) {
         best = D;
@@ -85,7 +86,7 @@ __global__ void __launch_bounds__(kTok) diag_kernel(
     if (theta_out) theta_out[t] = th;
     const int k = min(e + 1, K);
     int ids[8];
-    route::topk_ids<N>(row, r, v, K, keys, tid, ids);
+    route::topk_ids<N>(row, sm, v, K, keys, tid, ids);
     atomicAdd(&h_k[k], 1);
     atomicAdd(&h_e[e], 1);
     atomicAdd(&h_th[min(kThetaBins - 1, max(0, static_cast<int>(floorf(th))))], 1);

@@ -557,17 +557,17 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
         }
         int ids_sel[8];
         int k_sel = 0;
-        float rs = 0.0f;
+        float ssum = 0.0f;
         if (valid)
           k_sel = route::route_token<BN, RouteX>(row, grow, args.K, args.eps, args.topk_mode,
                                                  args.renorm, args.rx, args.k_out, args.ids_out,
-                                                 args.gates_out, ids_sel, rs);
+                                                 args.gates_out, ids_sel, ssum);
         // tokens the fast path left undecided: routed by their whole warp
         const unsigned undecided = __ballot_sync(0xffffffffu, valid && k_sel < 0);
         if constexpr (BN >= 64) if (undecided) {
           const float* wrow = rtile + q * 32 * (BN + 4);
           route::route_undecided<BN>(
-              undecided, [&](int l) { return wrow + l * (BN + 4); }, rs, grow, args.K, args.eps,
+              undecided, [&](int l) { return wrow + l * (BN + 4); }, ssum, grow, args.K, args.eps,
               args.topk_mode, args.renorm, args.k_out, args.ids_out, args.gates_out, k_sel,
               ids_sel);
         }

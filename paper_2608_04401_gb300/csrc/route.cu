@@ -11,7 +11,7 @@ namespace route {
 // keeps ranks k..K-1 and fills slots 0..k-1 with experts of rank >= K. Each
 // draw takes, among the remaining experts in ascending id order, the one at
 // index rand[t, s] mod (number remaining). Gates are the experts' own p (the
-// row holds their e, and 1/s is recomputed with the routing's tree order).
+// row holds their e, and s is recomputed with the routing's tree order).
 template <int N>
 __device__ __noinline__ void randomize_token(const float* row, int64_t t, int K, int mode,
                                              int renorm, int k, const int* top,
@@ -26,7 +26,7 @@ __device__ __noinline__ void randomize_token(const float* row, int64_t t, int K,
   for (int h = N / 2; h >= 1; h /= 2)
 #pragma unroll
     for (int i = 0; i < h; ++i) v[i] = __fadd_rn(v[i], v[i + h]);
-  const float r = __frcp_rn(v[0]);
+  const float sum = v[0], ys = __frcp_rn(sum);
   uint32_t taken[N / 32];
 #pragma unroll
   for (int w = 0; w < N / 32; ++w) taken[w] = 0u;
@@ -57,10 +57,10 @@ __device__ __noinline__ void randomize_token(const float* row, int64_t t, int K,
     --remaining;
   }
   float S = 0.0f;
-  for (int s = 0; s < K; ++s) S = __fadd_rn(S, __fmul_rn(row[ids[s]], r));
+  for (int s = 0; s < K; ++s) S = __fadd_rn(S, quot(row[ids[s]], sum, ys));
   k_out[t] = K;
   for (int s = 0; s < K; ++s) {
-    const float p = __fmul_rn(row[ids[s]], r);
+    const float p = quot(row[ids[s]], sum, ys);
     ids_out[t * K + s] = ids[s];
     gates_out[t * K + s] = renorm ? __fdiv_rn(p, S) : p;
   }
@@ -98,16 +98,16 @@ __global__ void __launch_bounds__(kTok) elbow_route_kernel(
   __syncthreads();
   int ids_sel[8];
   int k_sel = 0;
-  float r = 0.0f;
+  float ssum = 0.0f;
   const bool valid = tid < ntok;
   if (valid)
     k_sel = route_token<N, RouteConsts<N>>(tile + tid * kPitch, t0 + tid, K, eps, topk_mode,
-                                           renorm, rc, k_out, ids_out, gates_out, ids_sel, r);
+                                           renorm, rc, k_out, ids_out, gates_out, ids_sel, ssum);
   // tokens the fast path left undecided: routed by their whole warp
   const unsigned undecided = __ballot_sync(0xffffffffu, valid && k_sel < 0);
   if (undecided) {
     const float* wrow = tile + (tid & ~31) * kPitch;
-    route_undecided<N>(undecided, [&](int l) { return wrow + l * kPitch; }, r, t0 + tid, K, eps,
+    route_undecided<N>(undecided, [&](int l) { return wrow + l * kPitch; }, ssum, t0 + tid, K, eps,
                        topk_mode, renorm, k_out, ids_out, gates_out, k_sel, ids_sel);
   }
   if (valid) {
@@ -154,7 +154,30 @@ cudaError_t launch(const float* logits, int64_t T, int K, float eps, int topk_mo
   return cudaGetLastError();
 }
 
+// Self-check of the routing's quotients: out[3i .. 3i+2] = quot(a, b), the
+// packed quot2 (both numerators of a pair at once; only where both qualify),
+// and CUDA's __fdiv_rn, for a_i >= 0 and b_i in [2^-32, 2^8].
+__global__ void quotient_check_kernel(const float* __restrict__ a, const float* __restrict__ b,
+                                      int64_t n, float* __restrict__ out) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const float ai = a[i], bi = b[i], y = __frcp_rn(bi);
+  const bool fast = ai == 0.0f || ai >= kQuotMin;
+  const uint64_t q2 = quot2(pk(ai, fast ? ai : 0.0f), pk(-bi, -bi), pk(y, y));
+  out[3 * i] = quot(ai, bi, y);
+  out[3 * i + 1] = fast ? lo_of(q2) : __fdiv_rn(ai, bi);
+  out[3 * i + 2] = __fdiv_rn(ai, bi);
+}
+
 }  // namespace route
+
+cudaError_t launch_quotient_check(const float* a, const float* b, int64_t n, float* out,
+                                  cudaStream_t stream) {
+  if (n == 0) return cudaSuccess;
+  const int64_t blocks = (n + 255) / 256;
+  route::quotient_check_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(a, b, n, out);
+  return cudaGetLastError();
+}
 
 // blk_cnt (nullable): per-128-token-chunk expert counts, [N][ceil(T/128)].
 // rand (nullable) and rand_mode (0, or 2 / 3 for the tail / head randomisation).

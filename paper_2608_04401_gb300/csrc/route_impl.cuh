@@ -5,9 +5,10 @@
 // each thread's row reads are bank-conflict free). Each thread keeps its
 // token's values in registers and evaluates, in fp32 with every operation
 // rounded to nearest even (explicit .rn intrinsics / PTX, no contraction):
-//   m = max_j l_j; e_j = EXP(l_j - m); s = balanced tree sum; p_j = e_j * (1/s)
-//   sort p descending; p' = (p_(i) - p_min) * (1 / ((p_max - p_min) + eps));
+//   m = max_j l_j; e_j = EXP(l_j - m); s = balanced tree sum; p_j = e_j / s
+//   sort p descending; p' = (p_(i) - p_min) / ((p_max - p_min) + eps);
 //   x' = i / (N-1); D_i = (1 - p'_i) - x'_i; e = smallest argmax; k = min(e+1, K)
+// Each quotient is the correctly rounded one (quot / quot2 below).
 //
 // Fast path. The elbow decision only needs the exact curve at the top ranks:
 // for every rank i, D_i <= fl(1 - x'_i), so ranks i >= kTop - 1 cannot beat a
@@ -20,7 +21,7 @@
 //   M_head >= M_mid and M_head >= bound  ->  k = argmax + 1
 //   M_mid > M_head                        ->  k = K (the elbow lies at or past K-1)
 //   otherwise, or when a check fails      ->  undecided (rare)
-// Sorting is by e, not p; p = fl(e * (1/s)) is monotone in e, so the curve is
+// Sorting is by e, not p; p = fl(e / s) is monotone in e, so the curve is
 // the same, and ids inside groups of equal p are re-ordered by ascending id.
 // A p tie across the K boundary also leaves the token undecided.
 //
@@ -100,6 +101,41 @@ MOE_DEV float min3f(float a, float b, float c) {
   float r;
   asm("min.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
   return r;
+}
+
+// -------------------------------------------- correctly rounded quotients
+// The softmax p_j = e_j / s and Alg. 1's p'_i = (p_(i) - p_min) / den are
+// quotients rounded once. With y = RN(1/b) taken once per divisor b, each
+// quotient a / b costs a product and four fused multiply-adds (Markstein's
+// correction, IBM J. Res. Dev. 34(1), 1990):
+//   q0 = RN(a y)                 within 2 ulp of a / b
+//   q1 = RN(q0 + RN(a - b q0) y) within 1 ulp (a neighbour of a / b)
+//   r  = a - b q1                exact in one fma
+//   q  = RN(q1 + r y)            = RN(a / b)
+// The last step's rounding cannot differ from RN(a / b): q1 + r y differs from
+// a / b by (a / b - q1)(b y - 1), |b y - 1| <= B 2^-48 for the 24-bit
+// significand B of b, while a / b lies at least 2^-24 ulp / B from any
+// midpoint between floats (and never on one). Valid for a == 0 or
+// a >= kQuotMin with b in [2^-32, 2^8] (no step underflows); other
+// numerators take __fdiv_rn, which gives the same correctly rounded quotient.
+constexpr float kQuotMin = 0x1p-90f;
+MOE_DEV float quot(float a, float b, float y) {
+  if (a != 0.0f && a < kQuotMin) return __fdiv_rn(a, b);
+  float q = __fmul_rn(a, y);
+  float r = __fmaf_rn(-q, b, a);
+  q = __fmaf_rn(r, y, q);
+  r = __fmaf_rn(-q, b, a);
+  return __fmaf_rn(r, y, q);
+}
+// Two quotients at once with packed operations: a = (a0, a1), nb = (-b, -b),
+// y = (RN(1/b), RN(1/b)). The caller guarantees that both numerators are 0 or
+// at least kQuotMin.
+MOE_DEV uint64_t quot2(uint64_t a, uint64_t nb, uint64_t y) {
+  uint64_t q = mul2(a, y);
+  uint64_t r = fma2(q, nb, a);
+  q = fma2(r, y, q);
+  r = fma2(q, nb, a);
+  return fma2(r, y, q);
 }
 
 // EXP of two arguments z <= 0 at once with packed fp32 operations. z is
@@ -314,11 +350,21 @@ MOE_DEV void write_outputs(int64_t t, int K, int k, const int (&ids)[8], const f
   }
 }
 
+// The softmax sum s of a token and what its quotients e_j / s need: y = RN(1/s)
+// (for quot / quot2), and `regular`: every logit lies within 40 of the maximum,
+// so that every e_j >= EXP(-40) > 2^-58, every p_j > 2^-65, and every nonzero
+// difference p_(i) - p_min is at least an ulp of p_min (> 2^-88): every
+// numerator the routing divides is then 0 or at least kQuotMin.
+struct Softmax {
+  float s, y;
+  bool regular;
+};
+
 // Softmax numerators of one token: e_j = EXP(l_j - m) for the N logits in
-// row, written back into the row; the smallest e_j in emin; returns r = 1/s
-// with s the balanced tree sum of the e_j.
+// row, written back into the row; the smallest e_j in emin; returns the sum s
+// (the balanced tree sum of the e_j) with y = RN(1/s).
 template <int N>
-MOE_DEV float softmax_row(float* row, float& emin) {
+MOE_DEV Softmax softmax_row(float* row, float& emin) {
   float m, lmin;
   {
     float l[N];
@@ -357,7 +403,8 @@ MOE_DEV float softmax_row(float* row, float& emin) {
           make_float4(lo_of(e2), hi_of(e2), lo_of(e3), hi_of(e3));
     }
   };
-  if (__fsub_rn(lmin, m) >= -87.0f)
+  const float zmin = __fsub_rn(lmin, m);
+  if (zmin >= -87.0f)
     exp_pass([](uint64_t z) { return exp_spec2_inrange(z); });
   else
     exp_pass([](uint64_t z) { return exp_spec2(z); });
@@ -376,17 +423,21 @@ MOE_DEV float softmax_row(float* row, float& emin) {
     emin = fminf(min3f(acc[0], acc[1], acc[2]), acc[3]);
   }
   tree_sum_level2<N / 2>(ep);
-  return __frcp_rn(__fadd_rn(lo_of(ep[0]), hi_of(ep[0])));
+  Softmax sm;
+  sm.s = __fadd_rn(lo_of(ep[0]), hi_of(ep[0]));
+  sm.y = __frcp_rn(sm.s);
+  sm.regular = zmin >= -40.0f;
+  return sm;
 }
 
-// v = all N probabilities p_j = e_j * r (row holds the e_j), sorted descending.
+// v = all N probabilities p_j = e_j / s (row holds the e_j), sorted descending.
 template <int N>
-MOE_DEV void sorted_probs(const float* row, float r, float (&v)[N]) {
+MOE_DEV void sorted_probs(const float* row, const Softmax& sm, float (&v)[N]) {
 #pragma unroll
   for (int c = 0; c < N; c += 4) {
     const float4 q = *reinterpret_cast<const float4*>(row + c);
-    v[c] = __fmul_rn(q.x, r); v[c + 1] = __fmul_rn(q.y, r);
-    v[c + 2] = __fmul_rn(q.z, r); v[c + 3] = __fmul_rn(q.w, r);
+    v[c] = quot(q.x, sm.s, sm.y); v[c + 1] = quot(q.y, sm.s, sm.y);
+    v[c + 2] = quot(q.z, sm.s, sm.y); v[c + 3] = quot(q.w, sm.s, sm.y);
   }
   sort_desc_at<N, 0>(v);
 }
@@ -397,8 +448,8 @@ MOE_DEV void sorted_probs(const float* row, float r, float (&v)[N]) {
 // taken, and the equal ones in ascending id until K are taken. The (p, id)
 // keys go through this thread's 8-byte slots keys[s * kTok + tid].
 template <int N>
-MOE_DEV void topk_ids(const float* row, float r, const float (&v)[N], int K, uint64_t* keys,
-                      int tid, int (&ids)[8]) {
+MOE_DEV void topk_ids(const float* row, const Softmax& sm, const float (&v)[N], int K,
+                      uint64_t* keys, int tid, int (&ids)[8]) {
   float thr = v[0];
 #pragma unroll
   for (int s = 1; s < 8; ++s)
@@ -412,7 +463,8 @@ MOE_DEV void topk_ids(const float* row, float r, const float (&v)[N], int K, uin
 #pragma unroll
   for (int c = 0; c < N; c += 4) {
     const float4 q = *reinterpret_cast<const float4*>(row + c);
-    const float pq[4] = {__fmul_rn(q.x, r), __fmul_rn(q.y, r), __fmul_rn(q.z, r), __fmul_rn(q.w, r)};
+    const float pq[4] = {quot(q.x, sm.s, sm.y), quot(q.y, sm.s, sm.y), quot(q.z, sm.s, sm.y),
+                         quot(q.w, sm.s, sm.y)};
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       const float pj = pq[u];
@@ -435,14 +487,14 @@ MOE_DEV void topk_ids(const float* row, float r, const float (&v)[N], int K, uin
 }
 
 // Routes token t with the calling (whole, converged) warp from the token's
-// softmax numerators e (lane l holds experts l + 32c in e[c]) and r = 1/s,
-// in the routing specification's arithmetic: p_j = e_j * r; a bitonic sort of
+// softmax numerators e (lane l holds experts l + 32c in e[c]) and their sum s,
+// in the routing specification's arithmetic: p_j = e_j / s; a bitonic sort of
 // the N keys (p bits << 32 | ~id) across the warp, which orders by p
 // descending and ascending id on ties; p'_i and D_i on every rank; the first
 // argmax by a (max D, min index) warp reduction; k = min(e + 1, K). Writes the
 // token's outputs; returns k, and lane s < K gets the id of rank s in sel_id.
 template <int N>
-MOE_DEV int warp_route_from_e(const float (&e)[N / 32], float r, int64_t t, int K, float eps,
+MOE_DEV int warp_route_from_e(const float (&e)[N / 32], float s, int64_t t, int K, float eps,
                               int topk_mode, int renorm, int32_t* __restrict__ k_out,
                               int32_t* __restrict__ ids_out, float* __restrict__ gates_out,
                               int& sel_id) {
@@ -450,9 +502,10 @@ MOE_DEV int warp_route_from_e(const float (&e)[N / 32], float r, int64_t t, int 
   const unsigned full = 0xffffffffu;
   const int lane = threadIdx.x & 31;
   uint64_t key[C];
+  const float ys = __frcp_rn(s);
 #pragma unroll
   for (int c = 0; c < C; ++c) {
-    const float p = __fmul_rn(e[c], r);
+    const float p = quot(e[c], s, ys);
     key[c] = (static_cast<uint64_t>(__float_as_uint(p)) << 32) |
              static_cast<uint32_t>(~(32 * c + lane));
   }
@@ -481,14 +534,15 @@ MOE_DEV int warp_route_from_e(const float (&e)[N / 32], float r, int64_t t, int 
   const float pmax = __uint_as_float(static_cast<uint32_t>(__shfl_sync(full, key[0], 0) >> 32));
   const float pmin =
       __uint_as_float(static_cast<uint32_t>(__shfl_sync(full, key[C - 1], 31) >> 32));
-  const float inv = __frcp_rn(__fadd_rn(__fsub_rn(pmax, pmin), eps));
+  const float den = __fadd_rn(__fsub_rn(pmax, pmin), eps);
+  const float yd = __frcp_rn(den);
   float best = 0.0f;
   int bi = 0;
 #pragma unroll
   for (int c = 0; c < C; ++c) {
     const int i = 32 * c + lane;
     const float p = __uint_as_float(static_cast<uint32_t>(key[c] >> 32));
-    const float pn = __fmul_rn(__fsub_rn(p, pmin), inv);
+    const float pn = quot(__fsub_rn(p, pmin), den, yd);
     const float xi = __fdiv_rn(static_cast<float>(i), static_cast<float>(N - 1));
     const float D = __fsub_rn(__fsub_rn(1.0f, pn), xi);
     if (c == 0 || D > best) {
@@ -527,12 +581,12 @@ MOE_DEV int warp_route_from_e(const float (&e)[N / 32], float r, int64_t t, int 
 }
 
 // The tokens of this warp that route_token left undecided (lane l's bit in
-// `undecided`; its softmax numerators in row_of(l)[0 .. N), its 1/s in r,
+// `undecided`; its softmax numerators in row_of(l)[0 .. N), their sum in s,
 // its token index in t) are routed one after another by the whole warp;
 // their lanes receive k in k_sel and the selected ids in ids_sel. Every lane
 // of the warp must call this.
 template <int N, typename RowOf>
-MOE_DEV void route_undecided(unsigned undecided, RowOf row_of, float r, int64_t t, int K,
+MOE_DEV void route_undecided(unsigned undecided, RowOf row_of, float s, int64_t t, int K,
                              float eps, int topk_mode, int renorm, int32_t* __restrict__ k_out,
                              int32_t* __restrict__ ids_out, float* __restrict__ gates_out,
                              int& k_sel, int (&ids_sel)[8]) {
@@ -545,7 +599,7 @@ MOE_DEV void route_undecided(unsigned undecided, RowOf row_of, float r, int64_t 
     float e[N / 32];
 #pragma unroll
     for (int c = 0; c < N / 32; ++c) e[c] = srow[32 * c + lane];
-    const float rs = __shfl_sync(full, r, src);
+    const float rs = __shfl_sync(full, s, src);
     const int64_t ts = __shfl_sync(full, t, src);
     int sel = 0;
     const int kf = warp_route_from_e<N>(e, rs, ts, K, eps, topk_mode, renorm, k_out, ids_out,
@@ -562,17 +616,17 @@ MOE_DEV void route_undecided(unsigned undecided, RowOf row_of, float r, int64_t 
 // Routes the token of this thread (its logits are in `row`): writes its
 // outputs and returns k, with the selected ids in ids_sel; or, when the fast
 // path cannot settle the token, returns -1 and writes nothing (the row then
-// holds the softmax numerators and r_out = 1/s, for route_undecided).
+// holds the softmax numerators and s_out = s, for route_undecided).
 template <int N, typename RC>
 MOE_DEV int route_token(float* row, int64_t t, int K, float eps, int topk_mode, int renorm,
                         const RC& rc, int32_t* __restrict__ k_out, int32_t* __restrict__ ids_out,
-                        float* __restrict__ gates_out, int (&ids_sel)[8], float& r_out) {
+                        float* __restrict__ gates_out, int (&ids_sel)[8], float& s_out) {
   constexpr uint32_t kIdMask = N - 1;
 
-  // ---- e_j = EXP(l_j - m), stored back into the row; e_min; s; r = 1/s
+  // ---- e_j = EXP(l_j - m), stored back into the row; e_min; s; RN(1/s)
   float emin;
-  const float r = softmax_row<N>(row, emin);
-  r_out = r;
+  const Softmax sm = softmax_row<N>(row, emin);
+  s_out = sm.s;
 
   // ---- the kTop largest e, each key = truncated value | (N-1 - id): one
   // 32-key network (a loop, not unrolled, so its code is fetched once) sorts
@@ -611,25 +665,34 @@ MOE_DEV int route_token(float* row, int64_t t, int K, float eps, int topk_mode, 
 #pragma unroll
   for (int i = 0; i + 1 < kTop - 1; ++i) ok = ok && (ev[i] >= ev[i + 1]);
 
-  // ---- probabilities of the top ranks, elbow decision
+  // ---- probabilities of the top ranks: correctly rounded quotients e / s
+  // (rows with a logit more than 40 below their maximum are left to the warp
+  // path, which checks each numerator)
+  ok = ok && sm.regular;
   float pv[kTop];
-  const uint64_t rr = pk(r, r);
+  {
+    const uint64_t ys = pk(sm.y, sm.y), ns = pk(-sm.s, -sm.s);
 #pragma unroll
-  for (int i = 0; i < kTop; i += 2) {
-    const uint64_t q = mul2(pk(ev[i], ev[i + 1]), rr);
-    pv[i] = lo_of(q);
-    pv[i + 1] = hi_of(q);
+    for (int i = 0; i < kTop; i += 2) {
+      const uint64_t q = quot2(pk(ev[i], ev[i + 1]), ns, ys);
+      pv[i] = lo_of(q);
+      pv[i + 1] = hi_of(q);
+    }
   }
+  // ---- elbow decision
   int k = K;
   if (ok && !topk_mode) {
-    const float p_min = __fmul_rn(emin, r);
-    const float inv = __frcp_rn(__fadd_rn(__fsub_rn(pv[0], p_min), eps));
-    const uint64_t pmin2 = pk(p_min, p_min), inv2 = pk(inv, inv), one2 = pk(1.0f, 1.0f);
+    const float p_min = quot(emin, sm.s, sm.y);
+    const float den = __fadd_rn(__fsub_rn(pv[0], p_min), eps);
+    const float yd = __frcp_rn(den);
+    const uint64_t pmin2 = pk(p_min, p_min), nden2 = pk(-den, -den), yd2 = pk(yd, yd),
+                   one2 = pk(1.0f, 1.0f);
     float best = -__int_as_float(0x7f800000), mid = -__int_as_float(0x7f800000);
     int e = 0;
 #pragma unroll
     for (int i = 0; i < kTop; i += 2) {
-      const uint64_t pn = mul2(sub2(pk(pv[i], pv[i + 1]), pmin2), inv2);
+      // p'_i = (p_(i) - p_min) / den; D_i = (1 - p'_i) - x'_i
+      const uint64_t pn = quot2(sub2(pk(pv[i], pv[i + 1]), pmin2), nden2, yd2);
       const uint64_t D2 = sub2(sub2(one2, pn), pk(rc.x[i], rc.x[i + 1]));
       const float D[2] = {lo_of(D2), hi_of(D2)};
 #pragma unroll

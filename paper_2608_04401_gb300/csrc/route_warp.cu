@@ -6,7 +6,7 @@
 // bits as the thread-per-token kernels and the oracle:
 //   m = max l (warp reduction); e_j = EXP(l_j - m) (the packed spec
 //   exponential); s = balanced tree sum (levels h >= 32 inside the lane, then
-//   v_i += v_{i+h} by shuffles); p_j = e_j * (1/s);
+//   v_i += v_{i+h} by shuffles); p_j = e_j / s (correctly rounded);
 //   a bitonic sort of the N keys (p bits << 32 | ~id) across the warp (64-bit
 //   shuffles), which orders by p descending and ascending id on ties;
 //   p'_i, D_i on each rank, the first argmax by a (max D, min index) warp
@@ -147,10 +147,10 @@ MOE_DEV void route_one_warp(const float* __restrict__ row, int64_t t, int K, flo
     const float o = __shfl_down_sync(full, v0, h);
     if (lane < h) v0 = __fadd_rn(v0, o);
   }
-  const float r = __frcp_rn(__shfl_sync(full, v0, 0));
+  const float s = __shfl_sync(full, v0, 0);
 
   int sel_id;
-  route::warp_route_from_e<N>(e, r, t, K, eps, topk_mode, renorm, k_out, ids_out, gates_out,
+  route::warp_route_from_e<N>(e, s, t, K, eps, topk_mode, renorm, k_out, ids_out, gates_out,
                               sel_id);
 }
 

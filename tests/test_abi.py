@@ -142,3 +142,11 @@ def test_misaligned_int32_arrays_are_rejected(lib):
     ws = lib.moe_layer_workspace_size(64, 2048, 64, 1024, 8)
     assert lib.moe_layer_forward(fake, fake, fake, fake, 64, 2048, 64, 1024, _rp(), None, fake,
                                  None, odd, None, None, None, fake, ws, None) == 1
+
+
+def test_quotient_check_validation(lib):
+    fake = ctypes.c_void_p(256)
+    assert lib.moe_check_quotients(fake, fake, 0, fake, None) == 0
+    assert lib.moe_check_quotients(fake, fake, -1, fake, None) == 1
+    assert lib.moe_check_quotients(None, fake, 4, fake, None) == 1
+    assert lib.moe_check_quotients(fake, ctypes.c_void_p(258), 4, fake, None) == 1
