@@ -284,8 +284,9 @@ def run_ours(args, rank, world, local, pg):
     kern["gate_up"].update(tflops=gu_tf, frac=gu_tf / pk["bf16"])
     kern["down"].update(tflops=dn_tf, frac=dn_tf / pk["bf16"])
 
-    route = route_stress(moe, args, stream, dev, pk, cpu=rank == 0 and not args.no_cpu_baseline)
-    others = other_configs(moe, args, stream, dev, pk, pg)
+    cpu_leg = rank == 0 and not args.no_cpu_baseline
+    route = route_stress(moe, args, stream, dev, pk, cpu=cpu_leg)
+    others = other_configs(moe, args, stream, dev, pk, pg, cpu=cpu_leg)
 
     # end to end through the public API with host buffers: every step copies
     # its tokens in from pinned host memory and its outputs back out
@@ -345,9 +346,34 @@ def run_ours(args, rank, world, local, pg):
         "gpu_launches": KERNELS_PER_STEP * args.steps,
         "clocks": clocks,
     }
-    if rank == 0 and not args.no_cpu_baseline:
+    if cpu_leg:
+        out["routing"].update(k_flips(inp, it, K))
         out["cpu_baseline"] = cpu_baseline(inp, K)
     return out
+
+
+def k_flips(inp, it, K):
+    """The logit-induced flip fraction of the headline batch (CPU leg, after the
+    timed region): the oracle routes the GPU's fp32 logits and its own
+    fp64-accumulated logits of the same bf16 inputs; a token flips when its k or
+    its ids differ. Also whether the GPU's k, ids and gates are the oracle's
+    bits on the GPU's logits (every token)."""
+    import oracle
+    lg_gpu = it["logits"].cpu().numpy()
+    r_gpu = oracle.route(lg_gpu, K=K)
+    r_ora = oracle.route(oracle.router_logits(inp["x"], inp["w_router"]), K=K)
+    k_gpu, ids_gpu = it["k"].cpu().numpy(), it["ids"].cpu().numpy()
+    bitexact = bool(np.array_equal(r_gpu["k"], k_gpu) and np.array_equal(r_gpu["ids"], ids_gpu) and
+                    np.array_equal(r_gpu["gates"].view(np.uint32),
+                                   it["gates"].cpu().numpy().view(np.uint32)))
+    kf = r_gpu["k"] != r_ora["k"]
+    flip = kf | np.any(r_gpu["ids"] != r_ora["ids"], axis=1)
+    T = len(k_gpu)
+    return {"k_flip_frac": float(flip.mean()), "k_flip_tokens": int(flip.sum()),
+            "k_only_flip_tokens": int(kf.sum()), "tokens_compared": T,
+            "routing_bitexact_on_gpu_logits": bitexact,
+            "k_flip_note": "oracle routing of the GPU's fp32 logits vs of its fp64-accumulated "
+                           "logits, all tokens (k or ids differ)"}
 
 
 def kernel_breakdown(moe, x, wr, wgu, wd, T, d, N, I, K, args, stream, dev):
@@ -511,10 +537,12 @@ def time_layer_modes(moe, x, wr, wgu, wd, K, steps, stream, pg, residual=None):
     return out
 
 
-def other_configs(moe, args, stream, dev, pk, pg):
+def other_configs(moe, args, stream, dev, pk, pg, cpu=False):
     """The small (64-token), wide-router (N = 128) and 16-layer-stack workloads,
     timed with the same kernels in elbow and fixed top-8 mode. Expert weights
-    are drawn on the device; tokens and routers follow the synthetic recipe."""
+    are drawn on the device; tokens and routers follow the synthetic recipe.
+    With cpu (the CPU leg, after the timed regions): the stack's free-running
+    difference against an oracle-only chain on sampled tokens."""
     import torch
     from paper_2608_04401_gb300 import synth
     res = {}
@@ -577,23 +605,54 @@ def other_configs(moe, args, stream, dev, pk, pg):
         out[name] = time_steps(stack, max(5, steps // 4), stream, pg)
         out[name + "_graph"] = graph_ms(stack, max(5, steps // 4), stream, pg)
     moe.read_device_error(ws)
-    mean_k = []
+    mean_k, routed = [], []
     cur = x0
     for l, (wr, wgu, wd) in enumerate(layers):
         nxt = bufs[l % 2]
         _, it = moe.moe_layer_forward(cur, wr, wgu, wd, K=K, residual=cur, y=nxt, ws=ws,
                                       return_intermediates=True)
         mean_k.append(round(float(it["k"].float().mean().item()), 3))
+        routed.append((it["k"].cpu().numpy(), it["ids"].cpu().numpy()))
         cur = nxt
+    free = stack_free_running(x0_bits, routers, layers, routed, cur, K) if cpu else None
     res["stack16_t4k"] = {
         "workload": f"{L} layers, T={T}, d_model={d}, N={N}, I={I}, K={K}, residual add",
         "elbow_ms": out["elbow"], "topk_ms": out["topk"], "elbow_speedup": out["topk"] / out["elbow"],
         "elbow_graph_ms": out["elbow_graph"], "topk_graph_ms": out["topk_graph"],
         "tokens_per_s": T / (out["elbow"] * 1e-3), "mean_k_per_layer": mean_k,
+        "free_running_vs_oracle": free,
     }
     del layers
     torch.cuda.empty_cache()
     return res
+
+
+def stack_free_running(x0_bits, routers, layers, routed, x_last, K, n=64, seed=17):
+    """Reported, not gated: the GPU's 16-layer chain against an oracle-only
+    chain (each oracle layer fed the oracle's own previous output, rounded to
+    bf16 as the GPU stores it) on n sampled tokens: relative Frobenius and
+    relative max difference of the last layer's output, and the tokens whose
+    routing differed somewhere along the chain."""
+    import oracle
+    import torch
+    from paper_2608_04401_gb300 import synth
+    T = x0_bits.shape[0]
+    rows = np.sort(np.random.default_rng(seed).choice(T, n, replace=False))
+    xs = np.ascontiguousarray(x0_bits[rows])
+    host = lambda t: t.view(torch.int16).cpu().numpy().view(np.uint16)
+    diverged = np.zeros(n, bool)
+    for l, (wr, wgu, wd) in enumerate(layers):
+        ref = oracle.layer_rows(xs, routers[l], host(wgu), host(wd), K=K, residual_bits=xs)
+        k_l, ids_l = routed[l]
+        diverged |= (k_l[rows] != ref["k"]) | np.any(ids_l[rows] != ref["ids"], axis=1)
+        xs = synth.bf16_bits(ref["y"].astype(np.float32))
+    got = x_last.float().cpu().numpy().astype(np.float64)[rows]
+    want = synth.bf16_bits_to_f32(xs).astype(np.float64)
+    return {"tokens": n, "layers": len(layers),
+            "rel_fro": float(np.linalg.norm(got - want) / np.linalg.norm(want)),
+            "rel_max": float(np.abs(got - want).max() / np.abs(want).max()),
+            "tokens_routed_differently": int(diverged.sum()),
+            "note": "GPU chain vs oracle-only chain from the same x_0, final layer output"}
 
 
 def route_stress(moe, args, stream, dev, pk, cpu=False):

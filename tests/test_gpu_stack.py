@@ -1,21 +1,27 @@
-"""GPU parity of a stack of OLMoE-shaped MoE layers with the residual add
-between layers (x_{l+1} = bf16(x_l + MoE_l(x_l)), no attention), the 16-layer
-stack's shapes at T = 4096 with its first three layers.
+"""GPU parity of the 16-layer stack of OLMoE-shaped MoE layers with the
+residual add between layers (x_{l+1} = bf16(x_l + MoE_l(x_l)), no attention),
+at the stack workload's shapes (T = 4096, d = 2048, N = 64, I = 1024, K = 8).
 
 Teacher-forced per layer: the oracle gets the GPU's own bf16 input x_l of
-layer l and is compared with the GPU's x_{l+1} on sampled tokens, within the
-layer tolerance (tokens whose elbow decision flips between the GPU's fp32
-logits and the oracle's fp64 logits are counted and left out). The
-free-running difference against an oracle-only chain is not gated."""
+layer l. For every layer, every token's routing on the oracle's fp64 logits is
+compared with the GPU's (the flips over all 16 x 4096 token-layers are bounded
+like the single layer's, <= 1e-3), the layer's routing is bit-exact on its own
+fp32 logits, and the outputs x_{l+1} of 256 sampled tokens are compared with
+the oracle within the layer tolerance (tokens whose routing flips are left
+out). The free-running difference against an oracle-only chain is reported by
+the benchmark, not gated here."""
 import numpy as np
 import pytest
 
 import oracle
 from paper_2608_04401_gb300 import synth
 
-from gpu_util import assert_layer_close, to_dev, to_dev_bf16
+from gpu_util import assert_layer_close, to_dev_bf16
 
 pytestmark = pytest.mark.gpu
+
+SAMPLE = 256
+MAX_FLIP = 1e-3
 
 
 @pytest.fixture(scope="module")
@@ -37,13 +43,11 @@ def _bits(t):
 def test_stack_teacher_forced(moe):
     import torch
     w = synth.WORKLOADS["stack16_t4k"]
-    T, d, N, I, K = w["T"], w["d"], w["N"], w["I"], w["K"]
-    L = 3
+    T, d, N, I, K, L = w["T"], w["d"], w["N"], w["I"], w["K"], w["L"]
     x0, routers = synth.stack_inputs(T, d, N, L, w["seed"])
     ws = torch.empty(moe.layer_workspace_size(T, d, N, I, K), dtype=torch.uint8, device="cuda")
-    rows = np.unique(np.concatenate([[0, T - 1], np.random.default_rng(3).choice(T, 24, replace=False)]))
     cur = to_dev_bf16(x0)
-    mean_k = []
+    mean_k, flips = [], 0
     for l in range(L):
         wgu, wd = synth.expert_weights(synth.stack_expert_seed(w["seed"], l), N, d, I)
         x_in = _bits(cur)
@@ -57,13 +61,19 @@ def test_stack_teacher_forced(moe):
         # the layer's routing is bit-exact on its own fp32 logits
         r = oracle.route(it["logits"].cpu().numpy(), K=K)
         assert np.array_equal(r["k"], got_k) and np.array_equal(r["ids"], got_ids)
-        # teacher-forced output on sampled tokens
+        # every token's routing on the oracle's fp64 logits of the same input
+        ro = oracle.route(oracle.router_logits(x_in, routers[l]), K=K)
+        same_all = (ro["k"] == got_k) & np.all(ro["ids"] == got_ids, axis=1)
+        flips += int(np.count_nonzero(~same_all))
+        # teacher-forced outputs on sampled tokens
+        rows = np.unique(np.concatenate(
+            [[0, T - 1], np.random.default_rng(300 + l).choice(T, SAMPLE, replace=False)]))
         ref = oracle.layer_rows(x_in, routers[l], wgu, wd, rows=rows, K=K, residual_bits=x_in)
         same = (got_k[rows] == ref["k"]) & np.all(got_ids[rows] == ref["ids"], axis=1)
-        assert same.mean() >= 0.9, f"layer {l}: routing flips on {np.count_nonzero(~same)} rows"
         y = nxt.float().cpu().numpy().astype(np.float64)
-        assert_layer_close(y[rows][same], ref["y"][same], f"layer {l}")
-        # the residual path: the output differs from the input only by the MoE term
         assert np.all(np.isfinite(y))
+        assert_layer_close(y[rows][same], ref["y"][same], f"layer {l}")
         cur = nxt
+        del wgu, wd
+    assert flips <= MAX_FLIP * L * T, f"routing flips on {flips} of {L * T} token-layers"
     assert all(1.0 <= m <= K for m in mean_k)
