@@ -21,8 +21,8 @@
  *   - Supported shapes: N (experts) in {64, 128}; 1 <= K <= 8 and K <= N;
  *     0 <= T < 2^28 tokens (T = 0 is a no-op; larger T returns
  *     MOE_ERR_INVALID_ARG, so that the T * K pair counts fit in int32); for
- *     the layer, d_model a multiple of
- *     256 and the SwiGLU intermediate I a multiple of 128, d, I <= 16384.
+ *     the layer, d_model and the SwiGLU intermediate I multiples of 128,
+ *     d, I <= 16384.
  *   - Pointers must be 16-byte aligned.
  *
  * Routing arithmetic is fp32 and fully specified (see elbow_route), so that
@@ -255,7 +255,8 @@ moe_status moe_expert_gate_up(const uint16_t* xs, const uint16_t* w_gate_up, con
 
 /* Expert down projection (the second matrix of the expert MLP, App. A.4):
  * o[r] = W_down[e] h[r] for rows of expert e;
- * h [P, I] bf16 -> o [P, d] bf16. */
+ * h [P, I] bf16 -> o [P, d] bf16. d a multiple of 128 (256-column output
+ * tiles when d is a multiple of 256, else 128-column tiles), I of 64. */
 moe_status moe_expert_down(const uint16_t* h, const uint16_t* w_down, const int32_t* offsets,
                            const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* o,
                            int32_t* err_word, void* stream);
@@ -339,6 +340,19 @@ moe_status moe_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_
 moe_status elbow_route_randomized(const float* logits, int64_t T, int N, const moe_route_params* rp,
                                   const uint32_t* rand, int32_t* k_out, int32_t* ids_out,
                                   float* gates_out, void* stream);
+
+/* Bounds-check report of the debug build (the library compiled with
+ * -DELBOW_MOE_DEBUG, paper_2608_04401_gb300.buildlib.build(debug=True), which
+ * stands in for compute-sanitizer; no counterpart in the paper). In that build
+ * every index a kernel takes from its inputs (k_t <= K, expert ids < N,
+ * expert offsets and m-tile offsets consistent and within the row capacity,
+ * permutation entries and token rows within [0, T), pair positions within
+ * [0, T * K), finite logits) is checked on the device; a failed check counts
+ * one violation and the kernel goes on with the clamp or skip of the release
+ * build (it never traps). This call SYNCHRONISES the device, writes the
+ * number of violations counted since the previous call into *out and resets
+ * the count. Release build: *out = 0 and MOE_ERR_UNSUPPORTED. */
+moe_status moe_debug_violations(uint32_t* out);
 
 /* Self-check of the quotients the routing divides with (the softmax
  * p_j = e_j / s of Sec. 2 and Alg. 1's normalisation p'_i = (p_(i) - p_min) /

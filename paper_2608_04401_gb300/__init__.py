@@ -29,7 +29,10 @@ MODE_ELBOW = 0
 MODE_TOPK = 1
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_LIB_PATH = os.path.join(_HERE, "_lib", "libelbow_moe.so")
+# ELBOW_MOE_DEBUG=1 in the environment loads the bounds-checked debug build
+# (build(debug=True)) instead of the release library
+_DEBUG = os.environ.get("ELBOW_MOE_DEBUG", "") == "1"
+_LIB_PATH = os.path.join(_HERE, "_lib", "debug" if _DEBUG else "", "libelbow_moe.so")
 _lock = threading.Lock()
 _lib = None
 
@@ -58,10 +61,19 @@ class RouteDiag(ctypes.Structure):
                 ("cv_change_pct", ctypes.c_double)]
 
 
-def build(force: bool = False) -> str:
-    """Compile libelbow_moe.so in-tree (nvcc, sm_103a)."""
+def build(force: bool = False, debug: bool = None) -> str:
+    """Compile libelbow_moe.so in-tree (nvcc, sm_103a); debug (default: as
+    ELBOW_MOE_DEBUG says) builds the bounds-checked library."""
     from . import buildlib
-    return buildlib.build(force=force)
+    return buildlib.build(force=force, debug=_DEBUG if debug is None else debug)
+
+
+def debug_violations() -> int:
+    """Debug build only: synchronises the device and returns (and resets) the
+    number of failed device bounds checks since the last call."""
+    v = ctypes.c_uint32(0)
+    _check(library().moe_debug_violations(ctypes.byref(v)), "moe_debug_violations")
+    return int(v.value)
 
 
 def library():
@@ -88,6 +100,7 @@ def library():
             "moe_dispatch_tile_offsets": ([P, i64, i32, i32], P),
             "moe_dispatch_noalloc": ([P, P, i64, i32, i32, P, P, P, P], i32),
             "moe_check_quotients": ([P, P, i64, P, P], i32),
+            "moe_debug_violations": ([P], i32),
             "moe_dispatch_chunk_counts": ([P, i64, i32, i32], P),
             "moe_dispatch_counted": ([P, P, i64, i32, i32, P, P, P, P, sz, P], i32),
             "moe_layer_workspace_size": ([i64, i32, i32, i32, i32], sz),

@@ -60,6 +60,13 @@ cudaError_t launch_quotient_check(const float* a, const float* b, int64_t n, flo
 cudaError_t launch_route_diagnostics(const float* logits, int64_t T, int N, int K, float eps,
                                      int32_t* elbow_out, float* theta_out, moe_route_diag* dg,
                                      cudaStream_t stream);
+#ifdef ELBOW_MOE_DEBUG
+cudaError_t debug_take_route(unsigned int* out);
+cudaError_t debug_take_route_warp(unsigned int* out);
+cudaError_t debug_take_dispatch(unsigned int* out);
+cudaError_t debug_take_gemm(unsigned int* out);
+cudaError_t debug_take_diag(unsigned int* out);
+#endif
 }  // namespace moe
 
 namespace {
@@ -348,7 +355,7 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
                              int32_t* offsets_out, void* ws, size_t ws_bytes, void* stream) {
   if (T < 0 || T > kMaxTokens) return MOE_ERR_INVALID_ARG;
   if (!supported_n(N)) return MOE_ERR_UNSUPPORTED;
-  if (d <= 0 || d > kMaxDim || d % 256 != 0 || I <= 0 || I > kMaxDim || I % 128 != 0)
+  if (d <= 0 || d > kMaxDim || d % 128 != 0 || I <= 0 || I > kMaxDim || I % 128 != 0)
     return MOE_ERR_UNSUPPORTED;
   moe_status st = check_route_params(rp, N);
   if (st != MOE_OK) return st;
@@ -424,6 +431,25 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   return MOE_OK;
 }
 
+moe_status moe_debug_violations(uint32_t* out) {
+  if (!out) return MOE_ERR_INVALID_ARG;
+  *out = 0;
+#ifdef ELBOW_MOE_DEBUG
+  if (cudaDeviceSynchronize() != cudaSuccess) return MOE_ERR_CUDA;
+  unsigned int total = 0;
+  for (auto take : {moe::debug_take_route, moe::debug_take_route_warp, moe::debug_take_dispatch,
+                    moe::debug_take_gemm, moe::debug_take_diag}) {
+    unsigned int v = 0;
+    if (take(&v) != cudaSuccess) return MOE_ERR_CUDA;
+    total += v;
+  }
+  *out = total;
+  return MOE_OK;
+#else
+  return MOE_ERR_UNSUPPORTED;
+#endif
+}
+
 moe_status moe_check_quotients(const float* a, const float* b, int64_t n, float* out,
                                void* stream) {
   if (n < 0 || n > (int64_t(1) << 30)) return MOE_ERR_INVALID_ARG;
@@ -485,7 +511,7 @@ moe_status moe_expert_down(const uint16_t* h, const uint16_t* w_down, const int3
                            const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* o,
                            int32_t* err_word, void* stream) {
   if (P < 0 || P > kMaxTokens * 8) return MOE_ERR_INVALID_ARG;
-  if (!supported_n(N) || d <= 0 || d > kMaxDim || d % 256 != 0 || I <= 0 || I > kMaxDim ||
+  if (!supported_n(N) || d <= 0 || d > kMaxDim || d % 128 != 0 || I <= 0 || I > kMaxDim ||
       I % 64 != 0)
     return MOE_ERR_UNSUPPORTED;
   if (P == 0) return MOE_OK;

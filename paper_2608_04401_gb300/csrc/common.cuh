@@ -71,6 +71,37 @@ inline cudaError_t once_per_device(std::atomic<uint64_t>& done, SetUp set_up) {
   return e;
 }
 
+// ------------------------------------------------------- debug bounds checks
+// The debug build (-DELBOW_MOE_DEBUG) stands in for compute-sanitizer: every
+// index the kernels take from their inputs (expert offsets, permutation
+// entries, pair positions, token ids, tile rows) is checked against its array
+// with MOE_DCHECK. A failed check adds one to this translation unit's device
+// counter and the kernel goes on with the clamp or skip that the release
+// build also applies (no trap, no out-of-bounds access). moe_debug_violations
+// reads and clears the counters of all translation units. In the release
+// build MOE_DCHECK compiles to nothing.
+#ifdef ELBOW_MOE_DEBUG
+static __device__ unsigned int g_debug_violations;
+#define MOE_DCHECK(cond)                                        \
+  do {                                                          \
+    if (!(cond)) atomicAdd(&g_debug_violations, 1u);            \
+  } while (0)
+// Host: this translation unit's count, then cleared.
+#define MOE_DEBUG_TU(name)                                                         \
+  cudaError_t debug_take_##name(unsigned int* out) {                               \
+    unsigned int v = 0, zero = 0;                                                  \
+    cudaError_t e = cudaMemcpyFromSymbol(&v, g_debug_violations, sizeof v);        \
+    if (e == cudaSuccess) e = cudaMemcpyToSymbol(g_debug_violations, &zero, sizeof zero); \
+    *out = v;                                                                      \
+    return e;                                                                      \
+  }
+#else
+#define MOE_DCHECK(cond) \
+  do {                   \
+  } while (0)
+#define MOE_DEBUG_TU(name)
+#endif
+
 MOE_DEV uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }

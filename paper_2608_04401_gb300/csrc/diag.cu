@@ -184,4 +184,6 @@ cudaError_t launch_route_diagnostics(const float* logits, int64_t T, int N, int 
   return diag::launch<128>(logits, T, K, eps, elbow_out, theta_out, dg, stream);
 }
 
+MOE_DEBUG_TU(diag)
+
 }  // namespace moe

@@ -32,6 +32,7 @@ MOE_DEV void load_selection(const int32_t* __restrict__ k, const int32_t* __rest
                             int64_t t, bool valid, int K, int& kt, int (&my)[8], uint64_t& m0,
                             uint64_t& m1) {
   kt = valid ? min(k[t], K) : 0;
+  MOE_DCHECK(!valid || (k[t] >= 0 && k[t] <= K));
   if (valid && K == 8) {
     const int4 a = reinterpret_cast<const int4*>(ids + t * 8)[0];
     const int4 b = reinterpret_cast<const int4*>(ids + t * 8)[1];
@@ -45,6 +46,7 @@ MOE_DEV void load_selection(const int32_t* __restrict__ k, const int32_t* __rest
   m1 = 0;
 #pragma unroll
   for (int s = 0; s < 8; ++s) {
+    MOE_DCHECK(s >= kt || static_cast<unsigned>(my[s]) < static_cast<unsigned>(N));
     if (s < kt && static_cast<unsigned>(my[s]) < static_cast<unsigned>(N)) {
       if (my[s] < 64) m0 |= 1ull << my[s];
       else m1 |= 1ull << (my[s] - 64);
@@ -91,6 +93,7 @@ __global__ void __launch_bounds__(kChunk) count_kernel(const int32_t* __restrict
   const int64_t t = static_cast<int64_t>(blockIdx.x) * kChunk + threadIdx.x;
   const bool valid = t < T;
   const int kt = valid ? min(k[t], K) : 0;
+  MOE_DCHECK(!valid || (k[t] >= 0 && k[t] <= K));
   int my[8];
   if (valid && K == 8) {
     const int4 a = reinterpret_cast<const int4*>(ids + t * 8)[0];
@@ -103,8 +106,10 @@ __global__ void __launch_bounds__(kChunk) count_kernel(const int32_t* __restrict
   }
   __syncthreads();
 #pragma unroll
-  for (int s = 0; s < 8; ++s)
+  for (int s = 0; s < 8; ++s) {
+    MOE_DCHECK(s >= kt || static_cast<unsigned>(my[s]) < static_cast<unsigned>(N));
     if (s < kt && static_cast<unsigned>(my[s]) < static_cast<unsigned>(N)) atomicAdd(&hist[my[s]], 1);
+  }
   __syncthreads();
   for (int e = threadIdx.x; e < N; e += kChunk)
     cnt[static_cast<int64_t>(e) * nblk + blockIdx.x] = hist[e];
@@ -222,6 +227,7 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
       if (offsets_copy) offsets_copy[tid] = off;
     }
     if (tid == 0) {
+      MOE_DCHECK(total_pairs >= 0 && static_cast<int64_t>(total_pairs) <= T * K);
       offsets[N] = total_pairs;
       tile_off[N] = total_tiles;
       if (offsets_copy) offsets_copy[N] = total_pairs;
@@ -299,6 +305,7 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
     for (int i = tid; i < chunk_pairs; i += kChunk) {
       const int pos = s_gpos[i];
       // positions stay below T*K when the counts match the ids
+      MOE_DCHECK(pos >= 0 && static_cast<int64_t>(pos) < T * K);
       if (pos >= 0 && static_cast<int64_t>(pos) < T * K) perm[pos] = s_tok[i];
     }
   }
@@ -322,9 +329,11 @@ __global__ void __launch_bounds__(256) gather_kernel(const uint4* __restrict__ x
                                                      uint4* __restrict__ xs) {
   const int64_t total = min_of<int64_t>(offsets[N], P);
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  MOE_DCHECK(offsets[N] >= 0 && offsets[N] <= P);
   for (int64_t r = static_cast<int64_t>(blockIdx.x) * 8 + warp; r < total;
        r += static_cast<int64_t>(gridDim.x) * 8) {
     const int64_t pt = perm[r];
+    MOE_DCHECK(pt >= 0 && pt < T);
     const int64_t t = pt < 0 ? 0 : (pt >= T ? T - 1 : pt);
     const uint4* src = x + t * d8;
     uint4* dst = xs + r * d8;
@@ -394,6 +403,9 @@ __global__ void __launch_bounds__(32 * kCombineWarps) combine_kernel(
     m.s0 = SPLIT ? static_cast<int>(u % nslab) * C::kSlabChunks : 0;
     m.s1 = SPLIT ? m.s0 + C::kSlabChunks : d8;
     m.kt = min(k[m.t], K);
+    MOE_DCHECK(k[m.t] >= 0 && k[m.t] <= K);
+    MOE_DCHECK(lane >= m.kt || (pair_pos[m.t * K + lane] >= 0 &&
+                                static_cast<int64_t>(pair_pos[m.t * K + lane]) < cap));
     m.pos = lane < m.kt ? static_cast<int>(min_of<int64_t>(max(pair_pos[m.t * K + lane], 0), cap - 1))
                         : 0;
     m.g = lane < m.kt ? gates[m.t * K + lane] : 0.0f;
@@ -501,6 +513,8 @@ __global__ void __launch_bounds__(32 * kCombineWarps) combine_kernel(
 }
 
 }  // namespace disp
+
+MOE_DEBUG_TU(dispatch)
 
 static int num_chunks(int64_t T) { return static_cast<int>((T + disp::kChunk - 1) / disp::kChunk); }
 

@@ -160,6 +160,7 @@ MOE_DEV Tile decode(int tile, const Args& a, const int* s_off, const int* s_toff
     t.nb = tile % a.n_tiles;
     t.row0 = s_off[t.g];
     t.rows = s_off[t.g + 1] - t.row0;
+    MOE_DCHECK(t.rows >= 0 && t.row0 >= 0 && static_cast<int64_t>(t.row0) + t.rows <= a.p_rows);
     // rows stay inside [0, P) whatever the offsets say
     t.rows = (t.row0 < 0 || t.row0 >= a.p_rows)
                  ? 0
@@ -178,6 +179,9 @@ MOE_DEV Tile decode(int tile, const Args& a, const int* s_off, const int* s_toff
   t.nb = local / mt;
   t.row0 = s_off[lo] + mb * BM;
   t.rows = min(BM, s_off[lo + 1] - t.row0);
+  MOE_DCHECK(s_off[lo + 1] >= s_off[lo] && t.row0 >= 0 &&
+             static_cast<int64_t>(t.row0) + t.rows <= a.p_rows);
+  MOE_DCHECK(mt == (s_off[lo + 1] - s_off[lo] + BM - 1) / BM);
   // rows stay inside [0, P) whatever the offsets say
   t.rows = (t.row0 < 0 || t.row0 >= a.p_rows)
                ? 0
@@ -348,6 +352,7 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
         // rows past the expert's end (never stored) repeat its first token; a
         // tile left without rows reads token 0
         int tok = t.rows > 0 ? args.perm[t.row0 + (r < t.rows ? r : 0)] : 0;
+        MOE_DCHECK(tok >= 0 && tok < args.m_rows);
         tok = min(max(tok, 0), static_cast<int>(args.m_rows - 1));
         roff[i] = static_cast<int64_t>(tok) * args.lda + chunk * 8;
       }
@@ -781,6 +786,8 @@ static cudaError_t launch_mode(const CUtensorMap& a, const CUtensorMap& b, const
 
 }  // namespace gemm
 
+MOE_DEBUG_TU(gemm)
+
 // logits[T, N] = x[T, d] W_r[N, d]^T
 cudaError_t launch_router_gemm(const uint16_t* x, const uint16_t* wr, int64_t T, int d, int N,
                                float* logits, int32_t* err, int num_sms, cudaStream_t stream) {
@@ -898,15 +905,19 @@ cudaError_t launch_down_gemm(const uint16_t* h, const uint16_t* wd, const int32_
                              int32_t* err, int num_sms, cudaStream_t stream) {
   using namespace gemm;
   if (P == 0) return cudaSuccess;
+  // d a multiple of 256: 256-column output tiles; otherwise (d a multiple of
+  // 128) 128-column tiles
+  const int bn = d % 256 == 0 ? 256 : 128;
   CUtensorMap ma, mb;
-  if (!make_map(&ma, h, I, P, BM) || !make_map(&mb, wd, I, static_cast<uint64_t>(N) * d, 256))
+  if (!make_map(&ma, h, I, P, BM) ||
+      !make_map(&mb, wd, I, static_cast<uint64_t>(N) * d, static_cast<uint32_t>(bn)))
     return cudaErrorInvalidValue;
   Args a{};
   a.offsets = offsets;
   a.tile_off = tile_off;
   a.groups = N;
   a.p_rows = P;
-  a.n_tiles = d / 256;
+  a.n_tiles = d / bn;
   a.k_blocks = I / BK;
   a.b_rows = d;
   a.out = o;
@@ -914,6 +925,7 @@ cudaError_t launch_down_gemm(const uint16_t* h, const uint16_t* wd, const int32_
   a.err = err;
   CUtensorMap mc;  // o [P, d], boxes of 32 x 32, no swizzle (TMA stores)
   if (!make_map_plain(&mc, o, d, P, 32, 32)) return cudaErrorInvalidValue;
+  if (bn == 128) return launch_mode<kDown, 128>(ma, mb, mc, a, num_sms, stream);
   return launch_mode<kDown, 256>(ma, mb, mc, a, num_sms, stream);
 }
 

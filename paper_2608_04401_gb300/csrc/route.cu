@@ -193,4 +193,6 @@ cudaError_t launch_elbow_route(const float* logits, int64_t T, int N, int K, flo
                             blk_cnt, rand, rand_mode, stream);
 }
 
+MOE_DEBUG_TU(route)
+
 }  // namespace moe

@@ -384,6 +384,8 @@ MOE_DEV Softmax softmax_row(float* row, float& emin) {
     m = fmaxf(max3f(acc[0], acc[1], acc[2]), acc[3]);
     lmin = fminf(min3f(acn[0], acn[1], acn[2]), acn[3]);
   }
+  // the specification needs finite logits
+  MOE_DCHECK(isfinite(m) && isfinite(lmin));
   const uint64_t mm = pk(m, m);
   // e_j = EXP(l_j - m), eight at a time in place in the row; the loop is not
   // unrolled, so its code is fetched once instead of N / 8 times. When every

@@ -122,6 +122,7 @@ MOE_DEV void route_one_warp(const float* __restrict__ row, int64_t t, int K, flo
   for (int c = 1; c < C; ++c) m = fmaxf(m, l[c]);
 #pragma unroll
   for (int o = 16; o >= 1; o >>= 1) m = fmaxf(m, __shfl_xor_sync(full, m, o));
+  MOE_DCHECK(isfinite(m));
 
   // e = EXP(l - m) on pairs
   float e[C];
@@ -268,5 +269,7 @@ cudaError_t launch_router_small_route(const uint16_t* x, const uint16_t* w_route
   return launch_pdl(kern, grid, dim3(rwarp::kSmallThreads), 0, stream, xx, ww, T, d, partial, ticket, K,
                     eps, topk_mode, renorm, logits_out, k_out, ids_out, gates_out);
 }
+
+MOE_DEBUG_TU(route_warp)
 
 }  // namespace moe

@@ -88,6 +88,12 @@ def test_layer_validation(lib):
         fake, fake, fake, fake, T, d, N, I, rp or _rp(), None, fake, None, None, None, None, None,
         fake, wsb, None)
     assert lib.moe_layer_forward(*args(d=2000)) == 2
+    # d a multiple of 128 is supported (the check reaches the workspace size);
+    # a multiple of 64 only is not
+    ws384 = lib.moe_layer_workspace_size(64, 384, 64, 1024, 8)
+    assert ws384 > 0
+    assert lib.moe_layer_forward(*args(d=384, wsb=ws384 - 1)) == 3
+    assert lib.moe_layer_forward(*args(d=320)) == 2
     assert lib.moe_layer_forward(*args(I=1000)) == 2
     assert lib.moe_layer_forward(*args(N=32)) == 2
     assert lib.moe_layer_forward(*args(wsb=ws - 1)) == 3
@@ -150,3 +156,10 @@ def test_quotient_check_validation(lib):
     assert lib.moe_check_quotients(fake, fake, -1, fake, None) == 1
     assert lib.moe_check_quotients(None, fake, 4, fake, None) == 1
     assert lib.moe_check_quotients(fake, ctypes.c_void_p(258), 4, fake, None) == 1
+
+
+def test_debug_violations_release_build(lib):
+    """The release build has no device bounds checks: the report says so."""
+    v = ctypes.c_uint32(7)
+    assert lib.moe_debug_violations(ctypes.byref(v)) == 2 and v.value == 0
+    assert lib.moe_debug_violations(None) == 1

@@ -224,3 +224,15 @@ def test_layer_prefill_other_caps(moe, N, K, mode):
     d_ref = oracle.dispatch(got["k"], got["ids"], N)
     assert np.array_equal(d_ref["offsets"], got["offsets"])
     _compare_layer(inp, got, np.arange(T), K=K, mode=mode, max_flip=0.02)
+
+
+@pytest.mark.parametrize("T,mode", [(300, 0), (300, 1), (20, 0)])
+def test_layer_d_multiple_of_128(moe, T, mode):
+    """d = 384 (a multiple of 128, not of 256: the down GEMM's 128-column
+    output tiles), prefill and decode paths, every token against the oracle."""
+    N, d, I = 64, 384, 256
+    inp = synth.layer_inputs(T=T, d=d, N=N, I=I, seed=3300 + T)
+    got = _run_layer(moe, inp, mode=mode)
+    r = oracle.route(got["logits"], K=8, mode=mode)
+    assert np.array_equal(r["k"], got["k"]) and np.array_equal(r["ids"], got["ids"])
+    _compare_layer(inp, got, np.arange(T), mode=mode, max_flip=0.02)
