@@ -48,6 +48,13 @@ cudaError_t launch_gateup_decode_gemm(const uint16_t* xs, const uint16_t* wgu,
 cudaError_t launch_down_decode_gemm(const uint16_t* h, const uint16_t* wd, const int32_t* offsets,
                                     int64_t P, int64_t max_rows, int d, int N, int I, uint16_t* o,
                                     int32_t* err, int num_sms, cudaStream_t stream);
+cudaError_t launch_gateup_gather_gemm_pair(const uint16_t* x, int64_t T, const int32_t* perm,
+                                           const uint16_t* wgu, const int32_t* offsets, int64_t P,
+                                           int d, int N, int I, uint16_t* h, int32_t* err,
+                                           int num_sms, cudaStream_t stream);
+cudaError_t launch_down_gemm_pair(const uint16_t* h, const uint16_t* wd, const int32_t* offsets,
+                                  int64_t P, int d, int N, int I, uint16_t* o, int32_t* err,
+                                  int num_sms, cudaStream_t stream);
 cudaError_t launch_route_warp(const float* logits, int64_t T, int N, int K, float eps,
                               int topk_mode, int renorm, int32_t* k_out, int32_t* ids_out,
                               float* gates_out, cudaStream_t stream);
@@ -65,6 +72,7 @@ cudaError_t debug_take_route(unsigned int* out);
 cudaError_t debug_take_route_warp(unsigned int* out);
 cudaError_t debug_take_dispatch(unsigned int* out);
 cudaError_t debug_take_gemm(unsigned int* out);
+cudaError_t debug_take_gemm2(unsigned int* out);
 cudaError_t debug_take_diag(unsigned int* out);
 #endif
 }  // namespace moe
@@ -123,6 +131,22 @@ int sm_count() {
 }
 
 moe_status cuda_status(cudaError_t e) { return e == cudaSuccess ? MOE_OK : MOE_ERR_CUDA; }
+
+// The prefill expert GEMMs: two-CTA (M = 256) tiles; the down projection needs
+// d a multiple of 256 for them (else one-CTA 128-column tiles).
+cudaError_t gate_up_gathered(const uint16_t* x, int64_t T, const int32_t* perm, const uint16_t* wgu,
+                             const int32_t* offsets, const int32_t* tile_off, int64_t P, int d,
+                             int N, int I, uint16_t* h, int32_t* err, int nsm, cudaStream_t s) {
+  (void)tile_off;  // the two-CTA kernel derives its 256-row tiles from the offsets
+  return moe::launch_gateup_gather_gemm_pair(x, T, perm, wgu, offsets, P, d, N, I, h, err, nsm, s);
+}
+cudaError_t expert_down(const uint16_t* h, const uint16_t* wd, const int32_t* offsets,
+                        const int32_t* tile_off, int64_t P, int d, int N, int I, uint16_t* o,
+                        int32_t* err, int nsm, cudaStream_t s) {
+  if (d % 256 == 0)
+    return moe::launch_down_gemm_pair(h, wd, offsets, P, d, N, I, o, err, nsm, s);
+  return moe::launch_down_gemm(h, wd, offsets, tile_off, P, d, N, I, o, err, nsm, s);
+}
 
 moe_status check_route_params(const moe_route_params* rp, int N) {
   if (!rp) return MOE_ERR_INVALID_ARG;
@@ -420,10 +444,10 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
     if (e != cudaSuccess) return MOE_ERR_CUDA;
     const int32_t* tile_off = moe::dispatch_tile_off(w.disp, T, N);
     // gate/up GEMM gathers its token rows itself (no dispatched copy of x)
-    e = moe::launch_gateup_gather_gemm(x, T, w.perm, w_gate_up, w.offsets, tile_off, P, d, N, I,
-                                       w.h, w.err, nsm, s);
+    e = gate_up_gathered(x, T, w.perm, w_gate_up, w.offsets, tile_off, P, d, N, I, w.h, w.err, nsm,
+                         s);
     if (e != cudaSuccess) return MOE_ERR_CUDA;
-    e = moe::launch_down_gemm(w.h, w_down, w.offsets, tile_off, P, d, N, I, w.o, w.err, nsm, s);
+    e = expert_down(w.h, w_down, w.offsets, tile_off, P, d, N, I, w.o, w.err, nsm, s);
     if (e != cudaSuccess) return MOE_ERR_CUDA;
   }
   e = moe::launch_combine(w.o, kk, w.pair_pos, gates, residual, T, d, K, y, nsm, s);
@@ -438,7 +462,7 @@ moe_status moe_debug_violations(uint32_t* out) {
   if (cudaDeviceSynchronize() != cudaSuccess) return MOE_ERR_CUDA;
   unsigned int total = 0;
   for (auto take : {moe::debug_take_route, moe::debug_take_route_warp, moe::debug_take_dispatch,
-                    moe::debug_take_gemm, moe::debug_take_diag}) {
+                    moe::debug_take_gemm, moe::debug_take_gemm2, moe::debug_take_diag}) {
     unsigned int v = 0;
     if (take(&v) != cudaSuccess) return MOE_ERR_CUDA;
     total += v;
@@ -520,8 +544,8 @@ moe_status moe_expert_down(const uint16_t* h, const uint16_t* w_down, const int3
     return MOE_ERR_INVALID_ARG;
   const int nsm = sm_count();
   if (nsm <= 0) return MOE_ERR_CUDA;
-  return cuda_status(moe::launch_down_gemm(h, w_down, offsets, tile_off, P, d, N, I, o, err_word,
-                                           nsm, static_cast<cudaStream_t>(stream)));
+  return cuda_status(expert_down(h, w_down, offsets, tile_off, P, d, N, I, o, err_word, nsm,
+                                 static_cast<cudaStream_t>(stream)));
 }
 
 moe_status moe_expert_gate_up_decode(const uint16_t* xs, const uint16_t* w_gate_up,
@@ -613,9 +637,8 @@ moe_status moe_expert_gate_up_gathered(const uint16_t* x, int64_t T, const int32
     return MOE_ERR_INVALID_ARG;
   const int nsm = sm_count();
   if (nsm <= 0) return MOE_ERR_CUDA;
-  return cuda_status(moe::launch_gateup_gather_gemm(x, T, perm, w_gate_up, offsets, tile_off, P, d, N,
-                                                    I, h, err_word, nsm,
-                                                    static_cast<cudaStream_t>(stream)));
+  return cuda_status(gate_up_gathered(x, T, perm, w_gate_up, offsets, tile_off, P, d, N, I, h,
+                                      err_word, nsm, static_cast<cudaStream_t>(stream)));
 }
 
 moe_status moe_combine(const uint16_t* o, const int32_t* k, const int32_t* pair_pos,
