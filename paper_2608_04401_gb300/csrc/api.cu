@@ -37,10 +37,6 @@ cudaError_t launch_router_route(const uint16_t* x, const uint16_t* wr, int64_t T
                                 int K, float eps, int topk_mode, int renorm, float* logits_out,
                                 int32_t* k_out, int32_t* ids_out, float* gates_out,
                                 int32_t* blk_cnt, int32_t* err, int num_sms, cudaStream_t stream);
-cudaError_t launch_gateup_gather_gemm(const uint16_t* x, int64_t T, const int32_t* perm,
-                                      const uint16_t* wgu, const int32_t* offsets,
-                                      const int32_t* tile_off, int64_t P, int d, int N, int I,
-                                      uint16_t* h, int32_t* err, int num_sms, cudaStream_t stream);
 cudaError_t launch_gateup_decode_gemm(const uint16_t* xs, const uint16_t* wgu,
                                       const int32_t* offsets, int64_t P, int64_t max_rows, int d,
                                       int N, int I, uint16_t* h, int32_t* err, int num_sms,

@@ -1,5 +1,7 @@
 // Persistent tcgen05 GEMMs with TMA-fed shared-memory pipelines and TMEM
-// accumulators, for the three contractions of the layer:
+// accumulators, one CTA per tile, for the contractions of the layer (the
+// prefill layer's gathered gate/up and down GEMMs use the two-CTA kernels of
+// gemm2.cu; kDown here serves d not a multiple of 256):
 //
 //   kRouter       : logits[T, N] = x[T, d] . W_r[N, d]^T             (fp32 out)
 //   kRouterFused  : the same, with the elbow routing of each token run in the
@@ -8,9 +10,6 @@
 //                   expert counts; the logits need not leave the chip
 //   kGateUp       : h[P, I] = silu(xs W_gate[e]^T) * (xs W_up[e]^T), per expert
 //                   e over its dispatched rows [offsets[e], offsets[e+1]) (bf16)
-//   kGateUpGather : the same, with the A rows gathered from x[T, d] by the
-//                   dispatch permutation (cp.async into the swizzled layout),
-//                   so the dispatched copy of x is never materialised
 //   kDown         : o[P, d] = h W_down[e]^T, per expert                 (bf16 out)
 //   kDecGateUp, kDecDown : the same two expert contractions for decode-sized
 //                   batches (every expert has at most 64 rows), with the roles
@@ -28,7 +27,7 @@
 // halves of the SwiGLU and the epilogue fuses silu(g) * u.
 //
 // Warp roles (192 threads, one CTA per SM):
-//   warp 0     : TMA producer (one elected lane; all 32 lanes for gathers)
+//   warp 0     : TMA producer (one elected lane)
 //   warp 1     : TMEM allocator + MMA issuer (one elected lane)
 //   warps 2..5 : epilogue; warp w reads TMEM lanes [32 (w % 4), +32)
 // Two TMEM accumulators (2 x BN columns) let the epilogue of tile i overlap
@@ -52,7 +51,7 @@ constexpr int BK = 64;
 // Warps: kProdWarps producers, one MMA warp, four epilogue warps.
 template <int MODE>
 struct Roles {
-  static constexpr int kProdWarps = MODE == 3 ? 4 : 1;  // gathered A rows: four copy warps
+  static constexpr int kProdWarps = 1;
   static constexpr int kMmaWarp = kProdWarps;
   static constexpr int kEpiWarp0 = kProdWarps + 1;
   static constexpr int kThreads = 32 * (kProdWarps + 5);
@@ -61,7 +60,6 @@ enum Mode {
   kRouter = 0,
   kGateUp = 1,
   kDown = 2,
-  kGateUpGather = 3,
   kRouterFused = 4,
   kDecGateUp = 5,
   kDecDown = 6
@@ -70,7 +68,7 @@ enum Mode {
 template <int MODE>
 __host__ __device__ constexpr bool is_router() { return MODE == kRouter || MODE == kRouterFused; }
 template <int MODE>
-__host__ __device__ constexpr bool is_gateup() { return MODE == kGateUp || MODE == kGateUpGather; }
+__host__ __device__ constexpr bool is_gateup() { return MODE == kGateUp; }
 template <int MODE>
 __host__ __device__ constexpr bool is_decode() { return MODE == kDecGateUp || MODE == kDecDown; }
 
@@ -115,7 +113,7 @@ struct Args {
   const int32_t* offsets;   // [G + 1] row offsets per group (grouped modes)
   const int32_t* tile_off;  // [G + 1] prefix sums of ceil(rows_g / 128)
   int groups;               // G
-  int64_t m_rows;           // router: T (kGateUpGather: the rows of x)
+  int64_t m_rows;           // router: T
   int64_t p_rows;           // grouped and decode modes: the row capacity P of the
                             // dispatched operand and the output
   int n_tiles;              // n-blocks per group
@@ -125,9 +123,6 @@ struct Args {
   void* out;
   int64_t ldo;              // output row stride, elements
   int32_t* err;             // device error word (may be null)
-  const int32_t* perm;      // kGateUpGather: token of each dispatched row
-  const void* a_src;        // kGateUpGather: x [m_rows, lda] bf16
-  int64_t lda;
   // kRouterFused
   RouteX rx;
   int K, topk_mode, renorm, nblk;
@@ -218,9 +213,7 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
-      // gathered mode: the expect-tx arrival for B plus one arrival per
-      // producer lane for its A copies
-      mbar_init(full_bar(s), MODE == kGateUpGather ? 1 + 32 * R::kProdWarps : 1);
+      mbar_init(full_bar(s), 1);
       mbar_init(empty_bar(s), 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -278,65 +271,7 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
                     : is_decode<MODE>() ? s_toff[C::kMaxGroups] * args.n_tiles
                                         : s_toff[args.groups] * args.n_tiles;
 
-  if (MODE == kGateUpGather && warp < R::kProdWarps) {
-    // --------------------------------------- producers, gathered A rows
-    // A: cp.async, 16 bytes per lane, written straight into the 128B-swizzled
-    // K-major layout (chunk c of row r at r * 128 + ((c ^ (r & 7)) << 4)).
-    // Producer warp w owns rows 32w .. 32w+31; its copy i covers rows
-    // 32w + 4i .. +3 (lane l: row 32w + 4i + (l >> 3), chunk l & 7), four full
-    // 128-byte lines per copy. Each lane then arms an arrival on the stage's
-    // full barrier that fires when its copies have landed
-    // (cp.async.mbarrier.arrive.noinc); the MMA thread fences the async proxy
-    // after its wait. Lane 0 of warp 0 also brings B by TMA.
-    const __nv_bfloat16* xg = static_cast<const __nv_bfloat16*>(args.a_src);
-    const int chunk = lane & 7;
-    int stage = 0;
-    uint32_t phase = 0;
-    int issued = 0;
-    for (int tile = blockIdx.x; tile < total && !*abort_flag; tile += gridDim.x) {
-      const Tile t = decode<MODE>(tile, args, s_off, s_toff);
-      int64_t roff[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const int r = 32 * warp + 4 * i + (lane >> 3);
-        // rows past the expert's end (never stored) repeat its first token; a
-        // tile left without rows reads token 0
-        int tok = t.rows > 0 ? args.perm[t.row0 + (r < t.rows ? r : 0)] : 0;
-        MOE_DCHECK(tok >= 0 && tok < args.m_rows);
-        tok = min(max(tok, 0), static_cast<int>(args.m_rows - 1));
-        roff[i] = static_cast<int64_t>(tok) * args.lda + chunk * 8;
-      }
-      bool ok_tile = true;
-      for (int kb = 0; kb < args.k_blocks; ++kb) {
-        int ok = 1;
-        if (lane == 0) ok = mbar_wait_bounded(empty_bar(stage), phase ^ 1u, abort_flag) ? 1 : 0;
-        ok = __shfl_sync(0xffffffffu, ok, 0);
-        if (!ok) { ok_tile = false; break; }
-        const uint32_t a_dst = sbase + stage * C::kStageBytes;
-        const uint32_t b_dst = a_dst + C::kABytes;
-        if (warp == 0 && lane == 0) {
-          mbar_arrive_expect_tx(full_bar(stage), C::kBBytes);
-          const int brow = t.g * args.b_rows + t.nb * 128;
-          tma_load_2d(b_dst, &tmB, full_bar(stage), kb * BK, brow);
-          tma_load_2d(b_dst + 128 * BK * 2, &tmB, full_bar(stage), kb * BK, brow + args.b_half);
-        }
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const int r = 32 * warp + 4 * i + (lane >> 3);
-          const uint32_t dst = a_dst + r * 128 + ((chunk ^ (r & 7)) << 4);
-          cp_async_16(dst, xg + roff[i] + kb * BK);
-        }
-        cp_async_arrive_noinc(full_bar(stage));
-        ++issued;
-        if (++stage == S) {
-          stage = 0;
-          phase ^= 1u;
-        }
-      }
-      if (!ok_tile) break;
-    }
-    cp_async_wait_group<0>();  // nothing of this thread in flight at exit
-  } else if (warp == 0) {
+  if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       int stage = 0;
@@ -411,8 +346,6 @@ __global__ void __launch_bounds__(Roles<MODE>::kThreads, 1)
         bool ok = true;
         for (int kb = 0; kb < args.k_blocks; ++kb) {
           if (!mbar_wait_bounded(full_bar(stage), phase, abort_flag)) { ok = false; break; }
-          // A rows written by cp.async (generic proxy) are read by the tensor core
-          if (MODE == kGateUpGather) fence_proxy_async_smem();
           tc_fence_after();
           const uint32_t a_addr = sbase + stage * C::kStageBytes;
           const uint64_t adesc = smem_desc_sw128(a_addr);
@@ -792,36 +725,6 @@ cudaError_t launch_router_route(const uint16_t* x, const uint16_t* wr, int64_t T
   const int grid = static_cast<int>(tiles < num_sms ? tiles : num_sms);
   if (N == 64) return launch_mode<kRouterFused, 64>(ma, mb, ma, a, grid, stream);
   return launch_mode<kRouterFused, 128>(ma, mb, ma, a, grid, stream);
-}
-
-// h[P, I] = silu(x[perm] W_g^T) * (x[perm] W_u^T) per expert, rows gathered by TMA
-cudaError_t launch_gateup_gather_gemm(const uint16_t* x, int64_t T, const int32_t* perm,
-                                      const uint16_t* wgu, const int32_t* offsets,
-                                      const int32_t* tile_off, int64_t P, int d, int N, int I,
-                                      uint16_t* h, int32_t* err, int num_sms, cudaStream_t stream) {
-  using namespace gemm;
-  if (P == 0 || T == 0) return cudaSuccess;
-  CUtensorMap ma, mb;
-  if (!make_map(&ma, x, d, T, BM) ||
-      !make_map(&mb, wgu, d, static_cast<uint64_t>(N) * 2 * I, 128))
-    return cudaErrorInvalidValue;
-  Args a{};
-  a.offsets = offsets;
-  a.tile_off = tile_off;
-  a.groups = N;
-  a.p_rows = P;
-  a.n_tiles = I / 128;
-  a.k_blocks = d / BK;
-  a.b_rows = 2 * I;
-  a.b_half = I;
-  a.out = h;
-  a.ldo = I;
-  a.err = err;
-  a.perm = perm;
-  a.m_rows = T;  // gathered token rows are clamped to [0, T)
-  a.a_src = x;
-  a.lda = d;
-  return launch_mode<kGateUpGather, 256>(ma, mb, ma, a, num_sms, stream);
 }
 
 // h[P, I] = silu(xs W_g^T) * (xs W_u^T) per expert
