@@ -514,7 +514,29 @@ def graph_ms(step, steps, stream, pg):
     return time_steps(g.replay, steps, stream, pg)
 
 
-def time_layer_modes(moe, x, wr, wgu, wd, K, steps, stream, pg, residual=None):
+def graph_cold_ms(step, steps, stream):
+    """ms per replay of a CUDA graph of one `step` with L2 flushed before each
+    replay (the weights then come from HBM, as when a model's layers follow one
+    another; the flush is outside the timed events)."""
+    import torch
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for _ in range(2):
+            step()
+    torch.cuda.current_stream().wait_stream(side)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        step()
+    for _ in range(3):
+        g.replay()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    ms = time_flushed(g.replay, steps, stream, flush)
+    del flush
+    return ms
+
+
+def time_layer_modes(moe, x, wr, wgu, wd, K, steps, stream, pg, residual=None, cold=False):
     """ms per moe_layer_forward in elbow and in top-K mode; sum k of the elbow batch."""
     import torch
     T, d = x.shape
@@ -530,6 +552,8 @@ def time_layer_modes(moe, x, wr, wgu, wd, K, steps, stream, pg, residual=None):
             step()
         out[name] = time_steps(step, steps, stream, pg)
         out[name + "_graph"] = graph_ms(step, steps, stream, pg)
+        if cold:
+            out[name + "_graph_cold"] = graph_cold_ms(step, steps, stream)
     moe.read_device_error(ws)
     _, it = moe.moe_layer_forward(x, wr, wgu, wd, K=K, y=y, ws=ws, return_intermediates=True)
     out["sum_k"] = int(it["k"].sum().item())
@@ -572,14 +596,21 @@ def other_configs(moe, args, stream, dev, pk, pg, cpu=False):
             # single-token and 8-token decode steps on the same weights: the
             # elbow's k decides how many experts' weights are streamed at all
             dec = {}
-            for Td in (1, 8):
-                rd = time_layer_modes(moe, x[:Td].contiguous(), wr, wgu, wd, K, steps, stream, pg)
+            for Td in (1, 2, 8):
+                rd = time_layer_modes(moe, x[:Td].contiguous(), wr, wgu, wd, K, steps, stream, pg,
+                                      cold=True)
                 wb = rd["touched"] * 3 * d * I * 2
                 dec[f"T={Td}"] = {"elbow_ms": rd["elbow"], "topk_ms": rd["topk"],
                                   "elbow_graph_ms": rd["elbow_graph"],
                                   "topk_graph_ms": rd["topk_graph"],
+                                  "elbow_graph_cold_ms": rd["elbow_graph_cold"],
+                                  "topk_graph_cold_ms": rd["topk_graph_cold"],
+                                  "note": "graph replays; cold = L2 flushed before each replay "
+                                          "(weights from HBM)",
                                   "experts_touched": rd["touched"], "mean_k": rd["sum_k"] / Td,
-                                  "weight_hbm_frac_graph": wb / (rd["elbow_graph"] * 1e-3) / 1e9 / pk["hbm"]}
+                                  "weight_hbm_frac_graph": wb / (rd["elbow_graph"] * 1e-3) / 1e9 / pk["hbm"],
+                                  "weight_hbm_frac_graph_cold":
+                                      wb / (rd["elbow_graph_cold"] * 1e-3) / 1e9 / pk["hbm"]}
             res[name]["decode"] = dec
         del wgu, wd
         torch.cuda.empty_cache()

@@ -280,6 +280,33 @@ moe_status moe_expert_down_decode(const uint16_t* h, const uint16_t* w_down, con
                                   int64_t T, int64_t P, int d, int N, int I, uint16_t* o,
                                   int32_t* err_word, void* stream);
 
+/* The expert contractions for batches of T <= 4 tokens (the expert MLP of
+ * App. A.4 in the one-token latency regime of Sec. 3) on CUDA cores, which
+ * moe_layer_forward takes by itself for one-token steps (T = 1, d, I <= 4096;
+ * from two tokens on the tensor-core decode tiles are faster): an expert then
+ * has at most T rows, so its contraction is a few matrix-vector products that
+ * spread the expert's weight rows over many blocks. The same results as
+ * moe_expert_gate_up / moe_expert_down within fp32 accumulation (another
+ * summation order), with the token rows read from x [T, d] through perm (row p
+ * of expert e, p in [offsets[e], offsets[e+1]), is token perm[p]; no gathered
+ * copy):
+ *   moe_expert_gate_up_gemv: h [P, I] = silu(W_gate[e] x[perm[p]]) * (W_up[e] x[perm[p]])
+ *   moe_expert_down_gemv:    o [P, d] = W_down[e] h[p]
+ * K bounds the experts with rows (at most min(N, T * K)). T <= 4, d and I
+ * multiples of 8 and at most 4096 (else MOE_ERR_UNSUPPORTED); x, h (for the
+ * down step) and the weights 16-byte aligned. Rows of an expert past T or P
+ * are not computed; tokens outside [0, T) are clamped into it. Each block
+ * brings its weight rows into shared memory with bulk copies whose wait is
+ * bounded: a block that gives up writes a nonzero code into err_word (device
+ * int32, may be NULL) and leaves its outputs unwritten. */
+moe_status moe_expert_gate_up_gemv(const uint16_t* x, int64_t T, const int32_t* perm,
+                                   const int32_t* offsets, const uint16_t* w_gate_up, int64_t P,
+                                   int d, int N, int I, int K, uint16_t* h, int32_t* err_word,
+                                   void* stream);
+moe_status moe_expert_down_gemv(const uint16_t* h, const int32_t* offsets, const uint16_t* w_down,
+                                int64_t T, int64_t P, int d, int N, int I, int K, uint16_t* o,
+                                int32_t* err_word, void* stream);
+
 /* Device pointer, inside a moe_dispatch workspace, of the [N + 1] int32 tile
  * offsets (exclusive prefix sums of ceil(count_e / 128)) that the last
  * moe_dispatch on that workspace wrote. No counterpart in the paper (the

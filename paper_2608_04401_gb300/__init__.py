@@ -117,6 +117,8 @@ def library():
             "moe_expert_gate_up_gathered": ([P, i64, P, P, P, P, i64, i32, i32, i32, P, P, P], i32),
             "moe_expert_gate_up_decode": ([P, P, P, i64, i64, i32, i32, i32, P, P, P], i32),
             "moe_expert_down_decode": ([P, P, P, i64, i64, i32, i32, i32, P, P, P], i32),
+            "moe_expert_gate_up_gemv": ([P, i64, P, P, P, i64, i32, i32, i32, i32, P, P, P], i32),
+            "moe_expert_down_gemv": ([P, P, P, i64, i64, i32, i32, i32, i32, P, P, P], i32),
         }
         for name, (args, res) in sig.items():
             fn = getattr(lib, name)
@@ -498,6 +500,40 @@ def expert_down_decode(h, w_down, offsets, T: int, err=None, stream=None):
     o = torch.empty(max(P, 1), d, dtype=torch.bfloat16, device=h.device)
     _check(library().moe_expert_down_decode(_p(h), _p(w_down), _p(offsets), T, P, d, N, I, _p(o),
                                             _p(err), _stream(stream)), "moe_expert_down_decode")
+    return o
+
+
+def expert_gate_up_gemv(x, perm, w_gate_up, offsets, P: int, K: int = 8, err=None, stream=None):
+    """h [P, I] for batches of T <= 4 tokens (CUDA-core contractions reading x through perm)."""
+    torch = _torch()
+    bf = torch.bfloat16
+    _cuda(x, bf, "x")
+    _cuda(w_gate_up, bf, "w_gate_up")
+    _cuda(perm, torch.int32, "perm")
+    _cuda(offsets, torch.int32, "offsets")
+    T, d = x.shape
+    N, I2, _ = w_gate_up.shape
+    I = I2 // 2
+    h = torch.zeros(max(P, 1), I, dtype=bf, device=x.device)
+    _check(library().moe_expert_gate_up_gemv(_p(x), T, _p(perm), _p(offsets), _p(w_gate_up), P, d,
+                                             N, I, K, _p(h), _p(err), _stream(stream)),
+           "moe_expert_gate_up_gemv")
+    return h
+
+
+def expert_down_gemv(h, w_down, offsets, T: int, K: int = 8, err=None, stream=None):
+    """o [P, d] for batches of T <= 4 tokens (CUDA-core contractions)."""
+    torch = _torch()
+    bf = torch.bfloat16
+    _cuda(h, bf, "h")
+    _cuda(w_down, bf, "w_down")
+    _cuda(offsets, torch.int32, "offsets")
+    P, I = h.shape
+    N, d, _ = w_down.shape
+    o = torch.zeros(P, d, dtype=bf, device=h.device)
+    _check(library().moe_expert_down_gemv(_p(h), _p(offsets), _p(w_down), T, P, d, N, I, K, _p(o),
+                                          _p(err), _stream(stream)),
+           "moe_expert_down_gemv")
     return o
 
 

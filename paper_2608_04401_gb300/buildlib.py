@@ -19,7 +19,7 @@ LIB = os.path.join(OUT_DIR, "libelbow_moe.so")
 # the debug build (device bounds checks, -DELBOW_MOE_DEBUG) goes to its own folder
 DEBUG_DIR = os.path.join(OUT_DIR, "debug")
 DEBUG_LIB = os.path.join(DEBUG_DIR, "libelbow_moe.so")
-SOURCES = ["api.cu", "route.cu", "route_warp.cu", "dispatch.cu", "gemm.cu", "gemm2.cu", "diag.cu"]
+SOURCES = ["api.cu", "route.cu", "route_warp.cu", "dispatch.cu", "gemm.cu", "gemm2.cu", "gemv.cu", "diag.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

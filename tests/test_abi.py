@@ -163,3 +163,19 @@ def test_debug_violations_release_build(lib):
     v = ctypes.c_uint32(7)
     assert lib.moe_debug_violations(ctypes.byref(v)) == 2 and v.value == 0
     assert lib.moe_debug_violations(None) == 1
+
+
+def test_gemv_validation(lib):
+    fake = ctypes.c_void_p(256)
+    # T > 4, d > 4096, N unsupported
+    assert lib.moe_expert_gate_up_gemv(fake, 5, fake, fake, fake, 40, 512, 64, 256, 8, fake, None,
+                                       None) == 2
+    assert lib.moe_expert_gate_up_gemv(fake, 1, fake, fake, fake, 8, 8192, 64, 256, 8, fake, None,
+                                       None) == 2
+    assert lib.moe_expert_down_gemv(fake, fake, fake, 1, 8, 512, 96, 256, 8, fake, None, None) == 2
+    assert lib.moe_expert_down_gemv(fake, fake, fake, 1, 8, 512, 64, 256, 8, ctypes.c_void_p(257),
+                                    None, None) == 1
+    assert lib.moe_expert_down_gemv(fake, fake, fake, 1, 8, 512, 64, 256, 8, fake,
+                                    ctypes.c_void_p(258), None) == 1
+    assert lib.moe_expert_gate_up_gemv(fake, 0, fake, fake, fake, 0, 512, 64, 256, 8, fake, None,
+                                       None) == 0
