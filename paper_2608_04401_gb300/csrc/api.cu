@@ -57,7 +57,9 @@ cudaError_t launch_gate_up_gemv(const uint16_t* x, int64_t T, const int32_t* per
                                 cudaStream_t stream);
 cudaError_t launch_down_gemv(const uint16_t* h, const int32_t* offsets, const uint16_t* wd,
                              int64_t T, int64_t P, int d, int N, int I, int K, uint16_t* o,
-                             int32_t* err, cudaStream_t stream);
+                             int32_t* err, const int32_t* k, const int32_t* pair_pos,
+                             const float* gates, const uint16_t* residual, uint16_t* y,
+                             unsigned int* tickets, cudaStream_t stream);
 cudaError_t launch_route_warp(const float* logits, int64_t T, int N, int K, float eps,
                               int topk_mode, int renorm, int32_t* k_out, int32_t* ids_out,
                               float* gates_out, cudaStream_t stream);
@@ -65,6 +67,11 @@ cudaError_t launch_router_small_route(const uint16_t* x, const uint16_t* w_route
                                       int N, float* partial, unsigned int* ticket, int K, float eps,
                                       int topk_mode, int renorm, float* logits_out, int32_t* k_out,
                                       int32_t* ids_out, float* gates_out, cudaStream_t stream);
+cudaError_t launch_router_one(const uint16_t* x, const uint16_t* w_router, int d, int N, int K,
+                              float eps, int topk_mode, int renorm, float* logits_out,
+                              int32_t* k_out, int32_t* ids_out, float* gates_out, int32_t* offsets,
+                              int32_t* perm, int32_t* pair_pos, int32_t* offsets_copy,
+                              int32_t* clear, int nclear, cudaStream_t stream);
 cudaError_t launch_quotient_check(const float* a, const float* b, int64_t n, float* out,
                                   cudaStream_t stream);
 cudaError_t launch_route_diagnostics(const float* logits, int64_t T, int N, int K, float eps,
@@ -124,6 +131,7 @@ constexpr int64_t kSmallRouterMaxTokens = 64;
 // tensor-core tiles were faster (52.4 against 56.2 us).
 constexpr int64_t kGemvMaxTokens = 4;
 constexpr int64_t kGemvLayerMaxTokens = 1;
+static_assert(kGemvLayerMaxTokens == 1, "the one-token router serves the CUDA-core path");
 constexpr int kGemvMaxDim = 4096;
 constexpr int kSmallRouterSlice = 64;
 
@@ -189,6 +197,7 @@ struct LayerWs {
   uint16_t* h;
   uint16_t* o;
   float* partial;  // decode-sized batches: router partial sums [d/64][T][N]
+  unsigned int* tickets;  // one-token steps: the combine's counters [ceil(d/16)], after err
   size_t bytes;
 };
 
@@ -203,6 +212,7 @@ LayerWs layer_ws(void* base, int64_t T, int d, int N, int I, int K) {
   };
   const size_t P = static_cast<size_t>(T) * K;
   w.err = reinterpret_cast<int32_t*>(take(256));
+  w.tickets = reinterpret_cast<unsigned int*>(take(sizeof(unsigned int) * ((d + 15) / 16)));
   w.k = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * T));
   w.ids = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * P));
   w.gates = reinterpret_cast<float*>(take(sizeof(float) * P));
@@ -413,8 +423,11 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
       return MOE_ERR_INVALID_ARG;
   }
   // clear the device error word (and the small-batch router's four group
-  // tickets beside it), so that a no-op call reads clean
-  if (cudaMemsetAsync(w.err, 0, 8 * sizeof(int32_t), s) != cudaSuccess) return MOE_ERR_CUDA;
+  // tickets beside it), so that a no-op call reads clean; on the one-token
+  // path the router clears it, and the combine's tickets that follow
+  const bool gemv_path = T >= 1 && T <= kGemvLayerMaxTokens && d <= kGemvMaxDim && I <= kGemvMaxDim;
+  if (!gemv_path && cudaMemsetAsync(w.err, 0, 8 * sizeof(int32_t), s) != cudaSuccess)
+    return MOE_ERR_CUDA;
   if (T == 0) return MOE_OK;
 
   int32_t* kk = k_out ? k_out : w.k;
@@ -425,7 +438,16 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   if (nsm <= 0) return MOE_ERR_CUDA;
 
   cudaError_t e;
-  if (T <= kSmallRouterMaxTokens) {
+  if (gemv_path) {
+    // one token: router, routing and dispatch on one cluster, which also
+    // clears the error word and the combine's tickets
+    const int nclear = static_cast<int>((reinterpret_cast<char*>(w.tickets) -
+                                         reinterpret_cast<char*>(w.err)) / sizeof(int32_t)) +
+                       (d + 15) / 16;
+    e = moe::launch_router_one(x, w_router, d, N, K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
+                               rp->renorm, logits_out, kk, ids, gates, w.offsets, w.perm,
+                               w.pair_pos, offsets_out, w.err, nclear, s);
+  } else if (T <= kSmallRouterMaxTokens) {
     // a few tokens: the router GEMM split over d on many SMs, then one warp per
     // token routes (the single-chunk dispatch counts the pairs itself)
     e = moe::launch_router_small_route(x, w_router, static_cast<int>(T), d, N, w.partial,
@@ -440,16 +462,15 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
                                  moe::dispatch_counts(w.disp), w.err, nsm, s);
   }
   if (e != cudaSuccess) return MOE_ERR_CUDA;
-  if (T <= kGemvLayerMaxTokens && d <= kGemvMaxDim && I <= kGemvMaxDim) {
-    // one token: the single-chunk dispatch, then the CUDA-core expert
+  if (gemv_path) {
+    // one token (dispatched by its router): the CUDA-core expert
     // contractions, which read the token row through perm
-    e = moe::launch_dispatch(kk, ids, T, N, K, w.offsets, w.perm, w.pair_pos, w.disp, offsets_out,
-                             true, s);
-    if (e != cudaSuccess) return MOE_ERR_CUDA;
     e = moe::launch_gate_up_gemv(x, T, w.perm, w.offsets, w_gate_up, P, d, N, I, K, w.h, w.err, s);
     if (e != cudaSuccess) return MOE_ERR_CUDA;
-    e = moe::launch_down_gemv(w.h, w.offsets, w_down, T, P, d, N, I, K, w.o, w.err, s);
-    if (e != cudaSuccess) return MOE_ERR_CUDA;
+    // the down projection also combines (its last block per column block)
+    e = moe::launch_down_gemv(w.h, w.offsets, w_down, T, P, d, N, I, K, w.o, w.err, kk, w.pair_pos,
+                              gates, residual, y, w.tickets, s);
+    return e == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
   } else if (T <= kDecodeMaxTokens) {
     // decode-sized: the single-chunk dispatch also gathers the few token rows
     // (into o, which the down GEMM overwrites afterwards); the GEMMs stream
@@ -639,6 +660,7 @@ moe_status moe_expert_down_gemv(const uint16_t* h, const int32_t* offsets, const
       !aligned4(offsets) || (reinterpret_cast<uintptr_t>(o) & 1u) || !aligned4(err_word))
     return MOE_ERR_INVALID_ARG;
   return cuda_status(moe::launch_down_gemv(h, offsets, w_down, T, P, d, N, I, K, o, err_word,
+                                           nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
                                            static_cast<cudaStream_t>(stream)));
 }
 

@@ -56,6 +56,27 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
   return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
 
+// launch_pdl for a kernel launched in clusters of cluster_x CTAs (along x).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_cluster_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                                      cudaStream_t stream, unsigned cluster_x, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cluster_x;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 // One-time per-device set-up (a kernel attribute), safe under concurrent host
 // threads: `done` holds one bit per device ordinal below 64; ordinals past 63
 // simply repeat the set-up. Returns the set-up's error, or cudaSuccess.
@@ -166,6 +187,35 @@ MOE_DEV bool mbar_wait_bounded(uint32_t bar, uint32_t parity, volatile int* abor
       }
     }
   }
+}
+
+// ------------------------------------------------------------------ clusters
+MOE_DEV uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+// Address in the shared-memory window of the cluster of the same location in
+// CTA `rank` as the local shared::cta address `addr`.
+MOE_DEV uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+
+// fp32 load from the shared memory of a CTA of the cluster (address from map_to_rank)
+MOE_DEV float ld_cluster_f32(uint32_t cluster_addr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(cluster_addr) : "memory");
+  return v;
+}
+
+// All threads of all CTAs of the cluster: the arrival releases and the wait
+// acquires at cluster scope (shared and global memory).
+MOE_DEV void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" :::
+                   "memory");
 }
 
 // ----------------------------------------------------------------------- TMA

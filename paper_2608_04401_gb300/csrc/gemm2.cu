@@ -71,20 +71,6 @@ struct Cfg {
 };
 
 // ---------------------------------------------------------- cluster helpers
-MOE_DEV uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-
-// Address in the shared-memory window of the cluster of the same location in
-// CTA `rank` as the local shared::cta address `addr`.
-MOE_DEV uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
-  uint32_t r;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
-  return r;
-}
-
 // Arrive once on an mbarrier of the other CTA of the pair (the address from
 // map_to_rank). The default semantics of the remote arrive (release at CTA
 // scope) are those production two-SM kernels use for cross-CTA arrivals: a
@@ -137,11 +123,6 @@ MOE_DEV bool mbar_wait_cluster_bounded(uint32_t bar, uint32_t parity, volatile i
   }
 }
 
-// All threads of both CTAs.
-MOE_DEV void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" :::
-                   "memory");
-}
 
 // ------------------------------------------------------------ tcgen05, pair
 // TMEM allocation of the pair: one warp of each CTA, the same columns in both.

@@ -37,7 +37,8 @@ constexpr int kDownOut = 16;      // down: output columns per block (two per war
 
 // The j-th expert (ascending id) whose row range is nonempty, or -1; all
 // threads of the block get it. s_exp is one int of shared memory.
-MOE_DEV int jth_expert(const int32_t* __restrict__ offsets, int N, int j, int* s_exp) {
+MOE_DEV int jth_expert(const int32_t* __restrict__ offsets, int N, int j, int* s_exp,
+                       int* s_count = nullptr) {
   if (threadIdx.x < 32) {
     int base = 0, found = -1;
     for (int e0 = 0; e0 < N; e0 += 32) {
@@ -53,7 +54,10 @@ MOE_DEV int jth_expert(const int32_t* __restrict__ offsets, int N, int j, int* s
       }
       base += n;
     }
-    if (threadIdx.x == 0) *s_exp = found;
+    if (threadIdx.x == 0) {
+      *s_exp = found;
+      if (s_count) *s_count = base;
+    }
   }
   __syncthreads();
   return *s_exp;
@@ -193,16 +197,34 @@ __global__ void __launch_bounds__(kThreads) gemv_gate_up_kernel(
   }
 }
 
+// The weighted combine of a one-token batch, done by the down projection
+// itself (tickets == nullptr: not done): y[c] = sum_{s<k} g_s o[pair_pos[s], c]
+// (+ residual[c]), accumulated in fp32 in s order, one bf16 rounding at the end.
+struct Combine {
+  const int32_t* k;          // [1]
+  const int32_t* pair_pos;   // [K]
+  const float* gates;        // [K]
+  const uint16_t* residual;  // [d] or nullptr
+  uint16_t* y;               // [d]
+  unsigned int* tickets;     // [ceil(d / kDownOut)], zero on entry, left zero
+  int K;
+};
+
 // o [P, d]: down projection. Dynamic shared memory: kDownOut rows of W_down
 // (I bf16 each), then the expert's rows of h (T x I fp32).
+// With a Combine (T == 1): the blocks of one column block count themselves
+// on its ticket after their stores (a block barrier, then one acquire-release
+// atomic); the last of them, which sees every expert's slice of o, writes
+// those columns of y and resets the ticket. No block waits for another.
 __global__ void __launch_bounds__(kThreads) gemv_down_kernel(
     const uint16_t* __restrict__ h, const int32_t* __restrict__ offsets,
     const uint16_t* __restrict__ wd, int64_t T, int64_t P, int d, int N, int I,
-    uint16_t* __restrict__ o, int32_t* err) {
+    uint16_t* __restrict__ o, int32_t* err, Combine cmb) {
   extern __shared__ __align__(16) uint8_t smem[];
-  __shared__ int s_exp;
+  __shared__ int s_exp, s_count;
   __shared__ alignas(8) uint64_t bar;
   __shared__ int abort_flag;
+  __shared__ bool last;
   const uint32_t bar_a = smem_u32(&bar);
   if (threadIdx.x == 0) {
     mbar_init(bar_a, 1);
@@ -211,7 +233,7 @@ __global__ void __launch_bounds__(kThreads) gemv_down_kernel(
   }
   grid_dep_wait();
   grid_dep_launch();
-  const int e = jth_expert(offsets, N, blockIdx.y, &s_exp);
+  const int e = jth_expert(offsets, N, blockIdx.y, &s_exp, &s_count);
   if (e < 0) return;
   const int c0 = blockIdx.x * kDownOut;
   const int nout = min(kDownOut, d - c0);
@@ -240,10 +262,11 @@ __global__ void __launch_bounds__(kThreads) gemv_down_kernel(
     dst[1] = make_float4(f[4], f[5], f[6], f[7]);
   }
   __syncthreads();
-  if (!wait_rows(bar_a, &abort_flag, err)) return;
+  // one decision for the whole block (a thread may see the copy land just
+  // after another gave up)
+  if (__syncthreads_or(!wait_rows(bar_a, &abort_flag, err) ? 1 : 0)) return;
   const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-  if (rows == 0) return;
-  for (int u = warp; u < nout; u += kWarps) {
+  for (int u = warp; rows > 0 && u < nout; u += kWarps) {
     const uint4* row = reinterpret_cast<const uint4*>(wrows + u * I);
     float acc[kMaxRows] = {};
     for (int q8 = lane; q8 < i8; q8 += 32) {
@@ -269,6 +292,34 @@ __global__ void __launch_bounds__(kThreads) gemv_down_kernel(
       }
     }
   }
+  if (cmb.tickets == nullptr) return;
+  // the block's stores of o happen before thread 0's release (the barrier);
+  // the acquire half makes every earlier block's stores visible to the last
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned int prev;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;"
+                 : "=r"(prev) : "l"(cmb.tickets + blockIdx.x) : "memory");
+    last = static_cast<int>(prev) == s_count - 1;
+  }
+  __syncthreads();
+  if (!last) return;
+  if (threadIdx.x < nout) {
+    const int c = c0 + threadIdx.x;
+    const int kt = min(max(cmb.k[0], 0), cmb.K);
+    MOE_DCHECK(cmb.k[0] >= 0 && cmb.k[0] <= cmb.K);
+    float acc = 0.0f;
+    for (int s2 = 0; s2 < kt; ++s2) {
+      const int pos = cmb.pair_pos[s2];
+      MOE_DCHECK(pos >= 0 && pos < P);
+      const int pc = static_cast<int>(min_of<int64_t>(max(pos, 0), P - 1));
+      const uint16_t ov = __ldcg(o + static_cast<int64_t>(pc) * d + c);
+      acc = fmaf(cmb.gates[s2], __uint_as_float(static_cast<uint32_t>(ov) << 16), acc);
+    }
+    if (cmb.residual) acc += __uint_as_float(static_cast<uint32_t>(cmb.residual[c]) << 16);
+    cmb.y[c] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
+  }
+  if (threadIdx.x == 0) cmb.tickets[blockIdx.x] = 0u;
 }
 
 }  // namespace gemv
@@ -301,12 +352,18 @@ cudaError_t launch_gate_up_gemv(const uint16_t* x, int64_t T, const int32_t* per
                     wgu, P, d, N, I, h, err);
 }
 
+// With tickets not null (T == 1 only; ceil(d / 16) zeroed counters, left
+// zero), the kernel also writes y = the gate-weighted combine of o (+ residual).
 cudaError_t launch_down_gemv(const uint16_t* h, const int32_t* offsets, const uint16_t* wd,
                              int64_t T, int64_t P, int d, int N, int I, int K, uint16_t* o,
-                             int32_t* err, cudaStream_t stream) {
+                             int32_t* err, const int32_t* k, const int32_t* pair_pos,
+                             const float* gates, const uint16_t* residual, uint16_t* y,
+                             unsigned int* tickets, cudaStream_t stream) {
   using namespace gemv;
   if (P == 0 || T == 0) return cudaSuccess;
   if (T > kMaxRows || d > kMaxDim || I > kMaxDim || I % 8 != 0) return cudaErrorInvalidValue;
+  if (tickets && (T != 1 || !k || !pair_pos || !gates || !y)) return cudaErrorInvalidValue;
+  const Combine cmb{k, pair_pos, gates, residual, y, tickets, K};
   const size_t smem = static_cast<size_t>(kDownOut) * I * 2 + sizeof(float) * T * I;
   static std::atomic<uint64_t> attr_done{0};
   const cudaError_t e = once_per_device(attr_done, [] {
@@ -317,7 +374,7 @@ cudaError_t launch_down_gemv(const uint16_t* h, const int32_t* offsets, const ui
   if (e != cudaSuccess) return e;
   const dim3 grid(static_cast<unsigned>((d + kDownOut - 1) / kDownOut), gemv_experts(T, K, N));
   return launch_pdl(gemv_down_kernel, grid, dim3(kThreads), smem, stream, h, offsets, wd, T, P, d,
-                    N, I, o, err);
+                    N, I, o, err, cmb);
 }
 
 }  // namespace moe
