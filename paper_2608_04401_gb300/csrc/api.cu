@@ -72,6 +72,12 @@ cudaError_t launch_router_one(const uint16_t* x, const uint16_t* w_router, int d
                               int32_t* k_out, int32_t* ids_out, float* gates_out, int32_t* offsets,
                               int32_t* perm, int32_t* pair_pos, int32_t* offsets_copy,
                               int32_t* clear, int nclear, cudaStream_t stream);
+cudaError_t launch_expert_one_gemv(const uint16_t* x, const int32_t* offsets, const uint16_t* wgu,
+                                   const uint16_t* wd, int64_t P, int d, int N, int I, int K,
+                                   uint16_t* h, uint16_t* o, int32_t* err, unsigned int* done,
+                                   const int32_t* k, const int32_t* pair_pos, const float* gates,
+                                   const uint16_t* residual, uint16_t* y, unsigned int* tickets,
+                                   int num_sms, cudaStream_t stream);
 cudaError_t launch_quotient_check(const float* a, const float* b, int64_t n, float* out,
                                   cudaStream_t stream);
 cudaError_t launch_route_diagnostics(const float* logits, int64_t T, int N, int K, float eps,
@@ -197,7 +203,8 @@ struct LayerWs {
   uint16_t* h;
   uint16_t* o;
   float* partial;  // decode-sized batches: router partial sums [d/64][T][N]
-  unsigned int* tickets;  // one-token steps: the combine's counters [ceil(d/16)], after err
+  unsigned int* tickets;  // one-token steps: the combine's counters [ceil(d/16)], after err,
+                          // then the expert kernel's 8 completion counters
   size_t bytes;
 };
 
@@ -212,7 +219,7 @@ LayerWs layer_ws(void* base, int64_t T, int d, int N, int I, int K) {
   };
   const size_t P = static_cast<size_t>(T) * K;
   w.err = reinterpret_cast<int32_t*>(take(256));
-  w.tickets = reinterpret_cast<unsigned int*>(take(sizeof(unsigned int) * ((d + 15) / 16)));
+  w.tickets = reinterpret_cast<unsigned int*>(take(sizeof(unsigned int) * ((d + 15) / 16 + 8)));
   w.k = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * T));
   w.ids = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * P));
   w.gates = reinterpret_cast<float*>(take(sizeof(float) * P));
@@ -443,7 +450,7 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
     // clears the error word and the combine's tickets
     const int nclear = static_cast<int>((reinterpret_cast<char*>(w.tickets) -
                                          reinterpret_cast<char*>(w.err)) / sizeof(int32_t)) +
-                       (d + 15) / 16;
+                       (d + 15) / 16 + 8;
     e = moe::launch_router_one(x, w_router, d, N, K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
                                rp->renorm, logits_out, kk, ids, gates, w.offsets, w.perm,
                                w.pair_pos, offsets_out, w.err, nclear, s);
@@ -465,11 +472,10 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   if (gemv_path) {
     // one token (dispatched by its router): the CUDA-core expert
     // contractions, which read the token row through perm
-    e = moe::launch_gate_up_gemv(x, T, w.perm, w.offsets, w_gate_up, P, d, N, I, K, w.h, w.err, s);
-    if (e != cudaSuccess) return MOE_ERR_CUDA;
-    // the down projection also combines (its last block per column block)
-    e = moe::launch_down_gemv(w.h, w.offsets, w_down, T, P, d, N, I, K, w.o, w.err, kk, w.pair_pos,
-                              gates, residual, y, w.tickets, s);
+    // contractions and combine in one cooperative launch
+    e = moe::launch_expert_one_gemv(x, w.offsets, w_gate_up, w_down, P, d, N, I, K, w.h, w.o, w.err,
+                                    w.tickets + (d + 15) / 16, kk, w.pair_pos, gates, residual, y,
+                                    w.tickets, nsm, s);
     return e == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
   } else if (T <= kDecodeMaxTokens) {
     // decode-sized: the single-chunk dispatch also gathers the few token rows

@@ -25,6 +25,8 @@
 // and the lanes' partial sums meet in a butterfly reduction.
 #include "common.cuh"
 
+#include <algorithm>
+
 namespace moe {
 namespace gemv {
 
@@ -93,12 +95,12 @@ MOE_DEV void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t b
 // error word is set, and the copies still in flight are waited for again
 // (bounded) so that none lands after the block has exited. Returns whether
 // the data arrived.
-MOE_DEV bool wait_rows(uint32_t bar, volatile int* abort_flag, int32_t* err) {
-  const bool ok = mbar_wait_bounded(bar, 0u, abort_flag);
+MOE_DEV bool wait_rows(uint32_t bar, volatile int* abort_flag, int32_t* err, uint32_t parity = 0u) {
+  const bool ok = mbar_wait_bounded(bar, parity, abort_flag);
   if (!ok) {
     if (threadIdx.x == 0 && err) atomicExch(err, kDevErrTimeout);
     const uint64_t t0 = global_timer_ns();
-    while (!mbar_try_wait(bar, 0u) && global_timer_ns() - t0 < 100000000ull) {
+    while (!mbar_try_wait(bar, parity) && global_timer_ns() - t0 < 100000000ull) {
     }
   }
   return ok;
@@ -210,6 +212,40 @@ struct Combine {
   int K;
 };
 
+// The combine of one column block [c0, c0 + nout) by the last of the `count`
+// blocks that wrote its slices of o (see Combine); called by all threads of
+// each such block after its stores of o.
+MOE_DEV void combine_tail(const Combine& cmb, const uint16_t* o, int64_t P, int d, int c0, int nout,
+                          int cb, int count, bool* last) {
+  // the block's stores of o happen before thread 0's release (the barrier);
+  // the acquire half makes every earlier block's stores visible to the last
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned int prev;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;"
+                 : "=r"(prev) : "l"(cmb.tickets + cb) : "memory");
+    *last = static_cast<int>(prev) == count - 1;
+  }
+  __syncthreads();
+  if (!*last) return;
+  if (threadIdx.x < nout) {
+    const int c = c0 + threadIdx.x;
+    const int kt = min(max(cmb.k[0], 0), cmb.K);
+    MOE_DCHECK(cmb.k[0] >= 0 && cmb.k[0] <= cmb.K);
+    float acc = 0.0f;
+    for (int s2 = 0; s2 < kt; ++s2) {
+      const int pos = cmb.pair_pos[s2];
+      MOE_DCHECK(pos >= 0 && pos < P);
+      const int pc = static_cast<int>(min_of<int64_t>(max(pos, 0), P - 1));
+      const uint16_t ov = __ldcg(o + static_cast<int64_t>(pc) * d + c);
+      acc = fmaf(cmb.gates[s2], __uint_as_float(static_cast<uint32_t>(ov) << 16), acc);
+    }
+    if (cmb.residual) acc += __uint_as_float(static_cast<uint32_t>(cmb.residual[c]) << 16);
+    cmb.y[c] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
+  }
+  if (threadIdx.x == 0) cmb.tickets[cb] = 0u;
+}
+
 // o [P, d]: down projection. Dynamic shared memory: kDownOut rows of W_down
 // (I bf16 each), then the expert's rows of h (T x I fp32).
 // With a Combine (T == 1): the blocks of one column block count themselves
@@ -293,33 +329,199 @@ __global__ void __launch_bounds__(kThreads) gemv_down_kernel(
     }
   }
   if (cmb.tickets == nullptr) return;
-  // the block's stores of o happen before thread 0's release (the barrier);
-  // the acquire half makes every earlier block's stores visible to the last
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    unsigned int prev;
-    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;"
-                 : "=r"(prev) : "l"(cmb.tickets + blockIdx.x) : "memory");
-    last = static_cast<int>(prev) == s_count - 1;
-  }
-  __syncthreads();
-  if (!last) return;
-  if (threadIdx.x < nout) {
-    const int c = c0 + threadIdx.x;
-    const int kt = min(max(cmb.k[0], 0), cmb.K);
-    MOE_DCHECK(cmb.k[0] >= 0 && cmb.k[0] <= cmb.K);
-    float acc = 0.0f;
-    for (int s2 = 0; s2 < kt; ++s2) {
-      const int pos = cmb.pair_pos[s2];
-      MOE_DCHECK(pos >= 0 && pos < P);
-      const int pc = static_cast<int>(min_of<int64_t>(max(pos, 0), P - 1));
-      const uint16_t ov = __ldcg(o + static_cast<int64_t>(pc) * d + c);
-      acc = fmaf(cmb.gates[s2], __uint_as_float(static_cast<uint32_t>(ov) << 16), acc);
+  combine_tail(cmb, o, P, d, c0, nout, blockIdx.x, s_count, &last);
+}
+
+// ------------------------------------------------ one-token expert MLP, fused
+// The gate/up and down contractions of a one-token step (and its combine) in
+// one cooperative launch, so that no kernel boundary separates them and the
+// first down weights stream in while the last gate/up rows are computed. The
+// work items are those of the two kernels above, T = 1: gate/up items
+// (j, output block of 8) and down items (j, block of dn_rows columns) over the
+// j < n experts with a row (ascending id). Block b takes the gate/up items
+// b, b + G, ... and then the down items G - 1 - b, 2G - 1 - b, ... (G blocks,
+// all resident: the launch is cooperative). After a gate/up item's h stores, thread 0 adds
+// one to done[j] (release); a down item starts its weight copy, then thread 0
+// waits (acquire, bounded) until done[j] counts all of expert j's gate/up
+// items before the block reads h. Every block finishes its gate/up items
+// before it waits, and all blocks are resident, so every wait ends; a wait
+// that runs out sets the error word and the block leaves once its copy has
+// landed. The last block of each column block combines (combine_tail).
+constexpr int kOneMaxExperts = 8;  // experts with a row: k <= K <= 8
+
+MOE_DEV bool wait_count(const unsigned int* ctr, unsigned int target, volatile int* abort) {
+  const uint64_t t0 = global_timer_ns();
+  for (uint32_t spins = 1;; ++spins) {
+    unsigned int v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+    if (v >= target) return true;
+    if (spins % 64u == 0u) {
+      if (*abort) return false;
+      if (global_timer_ns() - t0 > kWaitLimitNs) {
+        *abort = 1;
+        return false;
+      }
     }
-    if (cmb.residual) acc += __uint_as_float(static_cast<uint32_t>(cmb.residual[c]) << 16);
-    cmb.y[c] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
+    __nanosleep(32);
   }
-  if (threadIdx.x == 0) cmb.tickets[blockIdx.x] = 0u;
+}
+
+// Dynamic shared memory: wbytes of weight rows (the gate/up item's 2 x 8 rows
+// of d, or the down item's dn_rows rows of I, bf16), then max(d, I) fp32 (x,
+// then h). A down item takes 16 rows, or more when the experts' down items
+// outnumber the blocks, up to dn_max rows: as many as the gate/up item's space
+// holds (a multiple of 8, 16 to 64).
+__global__ void __launch_bounds__(kThreads) gemv_expert_one_kernel(
+    const uint16_t* __restrict__ x, const int32_t* __restrict__ offsets,
+    const uint16_t* __restrict__ wgu, const uint16_t* __restrict__ wd, int64_t P, int d, int N,
+    int I, uint32_t wbytes, int dn_max, uint16_t* h, uint16_t* o, int32_t* err,
+    unsigned int* done, Combine cmb) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  __shared__ int s_used[kOneMaxExperts];
+  __shared__ int s_n, s_ok;
+  __shared__ alignas(8) uint64_t bar;
+  __shared__ int abort_flag;
+  __shared__ bool last;
+  const uint32_t bar_a = smem_u32(&bar);
+  if (threadIdx.x == 0) {
+    mbar_init(bar_a, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  grid_dep_wait();
+  grid_dep_launch();
+  if (threadIdx.x < 32) {  // the experts with a row, ascending id
+    const int lane = threadIdx.x;
+    int base = 0;
+    for (int e0 = 0; e0 < N; e0 += 32) {
+      const int e = e0 + lane;
+      const bool used = e < N && offsets[e + 1] > offsets[e];
+      const unsigned m = __ballot_sync(0xffffffffu, used);
+      const int idx = base + __popc(m & ((1u << lane) - 1u));
+      if (used && idx < kOneMaxExperts) s_used[idx] = e;
+      base += __popc(m);
+    }
+    MOE_DCHECK(base <= kOneMaxExperts);
+    if (lane == 0) s_n = min(base, kOneMaxExperts);
+  }
+  uint16_t* wrows = reinterpret_cast<uint16_t*>(smem);
+  float* vec = reinterpret_cast<float*>(smem + wbytes);
+  const int d8 = d / 8, i8 = I / 8;
+  for (int c = threadIdx.x; c < d8; c += kThreads) {  // the token row, fp32
+    float f[8];
+    bf16x8_to_f32(__ldg(reinterpret_cast<const uint4*>(x) + c), f);
+    reinterpret_cast<float4*>(vec + c * 8)[0] = make_float4(f[0], f[1], f[2], f[3]);
+    reinterpret_cast<float4*>(vec + c * 8)[1] = make_float4(f[4], f[5], f[6], f[7]);
+  }
+  __syncthreads();  // s_used, s_n, x, barrier init
+  const int n = s_n;
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int ngu = (I + kGateUpOut - 1) / kGateUpOut;
+  // down items: the fewest rows (16, 24, ... up to dn_max) that give each
+  // block at most one item, so that few experts still spread over all blocks
+  int dn_rows = 16;
+  while (dn_rows < dn_max && n * ((d + dn_rows - 1) / dn_rows) > static_cast<int>(gridDim.x))
+    dn_rows += 8;
+  const int ndn = (d + dn_rows - 1) / dn_rows;
+  uint32_t parity = 0;
+
+  for (int it = blockIdx.x; it < n * ngu; it += gridDim.x) {
+    const int j = it / ngu, i0 = (it % ngu) * kGateUpOut;
+    const int e = s_used[j];
+    const int nout = min(kGateUpOut, I - i0);
+    const uint32_t row_bytes = static_cast<uint32_t>(d) * 2;
+    if (threadIdx.x == 0) {
+      mbar_arrive_expect_tx(bar_a, 2 * nout * row_bytes);
+      const uint16_t* wg = wgu + static_cast<int64_t>(e) * 2 * I * d;
+      for (int u = 0; u < nout; ++u) {
+        bulk_load(smem_u32(wrows) + u * row_bytes, wg + static_cast<int64_t>(i0 + u) * d, row_bytes,
+                  bar_a);
+        bulk_load(smem_u32(wrows) + (kGateUpOut + u) * row_bytes,
+                  wg + static_cast<int64_t>(I + i0 + u) * d, row_bytes, bar_a);
+      }
+    }
+    const int p0 = offsets[e];
+    MOE_DCHECK(p0 >= 0 && p0 < P);
+    const bool ok = !__syncthreads_or(!wait_rows(bar_a, &abort_flag, err, parity) ? 1 : 0);
+    parity ^= 1u;
+    if (!ok) return;
+    if (warp < nout && p0 >= 0 && p0 < P) {
+      const uint4* grow = reinterpret_cast<const uint4*>(wrows + warp * d);
+      const uint4* urow = reinterpret_cast<const uint4*>(wrows + (kGateUpOut + warp) * d);
+      float g = 0.0f, v = 0.0f;
+      for (int c = lane; c < d8; c += 32) {
+        float fg[8], fu[8];
+        bf16x8_to_f32(grow[c], fg);
+        bf16x8_to_f32(urow[c], fu);
+        const float4 x0 = reinterpret_cast<const float4*>(vec + c * 8)[0];
+        const float4 x1 = reinterpret_cast<const float4*>(vec + c * 8)[1];
+        const float xv[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          g = fmaf(fg[q], xv[q], g);
+          v = fmaf(fu[q], xv[q], v);
+        }
+      }
+      const float gs = warp_sum(g), us = warp_sum(v);
+      if (lane == 0)
+        h[static_cast<int64_t>(p0) * I + i0 + warp] =
+            __bfloat16_as_ushort(__float2bfloat16_rn(silu(gs) * us));
+    }
+    // the item's h stores happen before the release; the weight rows are free
+    __syncthreads();
+    if (threadIdx.x == 0)
+      asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(done + j) : "memory");
+  }
+
+  // down items from the last block backwards: blocks with fewer gate/up
+  // items (the higher ones) take the second round of down items
+  for (int it = gridDim.x - 1 - blockIdx.x; it < n * ndn; it += gridDim.x) {
+    const int j = it / ndn, cb = it % ndn, c0 = cb * dn_rows;
+    const int e = s_used[j];
+    const int nout = min(dn_rows, d - c0);
+    const uint32_t row_bytes = static_cast<uint32_t>(I) * 2;
+    if (threadIdx.x == 0) {
+      // rows c0 .. c0 + nout - 1 of W_down[e] are contiguous: one copy
+      mbar_arrive_expect_tx(bar_a, nout * row_bytes);
+      bulk_load(smem_u32(wrows), wd + (static_cast<int64_t>(e) * d + c0) * I, nout * row_bytes,
+                bar_a);
+      s_ok = wait_count(done + j, static_cast<unsigned int>(ngu), &abort_flag) ? 1 : 0;
+      if (!s_ok && err) atomicExch(err, kDevErrTimeout);
+    }
+    __syncthreads();
+    const int p0 = offsets[e];
+    MOE_DCHECK(p0 >= 0 && p0 < P);
+    const bool have_h = s_ok && p0 >= 0 && p0 < P;
+    if (have_h) {
+      for (int c = threadIdx.x; c < i8; c += kThreads) {  // expert j's h row, fp32
+        float f[8];
+        bf16x8_to_f32(__ldcg(reinterpret_cast<const uint4*>(h + static_cast<int64_t>(p0) * I) + c), f);
+        reinterpret_cast<float4*>(vec + c * 8)[0] = make_float4(f[0], f[1], f[2], f[3]);
+        reinterpret_cast<float4*>(vec + c * 8)[1] = make_float4(f[4], f[5], f[6], f[7]);
+      }
+    }
+    const bool ok = !__syncthreads_or(!wait_rows(bar_a, &abort_flag, err, parity) ? 1 : 0);
+    parity ^= 1u;
+    if (!ok || !s_ok) return;  // uniform: s_ok is shared, the copy has landed or was waited for
+    for (int u = warp; have_h && u < nout; u += kWarps) {
+      const uint4* row = reinterpret_cast<const uint4*>(wrows + u * I);
+      float acc = 0.0f;
+      for (int q8 = lane; q8 < i8; q8 += 32) {
+        float fw[8];
+        bf16x8_to_f32(row[q8], fw);
+        const float4 h0 = reinterpret_cast<const float4*>(vec + q8 * 8)[0];
+        const float4 h1 = reinterpret_cast<const float4*>(vec + q8 * 8)[1];
+        const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc = fmaf(fw[q], hv[q], acc);
+      }
+      const float sum = warp_sum(acc);
+      if (lane == 0)
+        o[static_cast<int64_t>(p0) * d + c0 + u] = __bfloat16_as_ushort(__float2bfloat16_rn(sum));
+    }
+    combine_tail(cmb, o, P, d, c0, nout, cb, n, &last);
+    __syncthreads();  // the weight rows and h are free for the next item
+  }
 }
 
 }  // namespace gemv
@@ -375,6 +577,67 @@ cudaError_t launch_down_gemv(const uint16_t* h, const int32_t* offsets, const ui
   const dim3 grid(static_cast<unsigned>((d + kDownOut - 1) / kDownOut), gemv_experts(T, K, N));
   return launch_pdl(gemv_down_kernel, grid, dim3(kThreads), smem, stream, h, offsets, wd, T, P, d,
                     N, I, o, err, cmb);
+}
+
+
+// The expert MLP and combine of a one-token step (see gemv_expert_one_kernel):
+// h [K, I] and o [K, d] scratch, done: kOneMaxExperts zeroed counters (left
+// counting), tickets: ceil(d / 16) zeroed counters (left zero).
+cudaError_t launch_expert_one_gemv(const uint16_t* x, const int32_t* offsets, const uint16_t* wgu,
+                                   const uint16_t* wd, int64_t P, int d, int N, int I, int K,
+                                   uint16_t* h, uint16_t* o, int32_t* err, unsigned int* done,
+                                   const int32_t* k, const int32_t* pair_pos, const float* gates,
+                                   const uint16_t* residual, uint16_t* y, unsigned int* tickets,
+                                   int num_sms, cudaStream_t stream) {
+  using namespace gemv;
+  if (P == 0) return cudaSuccess;
+  if (d > kMaxDim || I > kMaxDim || d % 8 != 0 || I % 8 != 0 || K > kOneMaxExperts ||
+      num_sms <= 0 || !done || !tickets)
+    return cudaErrorInvalidValue;
+  const int dn_max = std::min(64, std::max(16, (2 * kGateUpOut * d / I) / 8 * 8));
+  const uint32_t wbytes = static_cast<uint32_t>(
+      std::max(2 * kGateUpOut * d * 2, dn_max * I * 2));
+  const size_t smem = wbytes + sizeof(float) * static_cast<size_t>(std::max(d, I));
+  static std::atomic<uint64_t> attr_done{0};
+  cudaError_t e = once_per_device(attr_done, [] {
+    return cudaFuncSetAttribute(gemv_expert_one_kernel,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                // (dn_rows * I <= max(16 I, 16 d): at most 2 x 8 rows of kMaxDim)
+                                static_cast<int>(2 * kGateUpOut * kMaxDim * 2 + 4 * kMaxDim));
+  });
+  if (e != cudaSuccess) return e;
+  // resident blocks per SM for this size (cached: the last size asked)
+  static thread_local size_t cached_smem = 0;
+  static thread_local int cached_dev = -1, cached_blocks = 0;
+  int dev = 0;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if (cached_smem != smem || cached_dev != dev) {
+    int nb = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, gemv_expert_one_kernel, kThreads, smem);
+    if (e != cudaSuccess) return e;
+    if (nb <= 0) return cudaErrorInvalidConfiguration;
+    cached_smem = smem;
+    cached_dev = dev;
+    cached_blocks = nb;
+  }
+  const int nexp = std::min(N, K);
+  const int items = nexp * std::max((I + kGateUpOut - 1) / kGateUpOut, (d + 15) / 16);
+  const int grid = std::min(items, cached_blocks * num_sms);
+  const Combine cmb{k, pair_pos, gates, residual, y, tickets, K};
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, gemv_expert_one_kernel, x, offsets, wgu, wd, P, d, N, I, wbytes,
+                            dn_max, h, o, err, done, cmb);
 }
 
 }  // namespace moe
