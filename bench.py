@@ -495,10 +495,12 @@ def dev_experts(N, d, I, seed, dev):
     return wgu, wd
 
 
-def graph_ms(step, steps, stream, pg):
-    """ms per replay of a CUDA graph that captured one call of `step` (the
-    library launches on the current stream and allocates nothing, so a whole
-    layer, or stack of layers, is one graph)."""
+def graph_ms(step, steps, stream, pg, reps=1):
+    """ms per call of `step` in a CUDA graph that captured `reps` calls of it
+    back to back (the library launches on the current stream and allocates
+    nothing, so a whole layer, or stack of layers, is one graph). With reps > 1
+    the host's per-replay submission is spread over reps steps: for steps of
+    a few microseconds a one-step graph measures the submission rate."""
     import torch
     side = torch.cuda.Stream()
     side.wait_stream(torch.cuda.current_stream())
@@ -508,10 +510,11 @@ def graph_ms(step, steps, stream, pg):
     torch.cuda.current_stream().wait_stream(side)
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g):
-        step()
+        for _ in range(reps):
+            step()
     for _ in range(3):
         g.replay()
-    return time_steps(g.replay, steps, stream, pg)
+    return time_steps(g.replay, max(1, steps // reps), stream, pg) / reps
 
 
 def graph_cold_ms(step, steps, stream):
@@ -536,7 +539,8 @@ def graph_cold_ms(step, steps, stream):
     return ms
 
 
-def time_layer_modes(moe, x, wr, wgu, wd, K, steps, stream, pg, residual=None, cold=False):
+def time_layer_modes(moe, x, wr, wgu, wd, K, steps, stream, pg, residual=None, cold=False,
+                     seq=0):
     """ms per moe_layer_forward in elbow and in top-K mode; sum k of the elbow batch."""
     import torch
     T, d = x.shape
@@ -552,6 +556,9 @@ def time_layer_modes(moe, x, wr, wgu, wd, K, steps, stream, pg, residual=None, c
             step()
         out[name] = time_steps(step, steps, stream, pg)
         out[name + "_graph"] = graph_ms(step, steps, stream, pg)
+        if seq:
+            out[name + "_graph_seq"] = graph_ms(step, seq * max(4, steps // seq), stream, pg,
+                                                reps=seq)
         if cold:
             out[name + "_graph_cold"] = graph_cold_ms(step, steps, stream)
     moe.read_device_error(ws)
@@ -598,17 +605,20 @@ def other_configs(moe, args, stream, dev, pk, pg, cpu=False):
             dec = {}
             for Td in (1, 2, 8):
                 rd = time_layer_modes(moe, x[:Td].contiguous(), wr, wgu, wd, K, steps, stream, pg,
-                                      cold=True)
+                                      cold=True, seq=16)
                 wb = rd["touched"] * 3 * d * I * 2
                 dec[f"T={Td}"] = {"elbow_ms": rd["elbow"], "topk_ms": rd["topk"],
                                   "elbow_graph_ms": rd["elbow_graph"],
                                   "topk_graph_ms": rd["topk_graph"],
+                                  "elbow_graph_seq16_ms": rd["elbow_graph_seq"],
+                                  "topk_graph_seq16_ms": rd["topk_graph_seq"],
                                   "elbow_graph_cold_ms": rd["elbow_graph_cold"],
                                   "topk_graph_cold_ms": rd["topk_graph_cold"],
-                                  "note": "graph replays; cold = L2 flushed before each replay "
-                                          "(weights from HBM)",
+                                  "note": "graph = one step per replay (host submission can "
+                                          "bound it); graph_seq16 = per step in graphs of 16 "
+                                          "steps (the device time); cold = one step per replay "
+                                          "with L2 flushed before it (weights from HBM)",
                                   "experts_touched": rd["touched"], "mean_k": rd["sum_k"] / Td,
-                                  "weight_hbm_frac_graph": wb / (rd["elbow_graph"] * 1e-3) / 1e9 / pk["hbm"],
                                   "weight_hbm_frac_graph_cold":
                                       wb / (rd["elbow_graph_cold"] * 1e-3) / 1e9 / pk["hbm"]}
             res[name]["decode"] = dec

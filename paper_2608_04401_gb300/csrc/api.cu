@@ -57,9 +57,7 @@ cudaError_t launch_gate_up_gemv(const uint16_t* x, int64_t T, const int32_t* per
                                 cudaStream_t stream);
 cudaError_t launch_down_gemv(const uint16_t* h, const int32_t* offsets, const uint16_t* wd,
                              int64_t T, int64_t P, int d, int N, int I, int K, uint16_t* o,
-                             int32_t* err, const int32_t* k, const int32_t* pair_pos,
-                             const float* gates, const uint16_t* residual, uint16_t* y,
-                             unsigned int* tickets, cudaStream_t stream);
+                             int32_t* err, cudaStream_t stream);
 cudaError_t launch_route_warp(const float* logits, int64_t T, int N, int K, float eps,
                               int topk_mode, int renorm, int32_t* k_out, int32_t* ids_out,
                               float* gates_out, cudaStream_t stream);
@@ -67,15 +65,16 @@ cudaError_t launch_router_small_route(const uint16_t* x, const uint16_t* w_route
                                       int N, float* partial, unsigned int* ticket, int K, float eps,
                                       int topk_mode, int renorm, float* logits_out, int32_t* k_out,
                                       int32_t* ids_out, float* gates_out, cudaStream_t stream);
-cudaError_t launch_router_one(const uint16_t* x, const uint16_t* w_router, int d, int N, int K,
-                              float eps, int topk_mode, int renorm, float* logits_out,
+cudaError_t launch_router_few(const uint16_t* x, const uint16_t* w_router, int T, int d, int N,
+                              int K, float eps, int topk_mode, int renorm, float* logits_out,
                               int32_t* k_out, int32_t* ids_out, float* gates_out, int32_t* offsets,
                               int32_t* perm, int32_t* pair_pos, int32_t* offsets_copy,
                               int32_t* clear, int nclear, cudaStream_t stream);
-cudaError_t launch_expert_one_gemv(const uint16_t* x, const int32_t* offsets, const uint16_t* wgu,
-                                   const uint16_t* wd, int64_t P, int d, int N, int I, int K,
-                                   uint16_t* h, uint16_t* o, int32_t* err, unsigned int* done,
-                                   const int32_t* k, const int32_t* pair_pos, const float* gates,
+cudaError_t launch_expert_few_gemv(const uint16_t* x, int64_t T, const int32_t* perm,
+                                   const int32_t* offsets, const uint16_t* wgu, const uint16_t* wd,
+                                   int64_t P, int d, int N, int I, int K, uint16_t* h, uint16_t* o,
+                                   int32_t* err, unsigned int* done, const int32_t* k,
+                                   const int32_t* pair_pos, const float* gates,
                                    const uint16_t* residual, uint16_t* y, unsigned int* tickets,
                                    int num_sms, cudaStream_t stream);
 cudaError_t launch_quotient_check(const float* a, const float* b, int64_t n, float* out,
@@ -129,15 +128,19 @@ constexpr int64_t kWarpRouteMaxTokens = 16;
 // through one SM.
 constexpr int64_t kSmallRouterMaxTokens = 64;
 // The CUDA-core expert contractions take batches of at most kGemvMaxTokens
-// tokens (d, I at most kGemvMaxDim); the layer uses them for one-token steps,
-// where they spread each touched expert's weight rows over many blocks instead
-// of paying the tensor-core decode tiles' fixed latency: with the weights
-// coming from HBM, a one-token step measured 33.0 against 40.7 us with two
-// experts and 51.3 against 51.4 us with eight, while from two tokens on the
-// tensor-core tiles were faster (52.4 against 56.2 us).
+// tokens (d, I at most kGemvMaxDim). Layer steps of at most
+// kGemvLayerMaxTokens tokens run as three kernels: the few-token cluster
+// router (routing, dispatch, clearing the step's counters), then the expert
+// MLP and combine in one cooperative kernel, which spreads each touched
+// expert's weight rows over all SMs instead of paying the tensor-core decode
+// tiles' fixed latency. Measured per step in graphs of 16 steps
+// (d = 2048, N = 64, I = 1024): one token 15.3 us with two experts and 27.6
+// us with eight (the tensor-core path 17.8 and 35.4), two tokens 32.7 and
+// 50.6 us (38.9 and 59.8); from three tokens on the tensor-core tiles are
+// faster (61.3 against 66.7 us).
 constexpr int64_t kGemvMaxTokens = 4;
-constexpr int64_t kGemvLayerMaxTokens = 1;
-static_assert(kGemvLayerMaxTokens == 1, "the one-token router serves the CUDA-core path");
+constexpr int64_t kGemvLayerMaxTokens = 2;
+static_assert(kGemvLayerMaxTokens <= 4, "the few-token router serves the CUDA-core path");
 constexpr int kGemvMaxDim = 4096;
 constexpr int kSmallRouterSlice = 64;
 
@@ -203,8 +206,8 @@ struct LayerWs {
   uint16_t* h;
   uint16_t* o;
   float* partial;  // decode-sized batches: router partial sums [d/64][T][N]
-  unsigned int* tickets;  // one-token steps: the combine's counters [ceil(d/16)], after err,
-                          // then the expert kernel's 8 completion counters
+  unsigned int* tickets;  // few-token steps: the combine's counters [ceil(d/16)], after err,
+                          // then the expert kernel's 32 completion counters
   size_t bytes;
 };
 
@@ -219,7 +222,7 @@ LayerWs layer_ws(void* base, int64_t T, int d, int N, int I, int K) {
   };
   const size_t P = static_cast<size_t>(T) * K;
   w.err = reinterpret_cast<int32_t*>(take(256));
-  w.tickets = reinterpret_cast<unsigned int*>(take(sizeof(unsigned int) * ((d + 15) / 16 + 8)));
+  w.tickets = reinterpret_cast<unsigned int*>(take(sizeof(unsigned int) * ((d + 15) / 16 + 32)));
   w.k = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * T));
   w.ids = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * P));
   w.gates = reinterpret_cast<float*>(take(sizeof(float) * P));
@@ -430,8 +433,8 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
       return MOE_ERR_INVALID_ARG;
   }
   // clear the device error word (and the small-batch router's four group
-  // tickets beside it), so that a no-op call reads clean; on the one-token
-  // path the router clears it, and the combine's tickets that follow
+  // tickets beside it), so that a no-op call reads clean; on the few-token
+  // path the router clears it, and the expert kernel's counters that follow
   const bool gemv_path = T >= 1 && T <= kGemvLayerMaxTokens && d <= kGemvMaxDim && I <= kGemvMaxDim;
   if (!gemv_path && cudaMemsetAsync(w.err, 0, 8 * sizeof(int32_t), s) != cudaSuccess)
     return MOE_ERR_CUDA;
@@ -446,14 +449,14 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
 
   cudaError_t e;
   if (gemv_path) {
-    // one token: router, routing and dispatch on one cluster, which also
-    // clears the error word and the combine's tickets
+    // a few tokens: router, routing and dispatch on one cluster, which also
+    // clears the error word and the expert kernel's counters
     const int nclear = static_cast<int>((reinterpret_cast<char*>(w.tickets) -
                                          reinterpret_cast<char*>(w.err)) / sizeof(int32_t)) +
-                       (d + 15) / 16 + 8;
-    e = moe::launch_router_one(x, w_router, d, N, K, rp->eps, rp->mode == MOE_ROUTE_TOPK,
-                               rp->renorm, logits_out, kk, ids, gates, w.offsets, w.perm,
-                               w.pair_pos, offsets_out, w.err, nclear, s);
+                       (d + 15) / 16 + 32;
+    e = moe::launch_router_few(x, w_router, static_cast<int>(T), d, N, K, rp->eps,
+                               rp->mode == MOE_ROUTE_TOPK, rp->renorm, logits_out, kk, ids, gates,
+                               w.offsets, w.perm, w.pair_pos, offsets_out, w.err, nclear, s);
   } else if (T <= kSmallRouterMaxTokens) {
     // a few tokens: the router GEMM split over d on many SMs, then one warp per
     // token routes (the single-chunk dispatch counts the pairs itself)
@@ -470,12 +473,12 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
   }
   if (e != cudaSuccess) return MOE_ERR_CUDA;
   if (gemv_path) {
-    // one token (dispatched by its router): the CUDA-core expert
-    // contractions, which read the token row through perm
-    // contractions and combine in one cooperative launch
-    e = moe::launch_expert_one_gemv(x, w.offsets, w_gate_up, w_down, P, d, N, I, K, w.h, w.o, w.err,
-                                    w.tickets + (d + 15) / 16, kk, w.pair_pos, gates, residual, y,
-                                    w.tickets, nsm, s);
+    // a few tokens (dispatched by their router): the CUDA-core expert
+    // contractions, which read the token rows through perm, and the combine,
+    // in one cooperative launch
+    e = moe::launch_expert_few_gemv(x, T, w.perm, w.offsets, w_gate_up, w_down, P, d, N, I, K, w.h,
+                                    w.o, w.err, w.tickets + (d + 15) / 16, kk, w.pair_pos, gates,
+                                    residual, y, w.tickets, nsm, s);
     return e == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
   } else if (T <= kDecodeMaxTokens) {
     // decode-sized: the single-chunk dispatch also gathers the few token rows
@@ -666,7 +669,6 @@ moe_status moe_expert_down_gemv(const uint16_t* h, const int32_t* offsets, const
       !aligned4(offsets) || (reinterpret_cast<uintptr_t>(o) & 1u) || !aligned4(err_word))
     return MOE_ERR_INVALID_ARG;
   return cuda_status(moe::launch_down_gemv(h, offsets, w_down, T, P, d, N, I, K, o, err_word,
-                                           nullptr, nullptr, nullptr, nullptr, nullptr, nullptr,
                                            static_cast<cudaStream_t>(stream)));
 }
 

@@ -22,8 +22,8 @@
 // in each group the block that finishes last adds the slices in order and
 // routes the group's tokens.
 //
-// router_one_kernel: the router of a one-token step with its routing and
-// dispatch, on one cluster of 8 CTAs that add their column slices' sums
+// router_few_kernel: the router of a step of at most 4 tokens with its routing
+// and dispatch, on one cluster of 8 CTAs that add their column slices' sums
 // through distributed shared memory (no global scratch, no counter).
 #include "route_impl.cuh"
 
@@ -239,95 +239,123 @@ __global__ void __launch_bounds__(kSmallThreads) router_small_route_kernel(
   if (threadIdx.x == 0) ticket[blockIdx.y] = 0u;
 }
 
-// ------------------------------------------------------- one-token router
-// The router of a one-token step on one cluster of kOneCtas CTAs, with the
-// token's dispatch, and no global scratch or counter: CTA r forms the dots of
-// columns [r cs, (r + 1) cs), cs = d / kOneCtas, thread (e, q) (q fastest)
-// over the 16-byte chunks q, q + Q, ... of that range (each an fp32 fma chain
-// in column order; the Q chains of an expert added by a shuffle tree); the
-// cluster's CTA 0 adds the CTAs' sums in rank order through distributed shared
-// memory, routes the token with one warp and writes the dispatch: the k
-// selected experts (distinct ids) get one row each in ascending id order,
-// offsets[e] = the number of selected ids below e, the row of slot s is the
-// rank of ids[s] among them, every row holds token 0, pair_pos[s] = -1 for
-// s >= k. CTA 0 also zeroes clear[0 .. nclear) (the step's error word and
-// counters) once the previous kernel has finished.
-constexpr int kOneCtas = 8;
-constexpr int kOneThreads = 512;
+// ----------------------------------------------------- few-token router
+// The router of a step of T <= 4 tokens on one cluster of kFewCtas CTAs, with
+// the step's dispatch, and no global scratch or counter: CTA r forms the dots
+// of columns [r cs, (r + 1) cs), cs = d / kFewCtas, thread (e, q) (q fastest)
+// over the 16-byte chunks q, q + Q, ... of that range, for every token (each
+// an fp32 fma chain in column order; the Q chains of an expert added by a
+// shuffle tree); the cluster's CTA 0 adds the CTAs' sums in rank order through
+// distributed shared memory, routes token t with warp t and writes the
+// dispatch. Its rows are the selected pairs (t, s), s < k_t (a token selects
+// an expert once), by expert id and then by token: offsets[e] = the number of
+// pairs with an id below e; the row of pair (t, s) is that count for its id
+// plus the pairs of the same expert from tokens before t; perm[row] = t;
+// pair_pos[t, s] = the row, or -1 for s >= k_t. CTA 0 also zeroes
+// clear[0 .. nclear) (the step's error word and counters) once the previous
+// kernel has finished.
+constexpr int kFewCtas = 8;
+constexpr int kFewThreads = 512;
+constexpr int kFewMaxT = 4;
 
-struct OneTokenOut {
-  float* logits;          // [N] or nullptr
-  int32_t* k;             // [1]
-  int32_t* ids;           // [K]
-  float* gates;           // [K]
+struct FewTokenOut {
+  float* logits;          // [T, N] or nullptr
+  int32_t* k;             // [T]
+  int32_t* ids;           // [T, K]
+  float* gates;           // [T, K]
   int32_t* offsets;       // [N + 1]
-  int32_t* perm;          // [K]
-  int32_t* pair_pos;      // [K]
+  int32_t* perm;          // [T K]
+  int32_t* pair_pos;      // [T, K]
   int32_t* offsets_copy;  // [N + 1] or nullptr
   int32_t* clear;         // [nclear]
   int nclear;
 };
 
-template <int N>
-__global__ void __launch_bounds__(kOneThreads) router_one_kernel(
+template <int N, int T>
+__global__ void __launch_bounds__(kFewThreads) router_few_kernel(
     const uint4* __restrict__ x, const uint4* __restrict__ w, int d, int K, float eps,
-    int topk_mode, int renorm, OneTokenOut out) {
-  constexpr int Q = kOneThreads / N;  // chains per expert
-  __shared__ float part[N];
-  __shared__ float lg[N];
+    int topk_mode, int renorm, FewTokenOut out) {
+  constexpr int Q = kFewThreads / N;  // chains per expert
+  __shared__ float part[T][N];
+  __shared__ float lg[T][N];
   grid_dep_wait();
   grid_dep_launch();
   const uint32_t rank = cluster_rank();
   const int d8 = d / 8;                // 16-byte chunks per row
-  const int cs8 = d8 / kOneCtas;       // chunks per CTA
+  const int cs8 = d8 / kFewCtas;       // chunks per CTA
   const int q = threadIdx.x % Q, e = threadIdx.x / Q;
   const uint4* wr = w + static_cast<int64_t>(e) * d8 + rank * cs8;
   const uint4* xr = x + rank * cs8;
-  float acc = 0.0f;
+  float acc[T];
+#pragma unroll
+  for (int t = 0; t < T; ++t) acc[t] = 0.0f;
 #pragma unroll 4
   for (int u = q; u < cs8; u += Q) {
-    const uint4 wv = __ldg(wr + u), xv = __ldg(xr + u);
-    const uint32_t wa[4] = {wv.x, wv.y, wv.z, wv.w}, xa[4] = {xv.x, xv.y, xv.z, xv.w};
+    const uint4 wv = __ldg(wr + u);
+    const uint32_t wa[4] = {wv.x, wv.y, wv.z, wv.w};
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      acc = fmaf(__uint_as_float(xa[c] << 16), __uint_as_float(wa[c] << 16), acc);
-      acc = fmaf(__uint_as_float(xa[c] & 0xFFFF0000u), __uint_as_float(wa[c] & 0xFFFF0000u), acc);
+    for (int t = 0; t < T; ++t) {
+      const uint4 xv = __ldg(xr + static_cast<int64_t>(t) * d8 + u);
+      const uint32_t xa[4] = {xv.x, xv.y, xv.z, xv.w};
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        acc[t] = fmaf(__uint_as_float(xa[c] << 16), __uint_as_float(wa[c] << 16), acc[t]);
+        acc[t] = fmaf(__uint_as_float(xa[c] & 0xFFFF0000u), __uint_as_float(wa[c] & 0xFFFF0000u),
+                      acc[t]);
+      }
     }
   }
 #pragma unroll
-  for (int o = Q / 2; o >= 1; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-  if (q == 0) part[e] = acc;
+  for (int t = 0; t < T; ++t) {
+#pragma unroll
+    for (int o = Q / 2; o >= 1; o >>= 1) acc[t] += __shfl_xor_sync(0xffffffffu, acc[t], o);
+    if (q == 0) part[t][e] = acc[t];
+  }
   if (rank == 0)
-    for (int i = threadIdx.x; i < out.nclear; i += kOneThreads) out.clear[i] = 0;
+    for (int i = threadIdx.x; i < out.nclear; i += kFewThreads) out.clear[i] = 0;
   cluster_sync();  // every CTA's part[] is written
-  if (rank == 0 && threadIdx.x < N) {
-    const uint32_t a = smem_u32(&part[threadIdx.x]);
-    float l = ld_cluster_f32(map_to_rank(a, 0));
-    for (int r = 1; r < kOneCtas; ++r) l = __fadd_rn(l, ld_cluster_f32(map_to_rank(a, r)));
-    lg[threadIdx.x] = l;
-    if (out.logits) out.logits[threadIdx.x] = l;
+  if (rank == 0) {
+    for (int i = threadIdx.x; i < T * N; i += kFewThreads) {
+      const int t = i / N, ee = i % N;
+      const uint32_t a = smem_u32(&part[t][ee]);
+      float l = ld_cluster_f32(map_to_rank(a, 0));
+      for (int r = 1; r < kFewCtas; ++r) l = __fadd_rn(l, ld_cluster_f32(map_to_rank(a, r)));
+      lg[t][ee] = l;
+      if (out.logits) out.logits[i] = l;
+    }
   }
   cluster_sync();  // CTA 0 is done reading the others' part[]: they may leave
   if (rank != 0) return;
-  if (threadIdx.x < 32)
-    route_one_warp<N>(lg, 0, K, eps, topk_mode, renorm, out.k, out.ids, out.gates);
+  const int wp = threadIdx.x / 32;
+  if (wp < T) route_one_warp<N>(lg[wp], wp, K, eps, topk_mode, renorm, out.k, out.ids, out.gates);
   __syncthreads();  // k and ids are visible to the block
-  const int k1 = min(max(out.k[0], 0), K);
-  for (int ee = threadIdx.x; ee <= N; ee += kOneThreads) {
+  // pair (t, s) is selected iff s < k_t
+  auto kt = [&](int t) { return min(max(out.k[t], 0), K); };
+  for (int ee = threadIdx.x; ee <= N; ee += kFewThreads) {
     int below = 0;
-    for (int s2 = 0; s2 < k1; ++s2) below += out.ids[s2] < ee ? 1 : 0;
+    for (int t = 0; t < T; ++t) {
+      const int k1 = kt(t);
+      for (int s2 = 0; s2 < k1; ++s2) below += out.ids[t * K + s2] < ee ? 1 : 0;
+    }
     out.offsets[ee] = below;
     if (out.offsets_copy) out.offsets_copy[ee] = below;
   }
-  if (threadIdx.x < K) {
-    const int s2 = threadIdx.x;
+  if (threadIdx.x < T * K) {
+    const int t = threadIdx.x / K, s2 = threadIdx.x % K;
     int pos = -1;
-    if (s2 < k1) {
+    if (s2 < kt(t)) {
+      const int id = out.ids[t * K + s2];
       pos = 0;
-      for (int s3 = 0; s3 < k1; ++s3) pos += out.ids[s3] < out.ids[s2] ? 1 : 0;
-      out.perm[pos] = 0;
+      for (int t2 = 0; t2 < T; ++t2) {
+        const int k2 = kt(t2);
+        for (int s3 = 0; s3 < k2; ++s3) {
+          const int id2 = out.ids[t2 * K + s3];
+          pos += (id2 < id || (id2 == id && t2 < t)) ? 1 : 0;
+        }
+      }
+      out.perm[pos] = t;
     }
-    out.pair_pos[s2] = pos;
+    out.pair_pos[threadIdx.x] = pos;
   }
 }
 
@@ -366,25 +394,32 @@ cudaError_t launch_router_small_route(const uint16_t* x, const uint16_t* w_route
                     eps, topk_mode, renorm, logits_out, k_out, ids_out, gates_out);
 }
 
-// Router, routing and dispatch of one token (d a multiple of 64): one cluster
-// of 8 CTAs. Writes logits_out [N] (if not null), k_out [1], ids_out and
-// gates_out [K], offsets [N + 1], perm [K], pair_pos [K] and offsets_copy
-// [N + 1] (if not null), and zeroes clear [nclear] after the previous kernel
-// on the stream has finished.
-cudaError_t launch_router_one(const uint16_t* x, const uint16_t* w_router, int d, int N, int K,
-                              float eps, int topk_mode, int renorm, float* logits_out,
+// Router, routing and dispatch of T <= 4 tokens (d a multiple of 64): one
+// cluster of 8 CTAs. Writes logits_out [T, N] (if not null), k_out [T],
+// ids_out and gates_out [T, K], offsets [N + 1], perm [T K], pair_pos [T, K]
+// and offsets_copy [N + 1] (if not null), and zeroes clear [nclear] after the
+// previous kernel on the stream has finished.
+cudaError_t launch_router_few(const uint16_t* x, const uint16_t* w_router, int T, int d, int N,
+                              int K, float eps, int topk_mode, int renorm, float* logits_out,
                               int32_t* k_out, int32_t* ids_out, float* gates_out, int32_t* offsets,
                               int32_t* perm, int32_t* pair_pos, int32_t* offsets_copy,
                               int32_t* clear, int nclear, cudaStream_t stream) {
-  if (d % (8 * rwarp::kOneCtas) != 0 || (N != 64 && N != 128) || nclear < 0)
+  if (T < 1 || T > rwarp::kFewMaxT || d % (8 * rwarp::kFewCtas) != 0 || (N != 64 && N != 128) ||
+      nclear < 0 || T * K > rwarp::kFewThreads)
     return cudaErrorInvalidValue;
-  const rwarp::OneTokenOut out{logits_out, k_out, ids_out, gates_out, offsets, perm,
+  const rwarp::FewTokenOut out{logits_out, k_out, ids_out, gates_out, offsets, perm,
                                pair_pos, offsets_copy, clear, nclear};
   auto xx = reinterpret_cast<const uint4*>(x);
   auto ww = reinterpret_cast<const uint4*>(w_router);
-  auto kern = N == 64 ? rwarp::router_one_kernel<64> : rwarp::router_one_kernel<128>;
-  return launch_cluster_pdl(kern, dim3(rwarp::kOneCtas), dim3(rwarp::kOneThreads), 0, stream,
-                            rwarp::kOneCtas, xx, ww, d, K, eps, topk_mode, renorm, out);
+  using Kern = void (*)(const uint4*, const uint4*, int, int, float, int, int, rwarp::FewTokenOut);
+  static const Kern kerns[2][rwarp::kFewMaxT] = {
+      {rwarp::router_few_kernel<64, 1>, rwarp::router_few_kernel<64, 2>,
+       rwarp::router_few_kernel<64, 3>, rwarp::router_few_kernel<64, 4>},
+      {rwarp::router_few_kernel<128, 1>, rwarp::router_few_kernel<128, 2>,
+       rwarp::router_few_kernel<128, 3>, rwarp::router_few_kernel<128, 4>}};
+  return launch_cluster_pdl(kerns[N == 128][T - 1], dim3(rwarp::kFewCtas),
+                            dim3(rwarp::kFewThreads), 0, stream, rwarp::kFewCtas, xx, ww, d, K,
+                            eps, topk_mode, renorm, out);
 }
 
 MOE_DEBUG_TU(route_warp)
