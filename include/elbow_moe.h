@@ -126,11 +126,18 @@ moe_status elbow_route_with_counts(const float* logits, int64_t T, int N,
  *                            are the tokens routed to expert e, ascending
  *                            (stable); entries from offsets[N] on are untouched
  *   pair_pos [T, K]   int32  position in perm of pair (t, s), -1 for s >= k_t
- *   ws       device workspace of at least moe_dispatch_workspace_size bytes
+ *   ws       device workspace of at least moe_dispatch_workspace_size bytes,
+ *            256-byte aligned; its first int32 is a device error word
  * A pair whose id lies outside [0, N) is dropped: it is not counted, not in
  * perm, and its pair_pos is -1 (elbow_route never produces such ids). Ids
  * repeated within a token give unspecified positions, but no access outside
  * the arrays above.
+ * moe_dispatch runs batches of more than 128 tokens whose per-block shared
+ * memory fits as one cooperative kernel (each block reads its tokens' selections once,
+ * counts, meets the others at one grid barrier, then places its pairs); that
+ * barrier's wait is bounded, and when it runs out the error word is set and
+ * moe_read_device_error(ws) returns MOE_ERR_DEVICE_TIMEOUT (the outputs are
+ * then incomplete). The word is cleared by each such call.
  */
 /* Bytes of moe_dispatch's workspace; 0 for unsupported sizes (T outside
  * [0, 2^28), N not 64 or 128). */

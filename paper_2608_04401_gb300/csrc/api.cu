@@ -15,7 +15,8 @@ int32_t* dispatch_tile_off(void* ws, int64_t T, int N);
 int32_t* dispatch_counts(void* ws);
 cudaError_t launch_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
                             int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
-                            int32_t* offsets_copy, bool counts_ready, cudaStream_t stream);
+                            int32_t* offsets_copy, bool counts_ready, int32_t* err,
+                            unsigned int* arrive, cudaStream_t stream);
 cudaError_t launch_dispatch_gather(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
                                    int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
                                    int32_t* offsets_copy, const uint16_t* x, int d, uint16_t* xs,
@@ -380,7 +381,8 @@ moe_status moe_dispatch_counted(const int32_t* k, const int32_t* ids, int64_t T,
   if (!aligned4(k) || !aligned4(offsets) || !aligned4(perm) || !aligned4(pair_pos))
     return MOE_ERR_INVALID_ARG;
   return cuda_status(moe::launch_dispatch(k, ids, T, N, K, offsets, perm, pair_pos, ws, nullptr,
-                                          true, static_cast<cudaStream_t>(stream)));
+                                          true, nullptr, nullptr,
+                                          static_cast<cudaStream_t>(stream)));
 }
 
 moe_status moe_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
@@ -396,7 +398,8 @@ moe_status moe_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, 
   if (!aligned4(k) || !aligned4(offsets) || !aligned4(perm) || !aligned4(pair_pos))
     return MOE_ERR_INVALID_ARG;
   return cuda_status(moe::launch_dispatch(k, ids, T, N, K, offsets, perm, pair_pos, ws, nullptr,
-                                          false, static_cast<cudaStream_t>(stream)));
+                                          false, nullptr, nullptr,
+                                          static_cast<cudaStream_t>(stream)));
 }
 
 size_t moe_layer_workspace_size(int64_t T, int d, int N, int I, int K) {
@@ -494,7 +497,7 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
     if (e != cudaSuccess) return MOE_ERR_CUDA;
   } else {
     e = moe::launch_dispatch(kk, ids, T, N, K, w.offsets, w.perm, w.pair_pos, w.disp, offsets_out,
-                             true, s);
+                             true, nullptr, nullptr, s);
     if (e != cudaSuccess) return MOE_ERR_CUDA;
     const int32_t* tile_off = moe::dispatch_tile_off(w.disp, T, N);
     // gate/up GEMM gathers its token rows itself (no dispatched copy of x)

@@ -14,6 +14,7 @@
 //             m-tile prefix sums ceil(count_e / 128) [N+1].
 // A pair whose expert id lies outside [0, N) is dropped by every pass (not
 // counted, not placed, pair_pos -1), so no id indexes outside the arrays.
+#include <atomic>
 #include <mutex>
 
 #include "common.cuh"
@@ -113,6 +114,275 @@ __global__ void __launch_bounds__(kChunk) count_kernel(const int32_t* __restrict
   __syncthreads();
   for (int e = threadIdx.x; e < N; e += kChunk)
     cnt[static_cast<int64_t>(e) * nblk + blockIdx.x] = hist[e];
+}
+
+// ------------------------------------------------ single-pass dispatch
+// The whole dispatch in one cooperative launch of G blocks (all resident),
+// reading each selection once: block b owns the TB tokens [b TB, (b+1) TB)
+// (TB a multiple of 32; unit u = its tokens 32u .. 32u + 31).
+//   1. Each warp loads its units' k and ids (the next unit's loads in flight
+//      while the current one is stored), keeps the ids as bytes (0xFF for
+//      s >= k_t and ids outside [0, N)) and the unit's expert bit masks
+//      mask[u][e] (bit l: token 32u + l selected e; a 32 x 32 transpose of
+//      the tokens' expert masks) in shared memory, then counts its range of
+//      units per expert. The block's per-expert count goes to agg[b][e].
+//   2. One grid barrier (an arrival counter, zero on entry; the wait is
+//      bounded and sets the error word when it runs out).
+//   3. Every block adds the counts of the blocks before it and of all blocks
+//      (its base and the expert totals); block 0 writes offsets, the m-tile
+//      prefix sums and offsets_copy.
+//   4. pair_pos: each warp walks its units in order with per-expert running
+//      positions (in shared memory) and ranks each pair in its unit by the
+//      popcount of the mask bits below its lane; a token's K positions leave
+//      as 16-byte stores.
+//   5. perm: each warp takes whole experts and walks their units 32 at a
+//      time (lane = unit), a warp scan of the units' counts placing each
+//      unit's tokens in ascending order.
+// The result equals the counting sort above: rows by expert, then token.
+constexpr int kCoopThreads = 1024;
+constexpr int kCoopWarps = kCoopThreads / 32;
+
+struct CoopSel {
+  int kt;
+  int id[8];
+};
+
+MOE_DEV CoopSel coop_load(const int32_t* __restrict__ k, const int32_t* __restrict__ ids,
+                          int64_t t, bool valid, int K, bool vec) {
+  CoopSel c;
+  c.kt = valid ? min(max(k[t], 0), K) : 0;
+  MOE_DCHECK(!valid || (k[t] >= 0 && k[t] <= K));
+  if (valid && vec) {
+    const int4 a = __ldg(reinterpret_cast<const int4*>(ids + t * 8));
+    const int4 b = __ldg(reinterpret_cast<const int4*>(ids + t * 8) + 1);
+    c.id[0] = a.x; c.id[1] = a.y; c.id[2] = a.z; c.id[3] = a.w;
+    c.id[4] = b.x; c.id[5] = b.y; c.id[6] = b.z; c.id[7] = b.w;
+  } else {
+#pragma unroll
+    for (int s = 0; s < 8; ++s) c.id[s] = (valid && s < K) ? __ldg(ids + t * K + s) : 0;
+  }
+  return c;
+}
+
+template <int N>
+__global__ void __launch_bounds__(kCoopThreads, 1) dispatch_coop_kernel(
+    const int32_t* __restrict__ k, const int32_t* __restrict__ ids, int64_t T, int K, int TB,
+    int32_t* agg, unsigned int* arrive, int32_t* err, int32_t* __restrict__ perm,
+    int32_t* __restrict__ pair_pos, int32_t* __restrict__ offsets, int32_t* __restrict__ tile_off,
+    int32_t* __restrict__ offsets_copy) {
+  constexpr int C = N / 32;      // mask words per unit (lane l: experts l + 32c)
+  constexpr int kPitch = N + 1;  // mask row pitch (odd: lane-per-unit reads hit distinct banks)
+  extern __shared__ __align__(16) uint8_t smem[];
+  uint2* ids8 = reinterpret_cast<uint2*>(smem);                       // [TB] 8 id bytes
+  uint32_t* mask = reinterpret_cast<uint32_t*>(smem + static_cast<size_t>(TB) * 8);  // [U][kPitch]
+  __shared__ int rc[kCoopWarps][N];  // per warp range: count, then global start per expert
+  __shared__ int s_base[N], s_tot[N], s_off[N], s_gbase[N];
+  __shared__ int s_part[kCoopThreads / N][N];
+  __shared__ int s_ok;
+  grid_dep_wait();
+  grid_dep_launch();
+  const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+  const int G = static_cast<int>(gridDim.x), b = static_cast<int>(blockIdx.x);
+  const int64_t t0 = static_cast<int64_t>(b) * TB;
+  const int U = TB / 32;
+  const int UR = (U + kCoopWarps - 1) / kCoopWarps;  // units per warp range
+  const int u0 = min(U, warp * UR), u1 = min(U, u0 + UR);
+  const bool vec = K == 8 && (reinterpret_cast<uintptr_t>(ids) & 15u) == 0;
+  const uint32_t lt_mask = (1u << lane) - 1u;
+
+  // 1. selections -> id bytes and unit masks (each warp its own range of units)
+  {
+    int64_t t = t0 + static_cast<int64_t>(u0) * 32 + lane;
+    CoopSel cur = coop_load(k, ids, t, u0 < u1 && t < T, K, vec);
+    for (int u = u0; u < u1; ++u) {
+      const int64_t tn = t + 32;
+      const CoopSel nxt = coop_load(k, ids, tn, u + 1 < u1 && tn < T, K, vec);
+      uint32_t lo = 0, hi = 0;
+      uint64_t m0 = 0, m1 = 0;
+#pragma unroll
+      for (int s = 0; s < 8; ++s) {
+        const bool ok = s < cur.kt && static_cast<unsigned>(cur.id[s]) < static_cast<unsigned>(N);
+        MOE_DCHECK(s >= cur.kt || static_cast<unsigned>(cur.id[s]) < static_cast<unsigned>(N));
+        const uint32_t byte = ok ? static_cast<uint32_t>(cur.id[s]) : 0xFFu;
+        if (s < 4) lo |= byte << (8 * s);
+        else hi |= byte << (8 * (s - 4));
+        if (ok) {
+          if (cur.id[s] < 64) m0 |= 1ull << cur.id[s];
+          else m1 |= 1ull << (cur.id[s] - 64);
+        }
+      }
+      ids8[u * 32 + lane] = make_uint2(lo, hi);
+#pragma unroll
+      for (int c = 0; c < C; ++c)
+        mask[u * kPitch + 32 * c + lane] = transpose32(mask_word(c, m0, m1), lane);
+      cur = nxt;
+      t = tn;
+    }
+    __syncwarp();
+    // the range's count per expert
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      int n = 0;
+      for (int u = u0; u < u1; ++u) n += __popc(mask[u * kPitch + 32 * c + lane]);
+      rc[warp][32 * c + lane] = n;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x < N) {
+    const int e = threadIdx.x;
+    int run = 0;
+    for (int w = 0; w < kCoopWarps; ++w) {
+      const int n = rc[w][e];
+      rc[w][e] = run;  // exclusive within the block, for now
+      run += n;
+    }
+    agg[static_cast<int64_t>(b) * N + e] = run;
+  }
+  // 2. grid barrier: the block's counts (the barrier) before thread 0's release
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(arrive) : "memory");
+    const uint64_t w0 = global_timer_ns();
+    bool ok = true;
+    for (uint32_t spins = 1;; ++spins) {
+      unsigned int v;
+      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(arrive) : "memory");
+      if (v >= static_cast<unsigned int>(G)) break;
+      if (spins % 64u == 0u && global_timer_ns() - w0 > kWaitLimitNs) {
+        ok = false;
+        break;
+      }
+      __nanosleep(64);
+    }
+    if (!ok && err) atomicExch(err, kDevErrTimeout);
+    s_ok = ok ? 1 : 0;
+  }
+  __syncthreads();
+  if (!s_ok) return;
+  // 3. this block's base and the expert totals
+  {
+    constexpr int kParts = kCoopThreads / N;
+    const int e = threadIdx.x % N, part = threadIdx.x / N;
+    int below = 0, tot = 0;
+    for (int bb = part; bb < G; bb += kParts) {
+      const int v = __ldcg(agg + static_cast<int64_t>(bb) * N + e);
+      tot += v;
+      below += bb < b ? v : 0;
+    }
+    s_part[part][e] = below;
+    __syncthreads();
+    if (part == 0) {
+      int sb = below;
+      for (int pp = 1; pp < kParts; ++pp) sb += s_part[pp][e];
+      s_base[e] = sb;
+    }
+    __syncthreads();
+    s_part[part][e] = tot;
+    __syncthreads();
+    if (part == 0) {
+      int st = tot;
+      for (int pp = 1; pp < kParts; ++pp) st += s_part[pp][e];
+      s_tot[e] = st;
+    }
+    __syncthreads();
+  }
+  if (warp == 0) {  // exclusive scans over the experts: offsets and m-tile counts
+    int run = 0, trun = 0;
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      const int e = 32 * c + lane;
+      const int v = s_tot[e], tv = (v + 127) / 128;
+      int x = v, tx = tv;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o), ty = __shfl_up_sync(0xffffffffu, tx, o);
+        if (lane >= o) {
+          x += y;
+          tx += ty;
+        }
+      }
+      const int off = run + x - v, toff = trun + tx - tv;
+      s_off[e] = off;
+      s_gbase[e] = off + s_base[e];
+      if (b == 0) {
+        offsets[e] = off;
+        tile_off[e] = toff;
+        if (offsets_copy) offsets_copy[e] = off;
+      }
+      run += __shfl_sync(0xffffffffu, x, 31);
+      trun += __shfl_sync(0xffffffffu, tx, 31);
+    }
+    if (b == 0 && lane == 0) {
+      MOE_DCHECK(static_cast<int64_t>(run) <= T * K);
+      offsets[N] = run;
+      tile_off[N] = trun;
+      if (offsets_copy) offsets_copy[N] = run;
+    }
+  }
+  __syncthreads();
+  // 4. pair_pos, each warp over its units in order; rc[warp][e] becomes the
+  // running position of expert e (global)
+#pragma unroll
+  for (int c = 0; c < C; ++c) rc[warp][32 * c + lane] += s_gbase[32 * c + lane];
+  __syncwarp();
+  {
+    int* run = rc[warp];
+    for (int u = u0; u < u1; ++u) {
+      const int64_t t = t0 + static_cast<int64_t>(u) * 32 + lane;
+      const uint2 w8 = ids8[u * 32 + lane];
+      const uint32_t* mrow = mask + u * kPitch;
+      int pp[8];
+#pragma unroll
+      for (int s = 0; s < 8; ++s) {
+        const uint32_t byte = __byte_perm(s < 4 ? w8.x : w8.y, 0u, 0x4440u | (s & 3));
+        const int e = static_cast<int>(byte & (N - 1));  // 0xFF: an in-range index, unused
+        const int v = run[e] + __popc(mrow[e] & lt_mask);
+        pp[s] = byte == 0xFFu ? -1 : v;
+      }
+      __syncwarp();
+#pragma unroll
+      for (int c = 0; c < C; ++c) run[32 * c + lane] += __popc(mrow[32 * c + lane]);
+      __syncwarp();
+      if (t < T) {
+        int32_t* dst = pair_pos + t * K;
+        if (K == 8 && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
+          reinterpret_cast<int4*>(dst)[0] = make_int4(pp[0], pp[1], pp[2], pp[3]);
+          reinterpret_cast<int4*>(dst)[1] = make_int4(pp[4], pp[5], pp[6], pp[7]);
+        } else {
+#pragma unroll
+          for (int s = 0; s < 8; ++s)
+            if (s < K) dst[s] = pp[s];
+        }
+      }
+    }
+  }
+  // 5. perm, each warp over whole experts (units 32 at a time, lane = unit):
+  // a warp scan of the units' counts places each unit's tokens in ascending
+  // order (consecutive lanes write neighbouring runs). A unit holds at most K
+  // bits per token and only ids below N, so the block's positions stay below
+  // the total pair count <= T K: no store leaves perm.
+  for (int e = warp; e < N; e += kCoopWarps) {
+    int run = s_gbase[e];
+    for (int ub = 0; ub < U; ub += 32) {
+      const int u = ub + lane;
+      uint32_t m = u < U ? mask[u * kPitch + e] : 0u;
+      const int c = __popc(m);
+      int x = c;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+      }
+      MOE_DCHECK(m == 0u || (run + x - c >= 0 && static_cast<int64_t>(run + x) <= T * K));
+      int32_t* dst = perm + (run + x - c);
+      const int32_t tu = static_cast<int32_t>(t0) + u * 32;
+      while (m) {
+        *dst++ = tu + (__ffs(static_cast<int>(m)) - 1);
+        m &= m - 1u;
+      }
+      run += __shfl_sync(0xffffffffu, x, 31);
+    }
+  }
 }
 
 // Block e: exclusive prefix sum of cnt[e][0 .. nblk) in place; total -> totals[e].
@@ -281,20 +551,33 @@ __global__ void __launch_bounds__(kChunk) scatter_kernel(
   __syncthreads();
   if (valid) {
     const uint32_t lt_mask = (1u << lane) - 1u;
+    int pp[8];
 #pragma unroll
     for (int s = 0; s < 8; ++s) {
-      if (s < K) {
-        if (s < kt && static_cast<unsigned>(my[s]) < static_cast<unsigned>(N)) {
-          const int e = my[s];
-          const int below = __popc(bal[warp][e] & lt_mask);
-          const int pos = wbase[warp][e] + below;
-          const int lpos = lbase[warp][e] + below;
-          s_tok[lpos] = static_cast<int32_t>(t);
-          s_gpos[lpos] = pos;
-          if (writer) pair_pos[t * K + s] = pos;
-        } else if (writer) {
-          pair_pos[t * K + s] = -1;
-        }
+      pp[s] = -1;
+      if (s < kt && static_cast<unsigned>(my[s]) < static_cast<unsigned>(N)) {
+        const int e = my[s];
+        const int below = __popc(bal[warp][e] & lt_mask);
+        const int pos = wbase[warp][e] + below;
+        const int lpos = lbase[warp][e] + below;
+        s_tok[lpos] = static_cast<int32_t>(t);
+        s_gpos[lpos] = pos;
+        pp[s] = pos;
+      }
+    }
+    if (writer) {
+      // the token's K positions are contiguous: whole 16-byte stores where
+      // they fit (one store per pair would touch a sector per lane)
+      int32_t* dst = pair_pos + t * K;
+      if (K == 8 && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
+        reinterpret_cast<int4*>(dst)[0] = make_int4(pp[0], pp[1], pp[2], pp[3]);
+        reinterpret_cast<int4*>(dst)[1] = make_int4(pp[4], pp[5], pp[6], pp[7]);
+      } else if (K == 4 && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
+        reinterpret_cast<int4*>(dst)[0] = make_int4(pp[0], pp[1], pp[2], pp[3]);
+      } else {
+#pragma unroll
+        for (int s = 0; s < 8; ++s)
+          if (s < K) dst[s] = pp[s];
       }
     }
   }
@@ -518,19 +801,27 @@ MOE_DEBUG_TU(dispatch)
 
 static int num_chunks(int64_t T) { return static_cast<int>((T + disp::kChunk - 1) / disp::kChunk); }
 
-// Workspace layout: cnt/base [N][nchunks] int32 | totals [N] | tile_off [N+1]
+// Workspace layout: header (256 bytes: error word, the single-pass
+// dispatch's barrier counter) | cnt/base [N][nchunks] int32 (the single-pass
+// dispatch's per-block counts [G][N], G <= nchunks) | totals [N] | tile_off [N+1]
+constexpr size_t kWsHeader = 256;
+
 size_t dispatch_ws_bytes(int64_t T, int N) {
   auto up = [](size_t b) { return (b + 255) & ~static_cast<size_t>(255); };
   const size_t nblk = static_cast<size_t>(num_chunks(T) > 0 ? num_chunks(T) : 1);
-  return up(nblk * N * sizeof(int32_t)) + up(N * sizeof(int32_t)) + up((N + 1) * sizeof(int32_t));
+  return kWsHeader + up(nblk * N * sizeof(int32_t)) + up(N * sizeof(int32_t)) +
+         up((N + 1) * sizeof(int32_t));
 }
 
-int32_t* dispatch_counts(void* ws) { return static_cast<int32_t*>(ws); }
+int32_t* dispatch_counts(void* ws) {
+  return reinterpret_cast<int32_t*>(static_cast<char*>(ws) + kWsHeader);
+}
 
 static int32_t* dispatch_totals(void* ws, int64_t T, int N) {
   auto up = [](size_t b) { return (b + 255) & ~static_cast<size_t>(255); };
   const size_t nblk = static_cast<size_t>(num_chunks(T) > 0 ? num_chunks(T) : 1);
-  return reinterpret_cast<int32_t*>(static_cast<char*>(ws) + up(nblk * N * sizeof(int32_t)));
+  return reinterpret_cast<int32_t*>(reinterpret_cast<char*>(dispatch_counts(ws)) +
+                                    up(nblk * N * sizeof(int32_t)));
 }
 
 int32_t* dispatch_tile_off(void* ws, int64_t T, int N) {
@@ -539,12 +830,85 @@ int32_t* dispatch_tile_off(void* ws, int64_t T, int N) {
                                     up(N * sizeof(int32_t)));
 }
 
-// counts_ready: the elbow router already wrote the per-chunk counts into
-// dispatch_counts(ws).
+// The single-pass dispatch's shape: G blocks of TB tokens and the dynamic
+// shared memory of one block; false when it does not fit (one block per SM,
+// at most kCoopMaxSmem bytes) or the batch is too small to need it.
+constexpr size_t kCoopMaxSmem = 200 * 1024;
+
+static bool coop_shape(int64_t T, int N, int num_sms, int& G, int& TB, size_t& smem) {
+  if (T <= disp::kChunk || num_sms <= 0) return false;
+  const int64_t nblk = num_chunks(T);  // the counts region holds nblk x N ints
+  int64_t g = num_sms < nblk ? num_sms : nblk;
+  int64_t tb = ((T + g - 1) / g + 31) / 32 * 32;
+  g = (T + tb - 1) / tb;
+  smem = static_cast<size_t>(tb) * 8 + static_cast<size_t>(tb / 32) * (N + 1) * sizeof(uint32_t);
+  if (smem > kCoopMaxSmem) return false;
+  G = static_cast<int>(g);
+  TB = static_cast<int>(tb);
+  return true;
+}
+
+// The single-pass dispatch (see dispatch_coop_kernel). arrive: a zeroed
+// counter; err: the word a barrier timeout sets.
+static cudaError_t launch_dispatch_coop(const int32_t* k, const int32_t* ids, int64_t T, int N,
+                                        int K, int G, int TB, size_t smem, int32_t* agg,
+                                        unsigned int* arrive, int32_t* err, int32_t* perm,
+                                        int32_t* pair_pos, int32_t* offsets, int32_t* tile_off,
+                                        int32_t* offsets_copy, cudaStream_t stream) {
+  using Kern = void (*)(const int32_t*, const int32_t*, int64_t, int, int, int32_t*, unsigned int*,
+                        int32_t*, int32_t*, int32_t*, int32_t*, int32_t*, int32_t*);
+  const Kern kern = N == 64 ? disp::dispatch_coop_kernel<64> : disp::dispatch_coop_kernel<128>;
+  static std::atomic<uint64_t> attr_done{0};
+  const cudaError_t e = once_per_device(attr_done, [] {
+    for (Kern f : {disp::dispatch_coop_kernel<64>, disp::dispatch_coop_kernel<128>}) {
+      const cudaError_t r = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 static_cast<int>(kCoopMaxSmem));
+      if (r != cudaSuccess) return r;
+    }
+    return cudaSuccess;
+  });
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(G));
+  cfg.blockDim = dim3(disp::kCoopThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, kern, k, ids, T, K, TB, agg, arrive, err, perm, pair_pos, offsets,
+                            tile_off, offsets_copy);
+}
+
+// SM count of the current device (cached per device ordinal below 64).
+static int sm_count_cached() {
+  static std::atomic<int> cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (dev >= 0 && dev < 64) {
+    const int c = cache[dev].load(std::memory_order_relaxed);
+    if (c > 0) return c;
+  }
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  if (dev >= 0 && dev < 64) cache[dev].store(n, std::memory_order_relaxed);
+  return n;
+}
+
+// counts_ready: the elbow router already wrote the per-chunk counts into cnt
+// (then the scan and scatter passes run: faster than the single pass, which
+// would count again). Otherwise arrive, a zeroed counter, enables the
+// single-pass dispatch (err: the word its barrier timeout sets); nullptr
+// gives the count / scan / scatter passes.
 static cudaError_t run_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
                                 int32_t* offsets, int32_t* perm, int32_t* pair_pos, int32_t* cnt,
                                 int32_t* totals, int32_t* tile_off, int32_t* offsets_copy,
-                                bool counts_ready, cudaStream_t stream) {
+                                bool counts_ready, int32_t* err, unsigned int* arrive,
+                                cudaStream_t stream) {
   const int nblk = num_chunks(T);
   const uint4* no_x = nullptr;
   uint4* no_xs = nullptr;
@@ -554,6 +918,12 @@ static cudaError_t run_dispatch(const int32_t* k, const int32_t* ids, int64_t T,
                       perm, pair_pos, offsets, tile_off, offsets_copy, no_x, 0, no_xs);
   }
   cudaError_t e;
+  int G = 0, TB = 0;
+  size_t smem = 0;
+  if (arrive && !counts_ready && coop_shape(T, N, sm_count_cached(), G, TB, smem)) {
+    return launch_dispatch_coop(k, ids, T, N, K, G, TB, smem, cnt, arrive, err, perm, pair_pos,
+                                offsets, tile_off, offsets_copy, stream);
+  }
   if (nblk > 0 && !counts_ready) {
     auto kern = N == 64 ? disp::count_kernel<64> : disp::count_kernel<128>;
     e = launch_pdl(kern, dim3(nblk), dim3(disp::kChunk), 0, stream, k, ids, T, K, nblk, cnt);
@@ -571,12 +941,25 @@ static cudaError_t run_dispatch(const int32_t* k, const int32_t* ids, int64_t T,
                     perm, pair_pos, offsets, tile_off, offsets_copy, no_x, 0, no_xs);
 }
 
+// err / arrive: the error word and a zeroed counter for the single-pass
+// dispatch, or nullptr to use the workspace header's two words, which are
+// cleared here when the single-pass dispatch runs.
 cudaError_t launch_dispatch(const int32_t* k, const int32_t* ids, int64_t T, int N, int K,
                             int32_t* offsets, int32_t* perm, int32_t* pair_pos, void* ws,
-                            int32_t* offsets_copy, bool counts_ready, cudaStream_t stream) {
+                            int32_t* offsets_copy, bool counts_ready, int32_t* err,
+                            unsigned int* arrive, cudaStream_t stream) {
+  int G = 0, TB = 0;
+  size_t smem = 0;
+  if (!arrive && !counts_ready && num_chunks(T) > 1 &&
+      coop_shape(T, N, sm_count_cached(), G, TB, smem)) {
+    err = static_cast<int32_t*>(ws);
+    arrive = reinterpret_cast<unsigned int*>(err + 1);
+    const cudaError_t e = cudaMemsetAsync(ws, 0, 2 * sizeof(int32_t), stream);
+    if (e != cudaSuccess) return e;
+  }
   return run_dispatch(k, ids, T, N, K, offsets, perm, pair_pos, dispatch_counts(ws),
                       dispatch_totals(ws, T, N), dispatch_tile_off(ws, T, N), offsets_copy,
-                      counts_ready, stream);
+                      counts_ready, err, arrive, stream);
 }
 
 // Single-chunk dispatch (T <= 128) fused with the row gather xs[r] = x[perm[r]].
@@ -716,7 +1099,7 @@ extern "C" moe_status moe_dispatch_noalloc(const int32_t* k, const int32_t* ids,
   int32_t* totals = scratch + kNoAllocChunks * kNoAllocMaxExperts;
   int32_t* tile_off = totals + kNoAllocMaxExperts;
   return moe::run_dispatch(k, ids, T, N, K, offsets, perm, pair_pos, cnt, totals, tile_off, nullptr,
-                           false, static_cast<cudaStream_t>(stream)) == cudaSuccess
+                           false, nullptr, nullptr, static_cast<cudaStream_t>(stream)) == cudaSuccess
              ? MOE_OK
              : MOE_ERR_CUDA;
 }

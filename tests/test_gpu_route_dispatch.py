@@ -237,6 +237,17 @@ def test_dispatch_edges(moe):
     assert np.all(off.cpu().numpy() == 0)
 
 
+@pytest.mark.parametrize("N,T,K", [(64, 150001, 8), (128, 300007, 8), (128, 99999, 5),
+                                   (64, 1000003, 3)])
+def test_dispatch_single_pass_ranges(moe, N, T, K):
+    """The single-pass dispatch with several 32-token units per warp (running
+    positions carried from unit to unit), ragged last block, both N and
+    K < 8 (element loads and stores)."""
+    rng = np.random.default_rng(T + N + K)
+    r = oracle.route(synth.boosted_logits(rng, T, N), K=K)
+    _dispatch_both(moe, r["k"], r["ids"], N)
+
+
 def test_dispatch_full_stress(moe):
     w = synth.WORKLOADS["route_t1m"]
     rng = np.random.Generator(np.random.PCG64(w["seed"] + 1))
