@@ -87,19 +87,23 @@ def test_layer_gemv_sizes(moe, T, mode, N):
     assert_layer_close(bf16_tensor_to_f64(y), ref["y"])
 
 
-@pytest.mark.parametrize("d,I,N,mode,K,res", [(256, 2048, 64, 0, 8, False),
-                                              (4096, 256, 128, 1, 8, True),
-                                              (384, 384, 64, 1, 3, True),
-                                              (1024, 4096, 128, 0, 1, False)])
-def test_layer_one_token_shapes(moe, d, I, N, mode, K, res):
-    """One-token layers of other shapes (down items of 16 to 64 columns, one to
-    eight experts, with a residual): y against the oracle, routing bit-exact on
-    the layer's own logits, and the device error word clean."""
+@pytest.mark.parametrize("T,d,I,N,mode,K,res", [(1, 256, 2048, 64, 0, 8, False),
+                                                (1, 4096, 256, 128, 1, 8, True),
+                                                (1, 384, 384, 64, 1, 3, True),
+                                                (1, 1024, 4096, 128, 0, 1, False),
+                                                (2, 4096, 1536, 128, 0, 8, True),
+                                                (2, 512, 256, 64, 1, 5, False),
+                                                (2, 2048, 1024, 128, 1, 8, False)])
+def test_layer_few_token_shapes(moe, T, d, I, N, mode, K, res):
+    """Layers of one and two tokens on other shapes (down items of 16 to 64
+    columns, one to sixteen experts, two rows for experts both tokens chose,
+    with a residual): y against the oracle, routing bit-exact on the layer's
+    own logits, and the device error word clean."""
     import torch
-    inp = synth.layer_inputs(T=1, d=d, N=N, I=I, seed=900 + d + I + K)
+    inp = synth.layer_inputs(T=T, d=d, N=N, I=I, seed=900 + T + d + I + K)
     x = to_dev_bf16(inp["x"])
-    resid = synth.bf16_bits(np.random.default_rng(d + I).standard_normal((1, d)).astype(np.float32))
-    ws = torch.empty(moe.layer_workspace_size(1, d, N, I, K), dtype=torch.uint8, device="cuda")
+    resid = synth.bf16_bits(np.random.default_rng(d + I).standard_normal((T, d)).astype(np.float32))
+    ws = torch.empty(moe.layer_workspace_size(T, d, N, I, K), dtype=torch.uint8, device="cuda")
     y, it = moe.moe_layer_forward(x, to_dev_bf16(inp["w_router"]), to_dev_bf16(inp["w_gate_up"]),
                                   to_dev_bf16(inp["w_down"]), K=K, mode=mode, ws=ws,
                                   residual=to_dev_bf16(resid) if res else None,
@@ -109,7 +113,7 @@ def test_layer_one_token_shapes(moe, d, I, N, mode, K, res):
     assert np.array_equal(r["k"], it["k"].cpu().numpy())
     assert np.array_equal(r["ids"], it["ids"].cpu().numpy())
     ref = oracle.layer_rows(inp["x"], inp["w_router"], inp["w_gate_up"], inp["w_down"],
-                            rows=np.arange(1), K=K, mode=mode,
+                            rows=np.arange(T), K=K, mode=mode,
                             residual_bits=resid if res else None)
     assert np.array_equal(ref["k"], r["k"]) and np.array_equal(ref["ids"], r["ids"])
     assert_layer_close(bf16_tensor_to_f64(y), ref["y"])
