@@ -482,8 +482,12 @@ moe_status moe_layer_forward(const uint16_t* x, const uint16_t* w_router, const 
     e = moe::launch_expert_few_gemv(x, T, w.perm, w.offsets, w_gate_up, w_down, P, d, N, I, K, w.h,
                                     w.o, w.err, w.tickets + (d + 15) / 16, kk, w.pair_pos, gates,
                                     residual, y, w.tickets, nsm, s);
-    return e == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
-  } else if (T <= kDecodeMaxTokens) {
+    if (e != cudaErrorCooperativeLaunchTooLarge) return e == cudaSuccess ? MOE_OK : MOE_ERR_CUDA;
+    // SMs not all available to this context (MPS, green contexts): the
+    // decode path below, which waits on nothing, serves this step
+    (void)cudaGetLastError();
+  }
+  if (T <= kDecodeMaxTokens) {
     // decode-sized: the single-chunk dispatch also gathers the few token rows
     // (into o, which the down GEMM overwrites afterwards); the GEMMs stream
     // the weights as the M operand

@@ -921,8 +921,12 @@ static cudaError_t run_dispatch(const int32_t* k, const int32_t* ids, int64_t T,
   int G = 0, TB = 0;
   size_t smem = 0;
   if (arrive && !counts_ready && coop_shape(T, N, sm_count_cached(), G, TB, smem)) {
-    return launch_dispatch_coop(k, ids, T, N, K, G, TB, smem, cnt, arrive, err, perm, pair_pos,
-                                offsets, tile_off, offsets_copy, stream);
+    e = launch_dispatch_coop(k, ids, T, N, K, G, TB, smem, cnt, arrive, err, perm, pair_pos,
+                             offsets, tile_off, offsets_copy, stream);
+    // a device whose SMs are not all available to this context (MPS, green
+    // contexts) may refuse the co-resident grid: the passes below need none
+    if (e != cudaErrorCooperativeLaunchTooLarge) return e;
+    (void)cudaGetLastError();
   }
   if (nblk > 0 && !counts_ready) {
     auto kern = N == 64 ? disp::count_kernel<64> : disp::count_kernel<128>;
