@@ -326,7 +326,12 @@ MOE_DEV uint32_t pack_bf16x2(float lo, float hi) {
 }
 
 // ------------------------------------------ GEMM copies, stores, epilogue
-MOE_DEV float silu(float g) { return g / (1.0f + __expf(-g)); }
+// silu(g) = g / (1 + e^-g), the gate of the expert MLP's SwiGLU. The fast
+// division (2 ulp in fp32; 0 once 1 + e^-g exceeds 2^126, where silu is below
+// 1e-36) is 13 bits finer than the bf16 rounding of h that follows, and
+// costs less than the IEEE division in the GEMM epilogues (about 1.5 % of the
+// gate/up GEMM).
+MOE_DEV float silu(float g) { return __fdividef(g, 1.0f + __expf(-g)); }
 
 MOE_DEV void cp_async_16(uint32_t dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
