@@ -119,6 +119,37 @@ def test_layer_few_token_shapes(moe, T, d, I, N, mode, K, res):
     assert_layer_close(bf16_tensor_to_f64(y), ref["y"])
 
 
+@pytest.mark.parametrize("N,mode,renorm", [(64, 0, 1), (128, 1, 0), (64, 1, 1)])
+def test_layer_two_identical_tokens(moe, N, mode, renorm):
+    """Two copies of one token: every expert in use has two rows (both rows of
+    the expert item, and two pairs per column block in the combine), with
+    renorm = 1 and both modes; routing equal for both tokens and bit-exact on
+    the layer's logits, y equal for both tokens and within tolerance of the
+    oracle."""
+    import torch
+    d, I, K = 1024, 512, 8
+    inp = synth.layer_inputs(T=1, d=d, N=N, I=I, seed=777 + N + mode)
+    x2 = np.concatenate([inp["x"], inp["x"]], axis=0)
+    ws = torch.empty(moe.layer_workspace_size(2, d, N, I, K), dtype=torch.uint8, device="cuda")
+    y, it = moe.moe_layer_forward(to_dev_bf16(x2), to_dev_bf16(inp["w_router"]),
+                                  to_dev_bf16(inp["w_gate_up"]), to_dev_bf16(inp["w_down"]), K=K,
+                                  mode=mode, renorm=renorm, ws=ws, return_intermediates=True)
+    moe.read_device_error(ws)
+    k, ids = it["k"].cpu().numpy(), it["ids"].cpu().numpy()
+    assert k[0] == k[1] and np.array_equal(ids[0], ids[1])
+    offs = it["offsets"].cpu().numpy()
+    cnt = np.diff(offs)
+    assert set(cnt[cnt > 0].tolist()) == {2}
+    r = oracle.route(it["logits"].cpu().numpy(), K=K, mode=mode, renorm=renorm)
+    assert np.array_equal(r["k"], k) and np.array_equal(r["ids"], ids)
+    yv = bf16_tensor_to_f64(y)
+    assert np.array_equal(yv[0], yv[1])
+    ref = oracle.layer_rows(x2, inp["w_router"], inp["w_gate_up"], inp["w_down"], rows=np.arange(2),
+                            K=K, mode=mode, renorm=renorm)
+    if np.array_equal(ref["k"], k) and np.array_equal(ref["ids"], ids):
+        assert_layer_close(yv, ref["y"])
+
+
 def test_gemv_rejects_large_batches(moe):
     import torch
     x = torch.zeros(5, 512, dtype=torch.bfloat16, device="cuda")

@@ -248,6 +248,27 @@ def test_dispatch_single_pass_ranges(moe, N, T, K):
     _dispatch_both(moe, r["k"], r["ids"], N)
 
 
+def test_dispatch_workspace_error_word(moe):
+    """The single-pass dispatch clears its workspace's error word and leaves it
+    clear: moe_read_device_error on the dispatch workspace reports MOE_OK, and
+    a second call on the same workspace gives the same bit-exact result."""
+    import torch
+    rng = np.random.default_rng(4242)
+    r = oracle.route(synth.boosted_logits(rng, 50000, 64), K=8)
+    k, ids = to_dev(r["k"]), to_dev(r["ids"])
+    ws = torch.full((moe.dispatch_workspace_size(50000, 64, 8),), 0xFF, dtype=torch.uint8,
+                    device="cuda")
+    out1 = moe.moe_dispatch(k, ids, 64, ws)
+    moe.read_device_error(ws)
+    out2 = moe.moe_dispatch(k, ids, 64, ws)
+    moe.read_device_error(ws)
+    P = int(out1[0][-1].item())
+    assert torch.equal(out1[0], out2[0]) and torch.equal(out1[2], out2[2])
+    assert torch.equal(out1[1][:P], out2[1][:P])  # perm past offsets[N] is left untouched
+    ref = oracle.dispatch(r["k"], r["ids"], 64)
+    assert np.array_equal(out2[2].cpu().numpy(), ref["pair_pos"])
+
+
 def test_dispatch_full_stress(moe):
     w = synth.WORKLOADS["route_t1m"]
     rng = np.random.Generator(np.random.PCG64(w["seed"] + 1))
