@@ -101,7 +101,8 @@ moe_status elbow_route(const float* logits, int64_t T, int N, const moe_route_pa
  * as elbow_route; a much shorter critical path per token, at about three
  * times the instructions per token, so elbow_route uses it by itself for
  * T <= 16 (and moe_layer_forward's router, after a router GEMM split over d
- * and 16-token groups, for T <= 64). Arguments and errors as elbow_route
+ * and 16-token groups, for 3 <= T <= 64; for T <= 2 one cluster of CTAs computes
+ * the logits and routes each token with one warp). Arguments and errors as elbow_route
  * (ids_out and gates_out need only 4-byte alignment). */
 moe_status elbow_route_warp(const float* logits, int64_t T, int N, const moe_route_params* rp,
                             int32_t* k_out, int32_t* ids_out, float* gates_out, void* stream);
@@ -179,7 +180,8 @@ moe_status moe_dispatch_noalloc(const int32_t* k, const int32_t* ids, int64_t T,
  * App. A.4): router logits l = W_r x (bf16 x bf16, fp32 accumulate), routing
  * as elbow_route, dispatch as moe_dispatch, per-expert SwiGLU
  *   h = silu(W_gate[e] x) * (W_up[e] x)   (bf16 tensor cores, fp32 accumulate,
- *                                          h stored as bf16)
+ *                                          h stored as bf16; CUDA cores with fp32
+ *                                          accumulation for T <= 2)
  *   o = W_down[e] h                       (stored as bf16)
  * and the combine y_t = sum_{s < k_t} g_{t,s} o_{t,s} (+ residual_t), summed
  * in s order in fp32 and rounded to bf16.
@@ -275,7 +277,7 @@ moe_status moe_expert_down(const uint16_t* h, const uint16_t* w_down, const int3
  * weights as the M operand (128 weight rows per tile, the expert's rows as N,
  * in a 16-, 32- or 64-column tile for T <= 16, <= 32, <= 64), so a tile
  * streams weights instead of a mostly empty 128-row token block.
- * moe_layer_forward takes this path by itself when T <= 64. T is the token
+ * moe_layer_forward takes this path by itself when 3 <= T <= 64. T is the token
  * count the rows came from (T > 64: MOE_ERR_UNSUPPORTED; rows of an expert
  * past T are not computed); xs [P, d] holds the dispatched rows
  * (moe_gather_rows), offsets [N + 1] the expert row offsets. I a multiple of
@@ -288,9 +290,10 @@ moe_status moe_expert_down_decode(const uint16_t* h, const uint16_t* w_down, con
                                   int32_t* err_word, void* stream);
 
 /* The expert contractions for batches of T <= 4 tokens (the expert MLP of
- * App. A.4 in the one-token latency regime of Sec. 3) on CUDA cores, which
- * moe_layer_forward takes by itself for one-token steps (T = 1, d, I <= 4096;
- * from two tokens on the tensor-core decode tiles are faster): an expert then
+ * App. A.4 in the one-token latency regime of Sec. 3) on CUDA cores.
+ * moe_layer_forward runs the same items, both contractions and the combine,
+ * in one cooperative kernel for steps of T <= 2 tokens (d, I <= 4096; from
+ * three tokens on the tensor-core decode tiles are faster): an expert then
  * has at most T rows, so its contraction is a few matrix-vector products that
  * spread the expert's weight rows over many blocks. The same results as
  * moe_expert_gate_up / moe_expert_down within fp32 accumulation (another
